@@ -1,0 +1,13 @@
+"""CPU oracle of the LC-VQ linear layer (LC-QAT, arxiv 2606.10531).
+
+TEST INFRASTRUCTURE ONLY. Only tests/, __graft_entry__.smoke() and bench.py's
+CPU-baseline / reference legs may import this package. The GPU library never
+imports it and shares no code with it.
+
+Pinned by tests/test_oracle_pins.py; every function has at least one pin that
+does not re-derive it from its own formula (closed forms, brute force,
+finite differences, hand-worked fixtures in tests/golden/).
+"""
+from .lcvq import (BITS, ZMAX, SingularMatrix, brute_nearest, decode, encode, gemm_packed2b,  # noqa: F401
+                   init_codebook, inverse, latent, linear_bwd, linear_fwd, mse, near_boundary,
+                   pack2b, quantize, round_clamp, unpack2b)

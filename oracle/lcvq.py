@@ -1,0 +1,224 @@
+"""Plain fp64 CPU oracle of the LC-VQ linear layer (LC-QAT, arxiv 2606.10531).
+
+TEST INFRASTRUCTURE ONLY. Nothing in the product path imports this module:
+only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py`` (its CPU
+baseline and reference legs) may use it. It shares no code, table or helper
+with the CUDA library; the two meet only through the seeded input
+generators, which hold none of the method's arithmetic.
+
+Every function is a literal restatement of one definition of the paper, in
+the paper's notation, using NumPy fp64 and library primitives (matmul,
+inverse) with no blocking, fusion or reordering:
+
+  * codebook            c = A z + B, z in {0,1,2,3}^d          (Sec. 2.2, Eq. lc_codebook)
+  * nearest codeword    i_g = argmin_k ||w_g - c_k||^2          (Sec. 2.1, Eq. vq_assign)
+  * integer weights     W_z = clip(round(W_p), 0, 2^b - 1)      (Sec. 3.2, Eq. quant_param)
+  * column grouping     G = n/d groups of d consecutive columns (Sec. 3.2)
+  * decode              W_hat^T = [A W_{z,i}^T + B 1^T]_i       (Sec. 3.2, Eq. def:forward)
+  * forward             Y = X W_hat^T (nn.Linear orientation)   (Sec. 3.2, Eq. def:forward_x)
+  * backward            exact gradients of the linear map, with the
+                        straight-through estimator dW_z/dW_p = 1 (Sec. 3.3)
+
+Readings where the paper is silent or inconsistent (listed in the design doc):
+  * encode maps a real weight group to latent coordinates u = A^{-1}(w - B)
+    and rounds/clamps u (Sec. 2.2 "rounding and clamping", Babai rounding);
+  * round is round-half-to-even; NaN latent values encode to 0;
+  * Y = X W_hat^T (the printed "Y = X W_hat" is shape-inconsistent);
+  * the optional latent affine z = clip(round(P/s + t)) with dP = dZ/s
+    reconciles Eq. quant_param with Eq. xavier_preprocess; s=1, t=0 is the
+    literal Eq. quant_param. P/s + t is evaluated in fp32 (the precision in
+    which the integer decision is taken on both sides): fl(fl(P*fl(1/s)) + t);
+  * packed storage: 4 codes per byte, column c in bits 2(c mod 4)..+1 of
+    byte floor(c/4), least significant first.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+BITS = 2                       # b = 2 (Sec. 3.2, Eq. quant_param)
+ZMAX = (1 << BITS) - 1         # 2^b - 1 = 3, largest level of {0,1,2,3}
+COND_LIMIT = 1e8               # A with a larger condition number is "singular"
+
+
+class SingularMatrix(ValueError):
+    pass
+
+
+def _f64(x):
+    return np.asarray(x, dtype=np.float64)
+
+
+def _grouped(M: np.ndarray, d: int) -> np.ndarray:
+    """View an m x n matrix as (m, G, d): G = n/d groups of d consecutive columns (Sec. 3.2)."""
+    m, n = M.shape
+    if n % d:
+        raise ValueError(f"n={n} is not a multiple of the group size d={d}")
+    return M.reshape(m, n // d, d)
+
+
+def inverse(A) -> np.ndarray:
+    """A^{-1} in fp64 by the library LU inverse; refuses ill-conditioned A."""
+    A64 = _f64(A)
+    if not np.all(np.isfinite(A64)) or np.linalg.cond(A64) > COND_LIMIT:
+        raise SingularMatrix("A is singular or ill-conditioned")
+    return np.linalg.inv(A64)
+
+
+def round_clamp(V) -> np.ndarray:
+    """clip(round(v), 0, 2^b - 1) element-wise (Eq. quant_param); round half to even; NaN -> 0."""
+    V64 = _f64(V)
+    R = np.clip(np.rint(V64), 0, ZMAX)
+    R = np.where(np.isnan(V64), 0.0, R)
+    return R.astype(np.uint8)
+
+
+def latent(W, A, b, d: int) -> np.ndarray:
+    """Latent coordinates u_g = A^{-1}(w_g - B) of every weight group (Sec. 2.2 reading).
+
+    Returns an (m, n) fp64 matrix laid out like W.
+    """
+    W64 = _f64(W)
+    m, n = W64.shape
+    Ainv = inverse(A)
+    Wg = _grouped(W64, d) - _f64(b)            # w_g - B
+    U = Wg @ Ainv.T                            # row-vector form of A^{-1} (w_g - B)
+    return U.reshape(m, n)
+
+
+def near_boundary(U, eps: float = 1e-5) -> np.ndarray:
+    """Mask of latent values within eps of a decision boundary k + 1/2 of clamp(round(.)).
+
+    Only 0.5, 1.5 and 2.5 are boundaries on {0,1,2,3}: below 0 and above 3
+    the clamp absorbs the rounding.
+    """
+    U64 = _f64(U)
+    mask = np.zeros(U64.shape, dtype=bool)
+    for k in range(ZMAX):
+        mask |= np.abs(U64 - (k + 0.5)) < eps
+    return mask
+
+
+def encode(W, A, b, d: int) -> dict:
+    """LC-VQ encoder: z_g = clip(round(A^{-1}(w_g - B)), 0, 3) (Sec. 2.2; Eq. lc_codebook).
+
+    Returns codes (uint8, m x n), latent u (fp64), the near-boundary mask and
+    the reconstruction MSE mean((W - W_hat)^2).
+    """
+    U = latent(W, A, b, d)
+    Z = round_clamp(U)
+    return {"codes": Z, "latent": U, "near": near_boundary(U), "mse": mse(W, Z, A, b, d)}
+
+
+def quantize(P, s: float = 1.0, t: float = 0.0) -> np.ndarray:
+    """Integer weights W_z = clip(round(P/s + t), 0, 3) (Eq. quant_param; s=1, t=0 literal).
+
+    P/s + t is formed in fp32 as fl(fl(P * fl(1/s)) + t): the precision in
+    which the integer decision is made.
+    """
+    P32 = np.asarray(P, dtype=np.float32)
+    inv_s = np.float32(1.0) / np.float32(s)
+    V = (P32 * inv_s).astype(np.float32) + np.float32(t)
+    return round_clamp(V.astype(np.float32))
+
+
+def decode(Z, A, b, d: int) -> np.ndarray:
+    """Affine decode w_hat_g = A z_g + B for every group (Eq. def:forward), fp64 (m x n)."""
+    Z64 = _f64(Z)
+    m, n = Z64.shape
+    What = _grouped(Z64, d) @ _f64(A).T + _f64(b)   # row-vector form of A z_g + B
+    return What.reshape(m, n)
+
+
+def mse(W, Z, A, b, d: int) -> float:
+    """Reconstruction error mean over all weights of (W - W_hat)^2 (fp64)."""
+    W64 = _f64(W)
+    if W64.size == 0:
+        return 0.0
+    return float(np.mean((W64 - decode(Z, A, b, d)) ** 2))
+
+
+def linear_fwd(X, Z, A, b, d: int) -> np.ndarray:
+    """Layer output Y = X W_hat^T with W_hat decoded from the integer weights (Eq. def:forward)."""
+    return _f64(X) @ decode(Z, A, b, d).T
+
+
+def linear_bwd(X, dY, Z, A, b, d: int, P=None, s: float = 1.0, t: float = 0.0,
+               ste: str = "identity") -> dict:
+    """Gradients of L with dL/dY = dY through Y = X W_hat^T, W_hat = decode(Z).
+
+    The layer is linear in X, A, B and in z treated as a real vector, so:
+        dW_hat = dY^T X
+        dX     = dY W_hat
+        dz_g   = A^T dw_hat_g          (row-vector form: dw_hat_g @ A)
+        dA     = sum_{r,g} dw_hat_{r,g} z_{r,g}^T
+        dB     = sum_{r,g} dw_hat_{r,g}
+    and the straight-through estimator dW_z/dW_p = 1 (Sec. 3.3) gives
+    dP = dZ / s; with ste="clipped" the gradient is zeroed where
+    P/s + t lies outside [-1/2, 2^b - 1/2].
+    """
+    X64, dY64, A64 = _f64(X), _f64(dY), _f64(A)
+    What = decode(Z, A, b, d)
+    dWhat = dY64.T @ X64
+    dX = dY64 @ What
+    dWg = _grouped(dWhat, d)
+    Zg = _grouped(_f64(Z), d)
+    dZ = (dWg @ A64).reshape(dWhat.shape)
+    dA = np.einsum("rgj,rgk->jk", dWg, Zg)
+    db = dWg.sum(axis=(0, 1))
+    dP = dZ / s
+    if ste == "clipped":
+        if P is None:
+            raise ValueError("ste='clipped' needs P")
+        P32 = np.asarray(P, dtype=np.float32)
+        V = ((P32 * (np.float32(1.0) / np.float32(s))).astype(np.float32) + np.float32(t)).astype(np.float64)
+        dP = np.where((V >= -0.5) & (V <= ZMAX + 0.5), dP, 0.0)
+    elif ste != "identity":
+        raise ValueError(f"unknown ste mode {ste!r}")
+    return {"dX": dX, "dP": dP, "dA": dA, "db": db, "dW_hat": dWhat}
+
+
+def pack2b(Z) -> np.ndarray:
+    """Pack 2-bit codes 4 per byte: column c -> bits 2(c mod 4) of byte floor(c/4), LSB first."""
+    Zu = np.asarray(Z, dtype=np.uint8)
+    m, n = Zu.shape
+    if n % 4:
+        raise ValueError("n must be a multiple of 4 to pack")
+    Q = Zu.reshape(m, n // 4, 4).astype(np.uint32)
+    out = np.zeros((m, n // 4), dtype=np.uint32)
+    for q in range(4):
+        out |= (Q[:, :, q] & 3) << (2 * q)
+    return out.astype(np.uint8)
+
+
+def unpack2b(packed, n: int) -> np.ndarray:
+    """Inverse of pack2b."""
+    Pk = np.asarray(packed, dtype=np.uint8)
+    m = Pk.shape[0]
+    Z = np.zeros((m, n // 4, 4), dtype=np.uint8)
+    for q in range(4):
+        Z[:, :, q] = (Pk >> (2 * q)) & 3
+    return Z.reshape(m, n)
+
+
+def gemm_packed2b(X, packed, A, b, d: int, n: int) -> np.ndarray:
+    """Deployment product Y = X W_hat^T from packed codes: unpack, decode, multiply."""
+    return linear_fwd(X, unpack2b(packed, n), A, b, d)
+
+
+def init_codebook(G, bits: int = BITS):
+    """A = s G, B = -s G mu 1 with mu = (2^b - 1)/2 and s = sqrt(12/(2^{2b} - 1)) (Eq. init_ab)."""
+    G64 = _f64(G)
+    mu = ((1 << bits) - 1) / 2.0
+    s = np.sqrt(12.0 / ((1 << (2 * bits)) - 1))
+    A = s * G64
+    B = -s * G64 @ (mu * np.ones(G64.shape[0]))
+    return A, B
+
+
+def brute_nearest(W, A, b, d: int):
+    """Exhaustive nearest codeword over all 4^d codewords (Eq. vq_assign on Eq. lc_codebook).
+
+    Runs the C searcher in oracle/brute.c. Returns (codes uint8 m x n, squared distance per group).
+    """
+    from . import _native
+    return _native.brute_nearest(W, A, b, d)

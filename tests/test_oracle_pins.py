@@ -1,0 +1,299 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Each test ties one oracle function to a closed form, a textbook special
+case, brute force on tiny inputs, finite differences, or a hand-worked
+fixture in tests/golden/. Together they fail on a dropped term, a wrong
+sign, a transposed operand or a wrong index in any oracle function.
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from tests.golden_io import read_keyed, read_rows
+
+RNG = np.random.default_rng(12345)
+
+
+def config_like_A(d, rng):
+    return 0.01 * np.eye(d) + rng.normal(0, 1e-3, (d, d))
+
+
+# ----------------------------------------------------------------------------- encode / quantize
+
+def test_round_clamp_table_matches_textbook(golden_dir):
+    rows = read_rows("round_clamp_table.txt")
+    v = np.array([float(r[0]) for r in rows])
+    want = np.array([int(r[1]) for r in rows], dtype=np.uint8)
+    assert np.array_equal(oracle.round_clamp(v), want)
+    # Python's round() is round-half-to-even: the scalar textbook rule.
+    assert [min(max(round(x), 0), 3) for x in v] == list(want)
+
+
+def test_identity_codebook_reduces_to_scalar_round_clamp():
+    """A = I, B = 0: LC-VQ encode is scalar clamp(round(w)) (SQ special case, Sec. 3.2)."""
+    for d in (4, 8):
+        W = RNG.uniform(-1.5, 4.5, (6, 8 * d))
+        codes = oracle.encode(W, np.eye(d), np.zeros(d), d)["codes"]
+        scalar = np.array([[min(max(round(w), 0), 3) for w in row] for row in W], dtype=np.uint8)
+        assert np.array_equal(codes, scalar)
+
+
+def test_encode_worked_example(golden_dir):
+    g = read_keyed("encode_worked_d4.txt")
+    d = int(g["d"][0])
+    A = g["A"].reshape(d, d)
+    out = oracle.encode(g["w"].reshape(1, -1), A, g["B"], d)
+    np.testing.assert_allclose(out["latent"].ravel(), g["u"], rtol=0, atol=1e-12)
+    assert np.array_equal(out["codes"].ravel(), g["z"].astype(np.uint8))
+    np.testing.assert_allclose(oracle.decode(out["codes"], A, g["B"], d).ravel(), g["w_hat"], atol=1e-12)
+
+
+def test_codes_lie_in_level_set_including_nan_and_inf():
+    for d in (4, 8):
+        A = config_like_A(d, RNG)
+        W = RNG.normal(0, 0.05, (16, 4 * d))
+        W[0, :3] = [np.nan, np.inf, -np.inf]
+        out = oracle.encode(W, A, RNG.normal(0, 1e-3, d), d)
+        assert out["codes"].dtype == np.uint8
+        assert set(np.unique(out["codes"])) <= {0, 1, 2, 3}
+    z = oracle.round_clamp(np.array([np.nan, np.inf, -np.inf]))
+    assert list(z) == [0, 3, 0]
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_reencoding_a_decoded_codeword_returns_its_codes(d):
+    """Codewords are fixed points of the encoder: encode(decode(z)) = z."""
+    for A in (config_like_A(d, RNG), oracle.init_codebook(np.linalg.qr(RNG.normal(size=(d, d)))[0])[0]):
+        b = RNG.normal(0, 1e-3, d)
+        Z = RNG.integers(0, 4, (32, 16 * d)).astype(np.uint8)
+        W = oracle.decode(Z, A, b, d)
+        assert np.array_equal(oracle.encode(W, A, b, d)["codes"], Z)
+
+
+@pytest.mark.parametrize("d,m,n", [(4, 16, 64), (8, 4, 32)])
+def test_bruteforce_nearest_equals_rounding_for_diagonal_positive_A(d, m, n):
+    """For diagonal positive A the distance separates per coordinate, so the exhaustive
+    4^d search of Eq. vq_assign must pick exactly the rounded-and-clamped latent."""
+    A = np.diag(RNG.uniform(0.005, 0.02, d))
+    b = RNG.normal(0, 1e-3, d)
+    W = RNG.normal(0.015, 0.02, (m, n))
+    codes_bf, _ = oracle.brute_nearest(W, A, b, d)
+    out = oracle.encode(W, A, b, d)
+    assert not out["near"].any()
+    assert np.array_equal(codes_bf, out["codes"])
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_rounding_never_beats_exhaustive_search_for_general_A(d):
+    A = config_like_A(d, RNG) + RNG.normal(0, 4e-3, (d, d))
+    b = RNG.normal(0, 1e-3, d)
+    W = RNG.normal(0, 0.02, (3, 4 * d))
+    codes_bf, dist_bf = oracle.brute_nearest(W, A, b, d)
+    Zr = oracle.encode(W, A, b, d)["codes"]
+    dist_r = ((W - oracle.decode(Zr, A, b, d)) ** 2).reshape(3, 4, d).sum(-1)
+    assert np.all(dist_r >= dist_bf - 1e-15)
+    # the brute force really is the minimum: its codes decode to its distance
+    np.testing.assert_allclose(((W - oracle.decode(codes_bf, A, b, d)) ** 2).reshape(3, 4, d).sum(-1), dist_bf,
+                               rtol=1e-12)
+
+
+def test_near_boundary_mask_marks_only_half_integers_inside_range():
+    u = np.array([0.5, 1.5 + 5e-6, 2.5 - 9e-6, 3.5, -0.5, 1.49, 0.0])
+    assert list(oracle.near_boundary(u)) == [True, True, True, False, False, False, False]
+
+
+def test_quantize_latent_affine_reading():
+    """s = 1, t = 0 is the literal Eq. quant_param; with s, t it rounds P/s + t formed in fp32."""
+    P = np.array([[-0.6, 0.2, 0.7, 1.5, 2.4999, 3.9, 2.5, 100.0]], dtype=np.float32)
+    assert list(oracle.quantize(P)[0]) == [0, 0, 1, 2, 2, 3, 2, 3]
+    s, t = 0.25, 1.5
+    want = [min(max(round(float(np.float32(np.float32(p) * np.float32(4.0)) + np.float32(1.5))), 0), 3)
+            for p in P[0]]
+    assert list(oracle.quantize(P, s, t)[0]) == want
+
+
+def test_mse_definition_and_zero_on_codewords():
+    d = 4
+    A, b = config_like_A(d, RNG), RNG.normal(0, 1e-3, d)
+    Z = RNG.integers(0, 4, (8, 32))
+    assert oracle.mse(oracle.decode(Z, A, b, d), Z, A, b, d) < 1e-30
+    W = RNG.normal(0, 0.02, (8, 32))
+    out = oracle.encode(W, A, b, d)
+    direct = sum((W[r, c] - oracle.decode(out["codes"], A, b, d)[r, c]) ** 2 for r in range(8) for c in range(32)) / 256
+    assert math.isclose(out["mse"], direct, rel_tol=1e-12)
+
+
+# ----------------------------------------------------------------------------- decode
+
+def test_decode_worked_example(golden_dir):
+    g = read_keyed("decode_worked_d4.txt")
+    d = int(g["d"][0])
+    W_hat = oracle.decode(g["z"].reshape(1, d), g["A"].reshape(d, d), g["B"], d)
+    np.testing.assert_allclose(W_hat.ravel(), g["w_hat"], rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_decode_permutation_A_moves_codes_in_stated_direction(d):
+    """A[j][(j+1) % d] = 1: w_hat_j = z_{(j+1) mod d} within every group (catches a transposed A)."""
+    A = np.zeros((d, d))
+    for j in range(d):
+        A[j, (j + 1) % d] = 1.0
+    Z = RNG.integers(0, 4, (5, 3 * d))
+    W_hat = oracle.decode(Z, A, np.zeros(d), d)
+    for r in range(5):
+        for g in range(3):
+            for j in range(d):
+                assert W_hat[r, g * d + j] == Z[r, g * d + (j + 1) % d]
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_initialised_codebook_has_zero_mean_and_identity_covariance(d, golden_dir):
+    """Eq. init_ab: over all 4^d codewords the codebook mean is 0 and its covariance is I."""
+    c = read_keyed("init_constants.txt")
+    G = np.linalg.qr(np.random.default_rng(7).normal(size=(d, d)))[0]
+    A, B = oracle.init_codebook(G)
+    np.testing.assert_allclose(A, c["s"][0] * G, rtol=1e-15)
+    allz = np.array(list(itertools.product(range(4), repeat=d)), dtype=np.uint8)   # 4^d x d
+    C = oracle.decode(allz, A, B, d)      # one group per row
+    np.testing.assert_allclose(C.mean(0), 0.0, atol=1e-12)
+    np.testing.assert_allclose(np.cov(C.T, bias=True), np.eye(d), atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- forward
+
+def test_forward_matches_explicit_loops_on_tiny_input():
+    N, m, n, d = 2, 3, 8, 4
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    Z = RNG.integers(0, 4, (m, n))
+    X = RNG.normal(size=(N, n))
+    Y = oracle.linear_fwd(X, Z, A, b, d)
+    for t in range(N):
+        for r in range(m):
+            acc = 0.0
+            for g in range(n // d):
+                for j in range(d):
+                    w = b[j] + sum(A[j][k] * Z[r][g * d + k] for k in range(d))
+                    acc += X[t][g * d + j] * w
+            assert math.isclose(Y[t, r], acc, rel_tol=1e-12, abs_tol=1e-12)
+
+
+def test_forward_one_hot_rows_select_decoded_weights():
+    """X = e_c: Y[:, r] = W_hat[r, c] (fixes the Y = X W_hat^T orientation)."""
+    d, m, n = 4, 5, 12
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    Z = RNG.integers(0, 4, (m, n))
+    Y = oracle.linear_fwd(np.eye(n), Z, A, b, d)
+    np.testing.assert_allclose(Y, oracle.decode(Z, A, b, d).T, atol=1e-13)
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_forward_equals_reformulated_sum(d):
+    """Eq. def:forward_x: Y = sum_i (X_i A) W_{z,i}^T + sum_i (X_i B) 1^T."""
+    N, m, n = 7, 9, 6 * d
+    A, b = config_like_A(d, RNG), RNG.normal(0, 1e-3, d)
+    Z = RNG.integers(0, 4, (m, n))
+    X = RNG.normal(size=(N, n))
+    Y = np.zeros((N, m))
+    for i in range(n // d):
+        Xi = X[:, i * d:(i + 1) * d]
+        Y += (Xi @ A) @ Z[:, i * d:(i + 1) * d].T + np.outer(Xi @ b, np.ones(m))
+    np.testing.assert_allclose(oracle.linear_fwd(X, Z, A, b, d), Y, rtol=1e-12, atol=1e-15)
+
+
+def test_packed_product_equals_unpacked_product():
+    d, m, n = 8, 6, 32
+    A, b = config_like_A(d, RNG), RNG.normal(0, 1e-3, d)
+    Z = RNG.integers(0, 4, (m, n)).astype(np.uint8)
+    X = RNG.normal(size=(3, n))
+    np.testing.assert_allclose(oracle.gemm_packed2b(X, oracle.pack2b(Z), A, b, d, n),
+                               oracle.linear_fwd(X, Z, A, b, d), rtol=1e-14)
+
+
+# ----------------------------------------------------------------------------- backward
+
+def _loss(X, A, b, Zc, dY, d):
+    """<dY, Y> with z continuous (the STE treats the integer weights as real)."""
+    m, n = Zc.shape
+    W_hat = (Zc.reshape(m, n // d, d) @ A.T + b).reshape(m, n)
+    return float(np.sum(dY * (X @ W_hat.T)))
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_backward_equals_central_finite_differences(d):
+    """L = <dY, Y> is linear in each of X, A, B and z, so central differences are exact."""
+    N, m, n = 3, 4, 2 * d
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    Z = RNG.integers(0, 4, (m, n)).astype(np.float64)
+    X, dY = RNG.normal(size=(N, n)), RNG.normal(size=(N, m))
+    g = oracle.linear_bwd(X, dY, Z, A, b, d)
+    h = 0.5
+
+    def fd(arr, idx, f):
+        old = arr[idx]
+        arr[idx] = old + h
+        up = f()
+        arr[idx] = old - h
+        dn = f()
+        arr[idx] = old
+        return (up - dn) / (2 * h)
+
+    L = lambda: _loss(X, A, b, Z, dY, d)  # noqa: E731
+    for idx in np.ndindex(X.shape):
+        assert math.isclose(g["dX"][idx], fd(X, idx, L), rel_tol=1e-9, abs_tol=1e-9)
+    for idx in np.ndindex(A.shape):
+        assert math.isclose(g["dA"][idx], fd(A, idx, L), rel_tol=1e-9, abs_tol=1e-9)
+    for idx in np.ndindex(b.shape):
+        assert math.isclose(g["db"][idx], fd(b, idx, L), rel_tol=1e-9, abs_tol=1e-9)
+    for idx in np.ndindex(Z.shape):
+        assert math.isclose(g["dP"][idx], fd(Z, idx, L), rel_tol=1e-9, abs_tol=1e-9)
+
+
+def test_ste_latent_scale_divides_gradient():
+    """With z = P/s + t treated as identity-rounded, dL/dP = dL/dz / s (chain rule)."""
+    d, s, t = 4, 0.25, 1.5
+    N, m, n = 2, 3, 8
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    P = RNG.normal(size=(m, n))
+    X, dY = RNG.normal(size=(N, n)), RNG.normal(size=(N, m))
+    Z = oracle.quantize(P, s, t)
+    g = oracle.linear_bwd(X, dY, Z, A, b, d, P=P, s=s, t=t)
+    h = 0.5
+    for idx in [(0, 0), (1, 3), (2, 7)]:
+        Zc = Z.astype(np.float64)
+        Zc[idx] += h / s
+        up = _loss(X, A, b, Zc, dY, d)
+        Zc[idx] -= 2 * h / s
+        dn = _loss(X, A, b, Zc, dY, d)
+        assert math.isclose(g["dP"][idx], (up - dn) / (2 * h), rel_tol=1e-9, abs_tol=1e-12)
+
+
+def test_clipped_ste_masks_outside_clip_range_only():
+    d, N, m, n = 4, 2, 2, 8
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    P = np.array([[-0.6, -0.5, 0.0, 1.7, 3.5, 3.6, 9.0, 2.0]] * 2, dtype=np.float32)
+    X, dY = RNG.normal(size=(N, n)), RNG.normal(size=(N, m))
+    Z = oracle.quantize(P)
+    full = oracle.linear_bwd(X, dY, Z, A, b, d)["dP"]
+    clip = oracle.linear_bwd(X, dY, Z, A, b, d, P=P, ste="clipped")["dP"]
+    keep = np.array([False, True, True, True, True, False, False, True])
+    assert np.all(clip[:, ~keep] == 0)
+    np.testing.assert_array_equal(clip[:, keep], full[:, keep])
+
+
+# ----------------------------------------------------------------------------- packing
+
+def test_pack_golden_bytes(golden_dir):
+    rows = read_rows("pack_bytes.txt")
+    Z = np.array([[int(v) for v in r[:4]] for r in rows], dtype=np.uint8)
+    want = np.array([int(r[4], 16) for r in rows], dtype=np.uint8)
+    assert np.array_equal(oracle.pack2b(Z).ravel(), want)
+
+
+def test_pack_unpack_round_trip():
+    Z = RNG.integers(0, 4, (7, 64)).astype(np.uint8)
+    P = oracle.pack2b(Z)
+    assert P.shape == (7, 16)
+    assert np.array_equal(oracle.unpack2b(P, 64), Z)
