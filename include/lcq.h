@@ -1,0 +1,185 @@
+/*
+ * lcq.h - C ABI of liblcq, the GB300 (sm_103a) LC-VQ linear layer.
+ *
+ * LC-QAT (arxiv 2606.10531) stores a weight matrix W (m x n, nn.Linear
+ * orientation: m outputs, n inputs) as 2-bit integer weights z in {0,1,2,3}
+ * grouped in d consecutive input columns, plus one affine map (A, B) per
+ * matrix (Sec. 2.2 Eq. lc_codebook; Sec. 3.2 Eq. def:forward):
+ *
+ *     w_hat[r, g*d + j] = sum_k A[j][k] * z[r, g*d + k] + B[j]
+ *
+ * Conventions shared by every call:
+ *   - Tensors are caller-owned DEVICE pointers, row-major and contiguous,
+ *     16-byte aligned (LCQ_ERR_ALIGN otherwise). A is d x d fp32 row-major,
+ *     b (the paper's B) is d fp32. bf16 tensors are passed as uint16_t bit
+ *     patterns.
+ *   - d must be 4 or 8 (LCQ_ERR_UNSUPPORTED); n must be a multiple of 8
+ *     (and of d); m, n, N >= 0. Empty problems are valid and write the
+ *     mathematically correct (zero) results.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream). Every call
+ *     is asynchronous and stream-ordered; argument validation is
+ *     synchronous and happens before anything is enqueued.
+ *   - The library never allocates device memory. Calls that need scratch
+ *     take `ws`/`ws_bytes`, a caller-owned device buffer of at least
+ *     lcq_workspace_size(op, ...) bytes (LCQ_ERR_WORKSPACE otherwise). The
+ *     first 256 bytes of a workspace hold a device status word that kernels
+ *     set on device-detected errors (LCQ_ERR_SINGULAR, LCQ_ERR_TIMEOUT);
+ *     read it with lcq_device_status(). A workspace must not be shared by
+ *     calls that may run concurrently.
+ *   - Packed codes: 4 per byte; column c of a row sits in bits
+ *     2*(c mod 4) .. 2*(c mod 4)+1 of byte c/4 of that row (LSB first);
+ *     a packed matrix is m x (n/4) bytes.
+ */
+#ifndef LCQ_H
+#define LCQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum lcq_status {
+    LCQ_OK = 0,
+    LCQ_ERR_NULL = 1,        /* a required pointer is NULL                              */
+    LCQ_ERR_SHAPE = 2,       /* negative size, n % d != 0, n % 8 != 0                   */
+    LCQ_ERR_ALIGN = 3,       /* a tensor pointer is not 16-byte aligned                 */
+    LCQ_ERR_UNSUPPORTED = 4, /* d not in {4, 8}, unknown STE mode                       */
+    LCQ_ERR_WORKSPACE = 5,   /* workspace NULL or smaller than lcq_workspace_size()     */
+    LCQ_ERR_CUDA = 6,        /* a CUDA runtime call or kernel launch failed             */
+    LCQ_ERR_SINGULAR = 7,    /* device-detected: A is not invertible (encode)           */
+    LCQ_ERR_TIMEOUT = 8,     /* device-detected: a bounded pipeline wait gave up        */
+    LCQ_ERR_ARG = 9          /* any other invalid argument (e.g. latent_scale == 0)     */
+} lcq_status;
+
+/* Operation selector for lcq_workspace_size(). */
+typedef enum lcq_op {
+    LCQ_OP_ENCODE = 1,
+    LCQ_OP_LINEAR_FWD = 2,
+    LCQ_OP_LINEAR_BWD = 3,
+    LCQ_OP_GEMM_PACKED2B = 4
+} lcq_op;
+
+/* Straight-through estimator variants for dP (Sec. 3.3). */
+typedef enum lcq_ste_mode {
+    LCQ_STE_IDENTITY = 0, /* dW_z/dW_p = 1 everywhere (the paper's STE)                  */
+    LCQ_STE_CLIPPED = 1   /* zero where P/s + t lies outside [-1/2, 7/2]                 */
+} lcq_ste_mode;
+
+/* Options of the training calls. NULL means {1, 0, LCQ_STE_IDENTITY}. */
+typedef struct lcq_opts {
+    float latent_scale;   /* s: integer weights are clip(round(P/s + t), 0, 3); must be != 0 */
+    float latent_offset;  /* t                                                                 */
+    int32_t ste_mode;     /* lcq_ste_mode                                                      */
+    int32_t reserved;     /* must be 0                                                         */
+} lcq_opts;
+
+/*
+ * Bytes of device workspace an operation needs for the given sizes
+ * (N = tokens, m = output rows, n = input dim, d = group size). Returns 0
+ * for an unknown op. The size only grows with each argument.
+ */
+size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d);
+
+/*
+ * lcq_encode - map real weights to 2-bit latent codes (Sec. 2.2: codewords
+ * A z + B; z obtained by rounding and clamping; Eq. quant_param with b = 2).
+ *
+ *   u[r, g*d + k] = sum_j Ainv[k][j] * (W[r, g*d + j] - b[j]),  Ainv = A^{-1}
+ *   z = clip(round_half_even(u), 0, 3)   (NaN -> 0, +inf -> 3, -inf -> 0)
+ *
+ * W       [m][n] fp32 input.
+ * packed  [m][n/4] uint8 output, or NULL.
+ * codes   [m][n] uint8 output (one code per byte), or NULL.
+ * latent  [m][n] fp32 output u, or NULL.
+ * mse     device double, receives mean((W - (A z + b))^2) over all m*n
+ *         weights (0 when m*n == 0), or NULL.
+ * A^{-1} is formed on the device (fp64 Gauss-Jordan, rounded to fp32); if A
+ * is singular the device status word becomes LCQ_ERR_SINGULAR and every code
+ * is 0. Needs lcq_workspace_size(LCQ_OP_ENCODE, 0, m, n, d) bytes of ws.
+ */
+lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b,
+                      uint8_t *packed, uint8_t *codes, float *latent, double *mse,
+                      void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * lcq_decode - affine decode of packed codes (Sec. 3.2 Eq. def:forward):
+ *   W_hat[r, g*d + j] = sum_k A[j][k] * z[r, g*d + k] + b[j]
+ * packed [m][n/4] uint8 input. W_hat_f32 [m][n] fp32 and/or W_hat_bf16 [m][n]
+ * bf16 outputs (either may be NULL, not both). Needs no workspace.
+ */
+lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const float *A, const float *b,
+                      float *W_hat_f32, uint16_t *W_hat_bf16, void *stream);
+
+/*
+ * lcq_pack2b - pack one-code-per-byte codes [m][n] into [m][n/4] bytes in the
+ * library's bit order (see the header comment). Only the two low bits of
+ * each input byte are used. n must be a multiple of 4. Needs no workspace.
+ */
+lcq_status lcq_pack2b(const uint8_t *codes, int64_t m, int64_t n, uint8_t *packed, void *stream);
+
+/*
+ * lcq_linear_fwd - forward pass of one LC-VQ linear layer (Sec. 3.2,
+ * Eq. quant_param and Eq. def:forward; output orientation of nn.Linear):
+ *   Z = clip(round(P/s + t), 0, 3)      (P/s + t formed in fp32 as fl(fl(P*fl(1/s)) + t))
+ *   W_hat = A Z_g + b per group          (rounded to bf16 as the GEMM operand)
+ *   Y = X W_hat^T                        (bf16 tensor-core GEMM, fp32 accumulation)
+ * X [N][n] bf16, P [m][n] fp32 latent (proxy) weights, Y [N][m] bf16 output,
+ * packed_saved [m][n/4] uint8 output (the integer weights, for the backward;
+ * may be NULL). Needs lcq_workspace_size(LCQ_OP_LINEAR_FWD, N, m, n, d).
+ */
+lcq_status lcq_linear_fwd(const uint16_t *X, int64_t N, const float *P, int64_t m, int64_t n, int d,
+                          const float *A, const float *b, const lcq_opts *opts,
+                          uint16_t *Y, uint8_t *packed_saved, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * lcq_linear_bwd - straight-through backward of one LC-VQ linear layer
+ * (Sec. 3.3; exact gradients of the linear map of Eq. def:forward):
+ *   dW_hat = dY^T X                                      (fp32, never stored)
+ *   dX     = dY W_hat                                    [N][n] bf16
+ *   dP[r, g*d + k] = (1/s) * sum_j dW_hat[r, g*d + j] A[j][k]  (masked in CLIPPED mode)
+ *   dA[j][k] = sum_{r,g} dW_hat[r, g*d + j] * z[r, g*d + k]     [d][d] fp32
+ *   db[j]    = sum_{r,g} dW_hat[r, g*d + j]                     [d] fp32
+ * X [N][n] bf16, dY [N][m] bf16, packed_saved [m][n/4] from lcq_linear_fwd,
+ * P [m][n] fp32 (read only in CLIPPED mode; may be NULL otherwise).
+ * dX may be NULL (skips the dX GEMM). dA and db are overwritten, not
+ * accumulated; the sums are taken in a fixed order (bitwise reproducible).
+ * Needs lcq_workspace_size(LCQ_OP_LINEAR_BWD, N, m, n, d).
+ */
+lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *packed_saved, const float *P,
+                          int64_t N, int64_t m, int64_t n, int d, const float *A, const float *b,
+                          const lcq_opts *opts, uint16_t *dX, float *dP, float *dA, float *db,
+                          void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * lcq_gemm_packed2b - deployment product from packed 2-bit codes through the
+ * reformulated forward (Sec. 3.2 Eq. def:forward_x):
+ *   Y = sum_g (X_g A) Z_g^T + sum_g (X_g b) 1^T  ( = X W_hat^T )
+ * X [N][n] bf16 activations (any N; built for N <= 16 tokens), packed
+ * [m][n/4] uint8 codes, Y [N][m] bf16 output. X_g A is rounded to bf16
+ * before the tensor-core product; accumulation is fp32.
+ * Needs lcq_workspace_size(LCQ_OP_GEMM_PACKED2B, N, m, n, d).
+ */
+lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
+                             int d, const float *A, const float *b, uint16_t *Y,
+                             void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * lcq_device_status - synchronise `stream`, then copy the workspace's device
+ * status word (LCQ_OK or a device-detected lcq_status) to *status_out and,
+ * if clear != 0, reset it to LCQ_OK.
+ */
+lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, int clear);
+
+/* Static description of a status code; never NULL. */
+const char *lcq_status_string(lcq_status s);
+
+/* Number of kernels this library has launched in the calling process. */
+uint64_t lcq_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LCQ_H */

@@ -1,0 +1,99 @@
+// Host-side internal interface between the C ABI (lcq_api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lcq {
+
+void count_launch();
+
+struct EncodeArgs {
+    const float *W;
+    int64_t m, n;
+    const float *A, *b;
+    uint8_t *packed, *codes;
+    float *latent;
+    double *mse;
+    double *partials;     // [grid] per-CTA sums of squared residuals
+    unsigned *counter;    // zeroed before launch
+    int32_t *status;
+};
+
+struct QuantDecodeArgs {
+    const float *P;
+    int64_t m, n;
+    const float *A, *b;
+    float inv_s, t;
+    uint8_t *packed;      // may be NULL
+    uint16_t *W_hat;      // bf16 [m][n]
+    int32_t *status;
+};
+
+struct DecodeArgs {
+    const uint8_t *packed;
+    int64_t m, n;
+    const float *A, *b;
+    float *W_f32;
+    uint16_t *W_bf16;
+};
+
+int encode_max_blocks(int num_sms);
+cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t st);
+cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cudaStream_t st);
+cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t st);
+cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, int num_sms, cudaStream_t st);
+cudaError_t launch_reduce_partials(const float *partials, int nparts, int d, float *dA, float *db, cudaStream_t st);
+
+// ---------------------------------------------------------------- tensor-core GEMM
+// C[M][N] = sum_k A(m, k) * B(n, k), bf16 operands, fp32 accumulation in TMEM.
+// Operand X is "K-major" when stored [rows][K] (K contiguous) and "MN-major"
+// when stored [K][rows].
+enum GemmEpilogue { EPI_STORE_BF16 = 0, EPI_DW = 1 };
+
+struct GemmOperand {
+    const uint16_t *ptr;
+    int64_t ld;          // elements between consecutive rows of the stored matrix
+    bool mn_major;
+};
+
+struct DwEpilogue {
+    const uint8_t *packed;   // [M][N/4] codes of the weight matrix
+    const float *A;          // d x d
+    const float *P;          // [M][N] latent weights (CLIPPED STE only), else NULL
+    float *dP;               // [M][N]
+    float *partials;         // [grid][d*d + d]
+    float inv_s, t;
+    int ste_mode;
+    int d;
+};
+
+struct GemmProblem {
+    int64_t M, N, K;
+    GemmOperand a, b;
+    uint16_t *C;             // EPI_STORE_BF16: [M][ldc] bf16
+    int64_t ldc;
+    DwEpilogue dw;
+    int32_t *status;
+};
+
+// Number of CTAs the persistent GEMM uses for this problem (partials rows for EPI_DW).
+int gemm_grid(int64_t M, int64_t N, int num_sms);
+cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cudaStream_t st);
+
+// ---------------------------------------------------------------- packed 2-bit GEMV / small GEMM
+struct PackedGemvArgs {
+    const uint16_t *X;       // [N][n] bf16
+    int64_t N, m, n;
+    const uint8_t *packed;   // [m][n/4]
+    const float *A, *b;
+    uint16_t *Y;             // [N][m] bf16
+    uint16_t *Xp;            // workspace: transformed activations
+    float *corr;             // workspace: per-token constant
+    int32_t *status;
+};
+size_t packed_gemv_workspace(int64_t N, int64_t n);
+cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);
+
+}  // namespace lcq

@@ -1,0 +1,315 @@
+// C ABI of liblcq: argument validation, workspace carving and kernel dispatch.
+// See include/lcq.h for the contract of every entry point.
+#include <atomic>
+#include <cstring>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace lcq {
+
+static std::atomic<uint64_t> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+static int num_sms_current() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 1;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+static inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+static inline bool al16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+static inline cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+constexpr size_t kHeader = 256;           // status word + counter
+constexpr int kMaxGemmCtas = 1024;        // upper bound on the persistent GEMM grid
+
+struct Header {
+    int32_t status;
+    uint32_t counter;
+};
+
+static lcq_status check_common(int64_t m, int64_t n, int d) {
+    if (d != 4 && d != 8) return LCQ_ERR_UNSUPPORTED;
+    if (m < 0 || n < 0) return LCQ_ERR_SHAPE;
+    if (n % 8 != 0 || n % d != 0) return LCQ_ERR_SHAPE;
+    if (m > (int64_t(1) << 31) || n > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    return LCQ_OK;
+}
+
+// A tensor of `elems` elements: NULL allowed only when empty; must be 16-byte aligned.
+static lcq_status check_tensor(const void *p, int64_t elems, bool required = true) {
+    if (elems == 0) return LCQ_OK;
+    if (!p) return required ? LCQ_ERR_NULL : LCQ_OK;
+    if (!al16(p)) return LCQ_ERR_ALIGN;
+    return LCQ_OK;
+}
+
+static lcq_status check_ws(void *ws, size_t ws_bytes, size_t need) {
+    if (!ws) return LCQ_ERR_WORKSPACE;
+    if (!al16(ws) || (reinterpret_cast<uintptr_t>(ws) & 255u)) return LCQ_ERR_ALIGN;
+    if (ws_bytes < need) return LCQ_ERR_WORKSPACE;
+    return LCQ_OK;
+}
+
+static lcq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LCQ_OK : LCQ_ERR_CUDA; }
+
+static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste) {
+    float s = 1.0f;
+    t = 0.0f;
+    ste = LCQ_STE_IDENTITY;
+    if (o) {
+        s = o->latent_scale;
+        t = o->latent_offset;
+        ste = o->ste_mode;
+        if (o->reserved != 0) return LCQ_ERR_ARG;
+    }
+    if (!(s != 0.0f) || !isfinite(s) || !isfinite(t)) return LCQ_ERR_ARG;
+    if (ste != LCQ_STE_IDENTITY && ste != LCQ_STE_CLIPPED) return LCQ_ERR_UNSUPPORTED;
+    inv_s = 1.0f / s;
+    return LCQ_OK;
+}
+
+}  // namespace lcq
+
+using namespace lcq;
+
+#define LCQ_TRY(x)                          \
+    do {                                    \
+        lcq_status _s = (x);                \
+        if (_s != LCQ_OK) return _s;        \
+    } while (0)
+
+extern "C" {
+
+size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d) {
+    if (N < 0 || m < 0 || n < 0 || (d != 4 && d != 8)) return 0;
+    const size_t mn = static_cast<size_t>(m) * static_cast<size_t>(n);
+    switch (op) {
+        case LCQ_OP_ENCODE:
+            return kHeader + align256(sizeof(double) * 2 * 1024);
+        case LCQ_OP_LINEAR_FWD:
+            return kHeader + align256(mn * 2);
+        case LCQ_OP_LINEAR_BWD:
+            return kHeader + align256(mn * 2) + align256(sizeof(float) * kMaxGemmCtas * (d * d + d));
+        case LCQ_OP_GEMM_PACKED2B:
+            return kHeader + packed_gemv_workspace(N, n);
+        default:
+            return 0;
+    }
+}
+
+const char *lcq_status_string(lcq_status s) {
+    switch (s) {
+        case LCQ_OK: return "ok";
+        case LCQ_ERR_NULL: return "a required pointer is NULL";
+        case LCQ_ERR_SHAPE: return "invalid shape (negative size, n % d != 0 or n % 8 != 0)";
+        case LCQ_ERR_ALIGN: return "pointer not 16-byte aligned (workspace: 256-byte)";
+        case LCQ_ERR_UNSUPPORTED: return "unsupported parameter (d must be 4 or 8; STE mode)";
+        case LCQ_ERR_WORKSPACE: return "workspace missing or too small";
+        case LCQ_ERR_CUDA: return "CUDA runtime error";
+        case LCQ_ERR_SINGULAR: return "A is singular";
+        case LCQ_ERR_TIMEOUT: return "device pipeline wait timed out";
+        case LCQ_ERR_ARG: return "invalid argument";
+        default: return "unknown status";
+    }
+}
+
+uint64_t lcq_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, int clear) {
+    if (!ws || !status_out) return LCQ_ERR_NULL;
+    cudaStream_t st = as_stream(stream);
+    int32_t v = 0;
+    if (cudaMemcpyAsync(&v, ws, sizeof(int32_t), cudaMemcpyDeviceToHost, st) != cudaSuccess) return LCQ_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return LCQ_ERR_CUDA;
+    *status_out = v;
+    if (clear) {
+        if (cudaMemsetAsync(const_cast<void *>(ws), 0, sizeof(int32_t), st) != cudaSuccess) return LCQ_ERR_CUDA;
+        if (cudaStreamSynchronize(st) != cudaSuccess) return LCQ_ERR_CUDA;
+    }
+    return LCQ_OK;
+}
+
+lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, uint8_t *packed,
+                      uint8_t *codes, float *latent, double *mse, void *ws, size_t ws_bytes, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    const int64_t mn = m * n;
+    LCQ_TRY(check_tensor(W, mn));
+    if (!A || !b) return LCQ_ERR_NULL;
+    LCQ_TRY(check_tensor(packed, mn, false));
+    LCQ_TRY(check_tensor(codes, mn, false));
+    LCQ_TRY(check_tensor(latent, mn, false));
+    if (mse && (reinterpret_cast<uintptr_t>(mse) & 7u)) return LCQ_ERR_ALIGN;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_ENCODE, 0, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    if (mn == 0) {
+        if (mse) return cuda_status(cudaMemsetAsync(mse, 0, sizeof(double), st));
+        return LCQ_OK;
+    }
+    Header *h = static_cast<Header *>(ws);
+    EncodeArgs a;
+    a.W = W; a.m = m; a.n = n; a.A = A; a.b = b;
+    a.packed = packed; a.codes = codes; a.latent = latent; a.mse = mse;
+    a.partials = reinterpret_cast<double *>(static_cast<uint8_t *>(ws) + kHeader);
+    a.counter = &h->counter;
+    a.status = &h->status;
+    if (mse) LCQ_TRY(cuda_status(cudaMemsetAsync(&h->counter, 0, sizeof(uint32_t), st)));
+    return cuda_status(launch_encode(a, d, num_sms_current(), st));
+}
+
+lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const float *A, const float *b,
+                      float *W_hat_f32, uint16_t *W_hat_bf16, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    const int64_t mn = m * n;
+    if (mn == 0) return LCQ_OK;
+    LCQ_TRY(check_tensor(packed, mn));
+    if (!A || !b) return LCQ_ERR_NULL;
+    if (!W_hat_f32 && !W_hat_bf16) return LCQ_ERR_NULL;
+    LCQ_TRY(check_tensor(W_hat_f32, mn, false));
+    LCQ_TRY(check_tensor(W_hat_bf16, mn, false));
+    DecodeArgs a;
+    a.packed = packed; a.m = m; a.n = n; a.A = A; a.b = b; a.W_f32 = W_hat_f32; a.W_bf16 = W_hat_bf16;
+    return cuda_status(launch_decode(a, d, num_sms_current(), as_stream(stream)));
+}
+
+lcq_status lcq_pack2b(const uint8_t *codes, int64_t m, int64_t n, uint8_t *packed, void *stream) {
+    if (m < 0 || n < 0) return LCQ_ERR_SHAPE;
+    if (n % 4 != 0) return LCQ_ERR_SHAPE;
+    const int64_t mn = m * n;
+    if (mn == 0) return LCQ_OK;
+    LCQ_TRY(check_tensor(codes, mn));
+    LCQ_TRY(check_tensor(packed, mn));
+    return cuda_status(launch_pack2b(codes, mn, packed, num_sms_current(), as_stream(stream)));
+}
+
+lcq_status lcq_linear_fwd(const uint16_t *X, int64_t N, const float *P, int64_t m, int64_t n, int d, const float *A,
+                          const float *b, const lcq_opts *opts, uint16_t *Y, uint8_t *packed_saved, void *ws,
+                          size_t ws_bytes, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    float inv_s, t;
+    int ste;
+    LCQ_TRY(opts_of(opts, inv_s, t, ste));
+    LCQ_TRY(check_tensor(X, N * n));
+    LCQ_TRY(check_tensor(P, m * n));
+    LCQ_TRY(check_tensor(Y, N * m));
+    LCQ_TRY(check_tensor(packed_saved, m * n, false));
+    if (!A || !b) return LCQ_ERR_NULL;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_LINEAR_FWD, N, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    const int sms = num_sms_current();
+    Header *h = static_cast<Header *>(ws);
+    uint16_t *W_hat = reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(ws) + kHeader);
+    if (m * n > 0) {
+        QuantDecodeArgs q;
+        q.P = P; q.m = m; q.n = n; q.A = A; q.b = b; q.inv_s = inv_s; q.t = t;
+        q.packed = packed_saved; q.W_hat = W_hat; q.status = &h->status;
+        LCQ_TRY(cuda_status(launch_quant_decode(q, d, sms, st)));
+    }
+    if (N * m == 0) return LCQ_OK;
+    if (n == 0) return cuda_status(cudaMemsetAsync(Y, 0, sizeof(uint16_t) * N * m, st));
+    GemmProblem g;
+    std::memset(&g, 0, sizeof(g));
+    g.M = N; g.N = m; g.K = n;
+    g.a = {X, n, false};
+    g.b = {W_hat, n, false};
+    g.C = Y; g.ldc = m;
+    g.status = &h->status;
+    return cuda_status(launch_gemm(g, EPI_STORE_BF16, sms, st));
+}
+
+lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *packed_saved, const float *P, int64_t N,
+                          int64_t m, int64_t n, int d, const float *A, const float *b, const lcq_opts *opts,
+                          uint16_t *dX, float *dP, float *dA, float *db, void *ws, size_t ws_bytes, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    float inv_s, t;
+    int ste;
+    LCQ_TRY(opts_of(opts, inv_s, t, ste));
+    LCQ_TRY(check_tensor(X, N * n));
+    LCQ_TRY(check_tensor(dY, N * m));
+    LCQ_TRY(check_tensor(packed_saved, m * n));
+    LCQ_TRY(check_tensor(P, m * n, ste == LCQ_STE_CLIPPED));
+    LCQ_TRY(check_tensor(dX, N * n, false));
+    LCQ_TRY(check_tensor(dP, m * n));
+    if (!A || !b || !dA || !db) return LCQ_ERR_NULL;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_LINEAR_BWD, N, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    const int sms = num_sms_current();
+    Header *h = static_cast<Header *>(ws);
+    uint16_t *W_hat = reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(ws) + kHeader);
+    float *partials = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kHeader +
+                                                align256(static_cast<size_t>(m) * static_cast<size_t>(n) * 2));
+
+    // dX = dY W_hat
+    if (dX && N * n > 0) {
+        if (m == 0) {
+            LCQ_TRY(cuda_status(cudaMemsetAsync(dX, 0, sizeof(uint16_t) * N * n, st)));
+        } else {
+            DecodeArgs da;
+            da.packed = packed_saved; da.m = m; da.n = n; da.A = A; da.b = b; da.W_f32 = nullptr; da.W_bf16 = W_hat;
+            LCQ_TRY(cuda_status(launch_decode(da, d, sms, st)));
+            GemmProblem g;
+            std::memset(&g, 0, sizeof(g));
+            g.M = N; g.N = n; g.K = m;
+            g.a = {dY, m, false};
+            g.b = {W_hat, n, true};
+            g.C = dX; g.ldc = n;
+            g.status = &h->status;
+            LCQ_TRY(cuda_status(launch_gemm(g, EPI_STORE_BF16, sms, st)));
+        }
+    }
+    // dW_hat = dY^T X  ->  dP, dA, db
+    if (m * n == 0 || N == 0) {
+        if (m * n > 0) LCQ_TRY(cuda_status(cudaMemsetAsync(dP, 0, sizeof(float) * m * n, st)));
+        LCQ_TRY(cuda_status(cudaMemsetAsync(dA, 0, sizeof(float) * d * d, st)));
+        return cuda_status(cudaMemsetAsync(db, 0, sizeof(float) * d, st));
+    }
+    GemmProblem g;
+    std::memset(&g, 0, sizeof(g));
+    g.M = m; g.N = n; g.K = N;
+    g.a = {dY, m, true};
+    g.b = {X, n, true};
+    g.dw.packed = packed_saved;
+    g.dw.A = A;
+    g.dw.P = ste == LCQ_STE_CLIPPED ? P : nullptr;
+    g.dw.dP = dP;
+    g.dw.partials = partials;
+    g.dw.inv_s = inv_s;
+    g.dw.t = t;
+    g.dw.ste_mode = ste;
+    g.dw.d = d;
+    g.status = &h->status;
+    LCQ_TRY(cuda_status(launch_gemm(g, EPI_DW, sms, st)));
+    return cuda_status(launch_reduce_partials(partials, gemm_grid(m, n, sms), d, dA, db, st));
+}
+
+lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n, int d,
+                             const float *A, const float *b, uint16_t *Y, void *ws, size_t ws_bytes, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    LCQ_TRY(check_tensor(X, N * n));
+    LCQ_TRY(check_tensor(packed, m * n));
+    LCQ_TRY(check_tensor(Y, N * m));
+    if (!A || !b) return LCQ_ERR_NULL;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_GEMM_PACKED2B, N, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    if (N * m == 0) return LCQ_OK;
+    if (n == 0) return cuda_status(cudaMemsetAsync(Y, 0, sizeof(uint16_t) * N * m, st));
+    Header *h = static_cast<Header *>(ws);
+    uint8_t *base = static_cast<uint8_t *>(ws) + kHeader;
+    PackedGemvArgs a;
+    a.X = X; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
+    a.Xp = reinterpret_cast<uint16_t *>(base);
+    a.corr = reinterpret_cast<float *>(base + align256(static_cast<size_t>(N) * ((n + 255) / 256 * 256) * 2));
+    a.status = &h->status;
+    return cuda_status(launch_packed_gemv(a, d, num_sms_current(), st));
+}
+
+}  // extern "C"

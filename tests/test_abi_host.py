@@ -1,0 +1,112 @@
+"""Host-only checks of the C ABI: the library loads, exports every symbol include/lcq.h
+declares, and rejects bad arguments synchronously, before anything is enqueued on a GPU.
+The pointers used here are never dereferenced: validation fails first."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2606_10531_gb300 as lcq
+from paper_2606_10531_gb300 import build as lcq_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "lcq.h")
+
+OK, NULL, SHAPE, ALIGN, UNSUP, WS, ARG = 0, 1, 2, 3, 4, 5, 9
+FAKE = 0x7F0000000000          # 256-byte aligned fake device address (never dereferenced)
+
+
+@pytest.fixture(scope="module")
+def L():
+    lcq_build.build()
+    return lcq.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:[\w\s\*]+?)\b(lcq_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_six_hot_path_calls():
+    names = declared_functions()
+    for want in ("lcq_encode", "lcq_decode", "lcq_linear_fwd", "lcq_linear_bwd", "lcq_pack2b", "lcq_gemm_packed2b"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    names = declared_functions()
+    assert names, "no declarations parsed"
+    for name in names:
+        assert hasattr(L, name), name
+    assert set(names) <= set(lcq.EXPORTS)
+
+
+def test_status_strings(L):
+    for s in range(0, 10):
+        assert L.lcq_status_string(s)
+    assert L.lcq_status_string(0) == b"ok"
+
+
+def test_workspace_size_monotone_and_rejects_bad_d(L):
+    for op in (1, 2, 3, 4):
+        a = L.lcq_workspace_size(op, 16, 64, 64, 8)
+        b = L.lcq_workspace_size(op, 32, 128, 128, 8)
+        assert 0 < a <= b
+    assert L.lcq_workspace_size(2, 16, 64, 64, 5) == 0
+    assert L.lcq_workspace_size(99, 16, 64, 64, 4) == 0
+    # forward workspace holds the bf16 decoded weights
+    assert L.lcq_workspace_size(2, 1, 4096, 4096, 8) >= 4096 * 4096 * 2
+
+
+def _encode(L, W=FAKE, m=8, n=16, d=4, A=FAKE, b=FAKE, packed=FAKE, ws=FAKE, ws_bytes=1 << 20):
+    return L.lcq_encode(W, m, n, d, A, b, packed, None, None, None, ws, ws_bytes, None)
+
+
+def test_encode_validation(L):
+    assert _encode(L, d=5) == UNSUP
+    assert _encode(L, n=12) == SHAPE          # n % 8 != 0
+    assert _encode(L, m=-1) == SHAPE
+    assert _encode(L, W=None) == NULL
+    assert _encode(L, A=None) == NULL
+    assert _encode(L, W=FAKE + 4) == ALIGN
+    assert _encode(L, packed=FAKE + 8) == ALIGN
+    assert _encode(L, ws=None) == WS
+    assert _encode(L, ws_bytes=16) == WS
+    assert _encode(L, ws=FAKE + 16) == ALIGN   # workspace must be 256-byte aligned
+
+
+def test_linear_validation(L):
+    o = lcq.lcq_opts(1.0, 0.0, 0, 0)
+    big = 1 << 30
+    fwd = lambda **k: L.lcq_linear_fwd(k.get("X", FAKE), k.get("N", 4), k.get("P", FAKE), k.get("m", 8),  # noqa: E731
+                                       k.get("n", 16), k.get("d", 8), FAKE, FAKE, k.get("o", ctypes.byref(o)),
+                                       k.get("Y", FAKE), None, FAKE, k.get("ws_bytes", big), None)
+    assert fwd(d=3) == UNSUP
+    assert fwd(N=-2) == SHAPE
+    assert fwd(X=None) == NULL
+    assert fwd(Y=FAKE + 2) == ALIGN
+    assert fwd(ws_bytes=8) == WS
+    bad = lcq.lcq_opts(0.0, 0.0, 0, 0)
+    assert fwd(o=ctypes.byref(bad)) == ARG
+    bad_mode = lcq.lcq_opts(1.0, 0.0, 7, 0)
+    assert fwd(o=ctypes.byref(bad_mode)) == UNSUP
+    bwd = lambda **k: L.lcq_linear_bwd(FAKE, FAKE, FAKE, k.get("P", None), 4, 8, 16, 8, FAKE, FAKE,  # noqa: E731
+                                       k.get("o", None), None, FAKE, k.get("dA", FAKE), FAKE, FAKE, big, None)
+    clipped = lcq.lcq_opts(1.0, 0.0, 1, 0)
+    assert bwd(o=ctypes.byref(clipped)) == NULL     # CLIPPED needs P
+    assert bwd(dA=None) == NULL
+
+
+def test_packed_and_decode_validation(L):
+    assert L.lcq_pack2b(FAKE, 4, 6, FAKE, None) == SHAPE
+    assert L.lcq_pack2b(None, 4, 8, FAKE, None) == NULL
+    assert L.lcq_decode(FAKE, 4, 16, 8, FAKE, FAKE, None, None, None) == NULL
+    assert L.lcq_decode(FAKE, 4, 16, 6, FAKE, FAKE, FAKE, None, None) == UNSUP
+    assert L.lcq_gemm_packed2b(FAKE, 1, FAKE, 8, 16, 8, FAKE, FAKE, FAKE, FAKE, 8, None) == WS
+
+
+def test_empty_problems_need_no_device(L):
+    # nothing to do: returns before touching CUDA
+    assert L.lcq_decode(None, 0, 16, 8, FAKE, FAKE, None, None, None) == OK
+    assert L.lcq_pack2b(None, 0, 16, None, None) == OK

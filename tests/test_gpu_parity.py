@@ -1,0 +1,257 @@
+"""Parity of every liblcq entry point against the CPU oracle on oracle-sized inputs that
+span several tiles, chunks and ragged tails, plus the degenerate cases.
+
+Matching rules: codes and packed bytes bit-exact (encode excludes latent values within 1e-5
+of a rounding boundary and reports how many); fp32 decoded weights within 1e-6 absolute;
+bf16 outputs and all gradients within 2e-2 of max|ref| (fp64 oracle)."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2606_10531_gb300 as lcq
+from paper_2606_10531_gb300 import workloads as wl
+from tests.gpu_util import (TOL_BF16, TOL_DECODE_F32, config_A, config_b, dev, dev_bf16, empty_bf16, host_bf16,
+                            max_rel)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_10531_gb300 import build
+    build.build()
+    lcq.lib()
+
+
+def T():
+    import torch
+    return torch
+
+
+# ----------------------------------------------------------------------------- encode
+
+ENCODE_CASES = [
+    (512, 512, 4),      # the oracle-sized single layer
+    (37, 24, 4),        # ragged: 888 weights, partial 16-weight slice
+    (129, 4104, 8),     # several 16 KB chunks, ragged tail
+    (300, 1000, 8),
+    (1, 8, 8),          # one group
+]
+
+
+@pytest.mark.parametrize("m,n,d", ENCODE_CASES)
+def test_encode_matches_oracle(m, n, d):
+    torch = T()
+    rng = np.random.default_rng(1000 + m + n + d)
+    W = rng.normal(0, 0.02, (m, n)).astype(np.float32)
+    heavy = rng.random((m, n)) < 0.01
+    W[heavy] = (0.02 * rng.standard_t(4, heavy.sum())).astype(np.float32)
+    A, b = config_A(d, rng), config_b(d, rng)
+    ref = oracle.encode(W, A, b, d)
+
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, n, d)
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    codes = torch.empty((m, n), dtype=torch.uint8, device="cuda")
+    latent = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    mse = torch.empty(1, dtype=torch.float64, device="cuda")
+    lcq.lcq_encode(dev(W), dev(A), dev(b), d, ws, packed=packed, codes=codes, latent=latent, mse=mse)
+    assert lcq.lcq_device_status(ws) == 0
+
+    z = codes.cpu().numpy()
+    keep = ~ref["near"]
+    mismatch = int(np.sum((z != ref["codes"]) & keep))
+    assert mismatch == 0, f"{mismatch} codes differ away from rounding boundaries"
+    assert set(np.unique(z)) <= {0, 1, 2, 3}
+    assert np.array_equal(oracle.unpack2b(packed.cpu().numpy(), n)[keep], z[keep])
+    assert np.array_equal(oracle.unpack2b(packed.cpu().numpy(), n), z)
+    u = latent.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(u - ref["latent"]) <= 1e-5 * np.maximum(1.0, np.abs(ref["latent"])))
+    # MSE of the GPU's own codes, oracle arithmetic; and vs the oracle's MSE
+    mse_own = oracle.mse(W, z, A, b, d)
+    assert abs(mse.item() - mse_own) <= 1e-4 * mse_own
+    assert abs(mse.item() - ref["mse"]) <= 1e-4 * ref["mse"] + 1e-12
+    print(f"near-boundary codes excluded: {int(np.sum(ref['near']))} of {m * n}")
+
+
+def test_encode_nonfinite_inputs():
+    torch = T()
+    d, m, n = 8, 4, 32
+    rng = np.random.default_rng(5)
+    W = rng.normal(0, 0.02, (m, n)).astype(np.float32)
+    W[0, :3] = [np.nan, np.inf, -np.inf]
+    A, b = config_A(d, rng), config_b(d, rng)
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, n, d)
+    codes = torch.empty((m, n), dtype=torch.uint8, device="cuda")
+    lcq.lcq_encode(dev(W), dev(A), dev(b), d, ws, codes=codes)
+    ref = oracle.encode(np.where(np.isfinite(W), W, 0), A, b, d)  # rows 1.. are finite
+    z = codes.cpu().numpy()
+    assert np.array_equal(z[1:], ref["codes"][1:])
+    assert set(np.unique(z)) <= {0, 1, 2, 3}
+    # group 0 holds the non-finite values: every latent coordinate mixing them is NaN/inf
+    Ainv = np.linalg.inv(A.astype(np.float64))
+    with np.errstate(invalid="ignore"):
+        u0 = Ainv @ (W[0, :8].astype(np.float64) - b)
+    assert np.array_equal(z[0, :8], oracle.round_clamp(u0))
+
+
+def test_encode_singular_A_sets_status():
+    torch = T()
+    d, m, n = 4, 8, 16
+    A = np.eye(d, dtype=np.float32)
+    A[2] = 0.0
+    W = np.random.default_rng(0).normal(0, 0.02, (m, n)).astype(np.float32)
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, n, d)
+    codes = torch.full((m, n), 7, dtype=torch.uint8, device="cuda")
+    lcq.lcq_encode(dev(W), dev(A), dev(np.zeros(d, np.float32)), d, ws, codes=codes)
+    assert lcq.lcq_device_status(ws, clear=True) == 7   # LCQ_ERR_SINGULAR
+    assert int(codes.max()) == 0
+    assert lcq.lcq_device_status(ws) == 0
+
+
+def test_encode_empty_writes_zero_mse():
+    torch = T()
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, 0, 16, 4)
+    mse = torch.full((1,), 5.0, dtype=torch.float64, device="cuda")
+    A = dev(np.eye(4, dtype=np.float32))
+    lcq.lcq_encode(torch.empty((0, 16), device="cuda"), A, dev(np.zeros(4, np.float32)), 4, ws, mse=mse)
+    assert mse.item() == 0.0
+
+
+# ----------------------------------------------------------------------------- decode / pack
+
+@pytest.mark.parametrize("m,n,d", [(64, 512, 4), (33, 40, 8), (1, 8, 8), (257, 1032, 4)])
+def test_decode_matches_oracle(m, n, d):
+    torch = T()
+    rng = np.random.default_rng(m * 7 + n)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    ref = oracle.decode(Z, A, b, d)
+    f32 = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    h16 = empty_bf16(m, n)
+    lcq.lcq_decode(dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), W_hat_f32=f32, W_hat_bf16=h16)
+    assert np.max(np.abs(f32.cpu().numpy() - ref)) <= TOL_DECODE_F32
+    # bf16: within half a bf16 ulp of the exact value, plus the fp32 error
+    got = host_bf16(h16)
+    assert np.all(np.abs(got - ref) <= np.abs(ref) * 2.0 ** -8 + TOL_DECODE_F32)
+
+
+@pytest.mark.parametrize("m,n", [(64, 512), (3, 4), (5, 12), (17, 1028)])
+def test_pack2b_matches_oracle(m, n):
+    torch = T()
+    Z = np.random.default_rng(m + n).integers(0, 256, (m, n)).astype(np.uint8)   # high bits must be ignored
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    lcq.lcq_pack2b(dev(Z), packed)
+    assert np.array_equal(packed.cpu().numpy(), oracle.pack2b(Z & 3))
+
+
+# ----------------------------------------------------------------------------- training layer
+
+LINEAR_CASES = [
+    # N tokens, m out, n in, d
+    (64, 512, 512, 4),     # the oracle-sized layer of the workload list
+    (200, 384, 320, 8),    # 2 x 2 tiles, ragged in M and N, 5 K-blocks
+    (130, 136, 72, 4),     # ragged everywhere, K tail of 8
+    (1, 8, 8, 8),          # one token, one group
+    (520, 1024, 256, 8),   # 5 x 4 tiles with two TMEM accumulators in flight
+]
+
+
+def _linear_inputs(N, m, n, d, seed):
+    rng = np.random.default_rng(seed)
+    W = rng.normal(0, 0.02, (m, n)).astype(np.float32)
+    A, b = config_A(d, rng), config_b(d, rng)
+    P = oracle.encode(W, A, b, d)["latent"].astype(np.float32)   # proxy weights = latent of W
+    X = wl.bf16_bits(rng.normal(0, 1, (N, n)).astype(np.float32))
+    dY = wl.bf16_bits(rng.normal(0, 1, (N, m)).astype(np.float32))
+    return P, A, b, X, dY
+
+
+@pytest.mark.parametrize("N,m,n,d", LINEAR_CASES)
+@pytest.mark.parametrize("ste", ["identity", "clipped"])
+def test_linear_fwd_bwd_match_oracle(N, m, n, d, ste):
+    torch = T()
+    P, A, b, Xb, dYb = _linear_inputs(N, m, n, d, seed=N * 31 + m + n + d)
+    X, dY = wl.bf16_to_f32(Xb), wl.bf16_to_f32(dYb)
+    s, t = (1.0, 0.0) if ste == "identity" else (0.5, 0.75)
+    mode = lcq.LCQ_STE_IDENTITY if ste == "identity" else lcq.LCQ_STE_CLIPPED
+    Z = oracle.quantize(P, s, t)
+    Yref = oracle.linear_fwd(X, Z, A, b, d)
+    g = oracle.linear_bwd(X, dY, Z, A, b, d, P=P, s=s, t=t, ste=ste)
+
+    Pd, Ad, bd, Xd, dYd = dev(P), dev(A), dev(b), dev_bf16(Xb), dev_bf16(dYb)
+    Y = empty_bf16(N, m)
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    wsf = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d)
+    lcq.lcq_linear_fwd(Xd, Pd, d, Ad, bd, Y, wsf, packed_saved=packed, latent_scale=s, latent_offset=t,
+                       ste_mode=mode)
+    assert np.array_equal(packed.cpu().numpy(), oracle.pack2b(Z)), "quantized integer weights differ"
+    assert max_rel(host_bf16(Y), Yref) <= TOL_BF16
+
+    wsb = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, N, m, n, d)
+    dX = empty_bf16(N, n)
+    dP = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    dA = torch.empty((d, d), dtype=torch.float32, device="cuda")
+    db = torch.empty(d, dtype=torch.float32, device="cuda")
+    lcq.lcq_linear_bwd(Xd, dYd, packed, m, n, d, Ad, bd, dP, dA, db, wsb, dX=dX, P=Pd, latent_scale=s,
+                       latent_offset=t, ste_mode=mode)
+    assert lcq.lcq_device_status(wsb) == 0 and lcq.lcq_device_status(wsf) == 0
+    errs = {"dX": max_rel(host_bf16(dX), g["dX"]), "dP": max_rel(dP.cpu().numpy(), g["dP"]),
+            "dA": max_rel(dA.cpu().numpy(), g["dA"]), "db": max_rel(db.cpu().numpy(), g["db"])}
+    assert all(e <= TOL_BF16 for e in errs.values()), errs
+
+
+def test_linear_backward_is_bitwise_reproducible():
+    torch = T()
+    N, m, n, d = 300, 512, 256, 8
+    P, A, b, Xb, dYb = _linear_inputs(N, m, n, d, seed=77)
+    Ad, bd, Xd, dYd = dev(A), dev(b), dev_bf16(Xb), dev_bf16(dYb)
+    packed = dev(oracle.pack2b(oracle.quantize(P)))
+    wsb = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, N, m, n, d)
+    outs = []
+    for _ in range(2):
+        dP = torch.empty((m, n), dtype=torch.float32, device="cuda")
+        dA = torch.empty((d, d), dtype=torch.float32, device="cuda")
+        db = torch.empty(d, dtype=torch.float32, device="cuda")
+        lcq.lcq_linear_bwd(Xd, dYd, packed, m, n, d, Ad, bd, dP, dA, db, wsb)
+        outs.append((dP.cpu().numpy(), dA.cpu().numpy(), db.cpu().numpy()))
+    for a, c in zip(outs[0], outs[1]):
+        assert np.array_equal(a, c)
+
+
+def test_linear_empty_tokens_gives_zero_gradients():
+    torch = T()
+    m, n, d = 16, 32, 8
+    A = dev(config_A(d, np.random.default_rng(3)))
+    b = dev(np.zeros(d, np.float32))
+    X = torch.empty((0, n), dtype=torch.bfloat16, device="cuda")
+    dY = torch.empty((0, m), dtype=torch.bfloat16, device="cuda")
+    packed = torch.zeros((m, n // 4), dtype=torch.uint8, device="cuda")
+    dP = torch.full((m, n), 3.0, device="cuda")
+    dA = torch.full((d, d), 3.0, device="cuda")
+    db = torch.full((d,), 3.0, device="cuda")
+    ws = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, 0, m, n, d)
+    lcq.lcq_linear_bwd(X, dY, packed, m, n, d, A, b, dP, dA, db, ws)
+    assert float(dP.abs().max()) == 0 and float(dA.abs().max()) == 0 and float(db.abs().max()) == 0
+    Y = torch.empty((0, m), dtype=torch.bfloat16, device="cuda")
+    wsf = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, 0, m, n, d)
+    lcq.lcq_linear_fwd(X, torch.zeros((m, n), device="cuda"), d, A, b, Y, wsf)
+
+
+# ----------------------------------------------------------------------------- deployment product
+
+@pytest.mark.parametrize("N", [1, 4, 16, 17, 40])
+@pytest.mark.parametrize("m,n,d", [(200, 512, 8), (64, 1024, 4), (70, 200, 4), (8, 8, 8)])
+def test_gemm_packed2b_matches_oracle(N, m, n, d):
+    torch = T()
+    rng = np.random.default_rng(N * 1000 + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    Xb = wl.bf16_bits(rng.normal(0, 1, (N, n)).astype(np.float32))
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+    lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert max_rel(host_bf16(Y), ref) <= TOL_BF16
