@@ -1,0 +1,563 @@
+#!/usr/bin/env python
+"""Benchmark of the LC-VQ linear-layer hot path (LC-QAT, arxiv 2606.10531) on GB300.
+
+One step = one pass of the whole hot path over one Llama-3-8B-shaped decoder layer
+(7 LC-VQ linears, d = 8, 8 x 2048 tokens), per linear:
+    lcq_encode         W -> latent P, packed codes, MSE          (encode, pack)
+    lcq_linear_fwd     P -> Z -> W_hat (bf16) -> Y = X W_hat^T     (quantize, decode, GEMM)
+    lcq_linear_bwd     dX = dY W_hat, dW_hat = dY^T X -> dP, dA, db (decode, 2 GEMMs, STE epilogue)
+    lcq_gemm_packed2b  16-token deployment product from the packed codes
+`value` is the layer's fwd+bwd GEMM work (6 N m n summed over the linears) divided by the
+step time, in TFLOP/s. Separately timed in the same run: bulk encode of a Llama-3-70B layer
+(GB/s) and the packed-2-bit product of the 70B gate projection at 1/4/16 tokens (GB/s).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun each rank runs its own replica of the layer (weak scaling, no collective in
+the data path); timing is bracketed by barriers and the max over ranks is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "fwd+bwd LC-VQ linear TFLOP/s (% bf16 peak); encode/packed-decode GB/s (% HBM)"
+UNIT = "TFLOP/s"
+WORKLOAD = ("llama3-8b-layer: 7 LC-VQ linears q,o 4096x4096, k,v 1024x4096, gate,up 14336x4096, "
+            "down 4096x14336; d=8; 16384 tokens (8 x 2048)")
+GEMV_TOKENS = 16
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true", help="skip the separate encode / packed-product timings")
+    ap.add_argument("--case", choices=["linear", "encode", "gemv"], default=None,
+                    help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
+                         "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
+                         "28672 x 8192, gemv = 70B gate at 16 tokens")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm": float(j["hbm_gbs"]), "bf16": float(j["bf16_tflops"]),
+                "bf16_sustained": float(j.get("bf16_tflops_sustained", j["bf16_tflops"])), "src": "measured"}
+    return {"hbm": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "src": "fallback"}
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(device_index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                rows.append((float(f[0]), float(f[1]), f[4:8]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i in range(4) if r[i].lower() == "active"})
+        loaded = [r[0] for r in rows if r[0] > 0.5 * r[1]] or [r[0] for r in rows]
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- layer buffers
+
+class Linear:
+    def __init__(self, torch, lcq, wl, mx, seed, index, device, with_inputs=True):
+        self.mx = mx
+        m, n, d, N = mx.m, mx.n, mx.d, mx.N
+        self.m, self.n, self.d, self.N = m, n, d, N
+        self.A = wl.torch_A(torch, mx, seed, index, device).contiguous()
+        self.b = wl.torch_b(torch, mx, seed, index, device).contiguous()
+        self.W = wl.torch_W(torch, mx, seed, index, device)
+        self.X = wl.torch_X(torch, mx, seed, index, device)
+        self.dY = wl.torch_dY(torch, mx, seed, index, device)
+        self.Xg = self.X[:GEMV_TOKENS].contiguous()
+        f32, bf16, u8 = torch.float32, torch.bfloat16, torch.uint8
+        self.P = torch.empty((m, n), dtype=f32, device=device)
+        self.enc_packed = torch.empty((m, n // 4), dtype=u8, device=device)
+        self.saved = torch.empty((m, n // 4), dtype=u8, device=device)
+        self.mse = torch.empty(1, dtype=torch.float64, device=device)
+        self.Y = torch.empty((N, m), dtype=bf16, device=device)
+        self.dX = torch.empty((N, n), dtype=bf16, device=device)
+        self.dP = torch.empty((m, n), dtype=f32, device=device)
+        self.dA = torch.empty((d, d), dtype=f32, device=device)
+        self.db = torch.empty(d, dtype=f32, device=device)
+        self.Yg = torch.empty((GEMV_TOKENS, m), dtype=bf16, device=device)
+        self.ws_e = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, n, d, device)
+        self.ws_f = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d, device)
+        self.ws_b = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, N, m, n, d, device)
+        self.ws_g = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, GEMV_TOKENS, m, n, d, device)
+
+    def flops(self):
+        return 6.0 * self.N * self.m * self.n
+
+    def step(self, lcq):
+        d = self.d
+        lcq.lcq_encode(self.W, self.A, self.b, d, self.ws_e, packed=self.enc_packed, latent=self.P, mse=self.mse)
+        lcq.lcq_linear_fwd(self.X, self.P, d, self.A, self.b, self.Y, self.ws_f, packed_saved=self.saved)
+        lcq.lcq_linear_bwd(self.X, self.dY, self.saved, self.m, self.n, d, self.A, self.b, self.dP, self.dA, self.db,
+                           self.ws_b, dX=self.dX)
+        lcq.lcq_gemm_packed2b(self.Xg, self.saved, self.n, d, self.A, self.b, self.Yg, self.ws_g)
+
+    def statuses(self, lcq):
+        return [lcq.lcq_device_status(w) for w in (self.ws_e, self.ws_f, self.ws_b, self.ws_g)]
+
+
+def gemm_flops_per_kind(layer):
+    """Algorithmic flops of every tensor-core GEMM launch of one step, by launch kind."""
+    return {"gemm_fwd": sum(2.0 * L.N * L.m * L.n for L in layer),
+            "gemm_dx": sum(2.0 * L.N * L.m * L.n for L in layer),
+            "gemm_dw": sum(2.0 * L.N * L.m * L.n for L in layer)}
+
+
+def traffic_from_profile(kernel_src: str):
+    """Per-launch DRAM traffic of the GEMM from the committed ncu summary, or None if the kernel
+    source changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "gemm_tc_llama3_8b.txt")
+    if not os.path.exists(p):
+        return None
+    want = hashlib.sha256(open(kernel_src, "rb").read()).hexdigest()[:16]
+    src_hash, traffic = None, None
+    for line in open(p):
+        if line.startswith("source_sha256_16:"):
+            src_hash = line.split(":", 1)[1].strip()
+        if line.startswith("dram_bytes_per_launch_full_size:"):
+            traffic = float(line.split(":", 1)[1].strip())
+    return traffic if (src_hash == want and traffic) else None
+
+
+# ----------------------------------------------------------------------------- extras
+
+def time_encode_70b(torch, lcq, wl, seed, device, pk):
+    """Bulk encode of all linears of a Llama-3-70B layer (d=8): packed codes + MSE."""
+    mats = wl.llama3_70b_layer_encode()
+    bufs = []
+    for i, mx in enumerate(mats):
+        W = wl.torch_W(torch, mx, seed + 1000, i, device)
+        A = wl.torch_A(torch, mx, seed + 1000, i, device).contiguous()
+        b = wl.torch_b(torch, mx, seed + 1000, i, device).contiguous()
+        bufs.append((mx, W, A, b, torch.empty((mx.m, mx.n // 4), dtype=torch.uint8, device=device),
+                     torch.empty(1, dtype=torch.float64, device=device),
+                     lcq.workspace(lcq.LCQ_OP_ENCODE, 0, mx.m, mx.n, mx.d, device)))
+
+    def run():
+        for mx, W, A, b, pk_, mse, ws in bufs:
+            lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
+
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    iters = 10
+    e0.record()
+    for _ in range(iters):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    t = e0.elapsed_time(e1) / 1e3 / iters
+    weights = sum(mx.m * mx.n for mx in mats)
+    gbs = weights * 4.25 / t / 1e9
+    for *_, ws in bufs:
+        assert lcq.lcq_device_status(ws) == 0
+    mses = [float(x[5].item()) for x in bufs]
+    del bufs
+    return {"workload": "llama3-70b-layer bulk encode: q,o 8192x8192, k,v 1024x8192, gate,up 28672x8192, "
+                        "down 8192x28672; d=8; W ~N(0,0.015) + 0.1% Student-t(4); packed codes + MSE",
+            "weights": weights, "ms": t * 1e3, "GB/s": gbs, "bytes_per_weight": 4.25,
+            "frac_hbm": gbs / pk["hbm"], "mse": mses, "l2": "inputs larger than L2 (3.4 GB per pass)"}
+
+
+def time_gemv_70b(torch, lcq, wl, seed, device, pk):
+    """Packed 2-bit product of the Llama-3-70B gate projection (28672 x 8192, d = 8) at 1/4/16 tokens,
+    L2 flushed before every timed launch."""
+    mx0 = wl.llama3_70b_gate_decode(1)[0]
+    packed = wl.torch_packed_codes(torch, mx0, seed + 2000, 0, device)
+    A = wl.torch_A(torch, mx0, seed + 2000, 0, device).contiguous()
+    b = wl.torch_b(torch, mx0, seed + 2000, 0, device).contiguous()
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=device)
+    out = {}
+    for B in (1, 4, 16):
+        X = wl.torch_X(torch, wl.llama3_70b_gate_decode(B)[0], seed + 2000, B, device)
+        Y = torch.empty((B, mx0.m), dtype=torch.bfloat16, device=device)
+        ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, B, mx0.m, mx0.n, mx0.d, device)
+        times = []
+        for it in range(23):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            lcq.lcq_gemm_packed2b(X, packed, mx0.n, mx0.d, A, b, Y, ws)
+            e1.record()
+            torch.cuda.synchronize()
+            if it >= 3:
+                times.append(e0.elapsed_time(e1) * 1e-3)
+        assert lcq.lcq_device_status(ws) == 0
+        t = statistics.median(times)
+        nbytes = mx0.m * mx0.n / 4 + 2 * B * mx0.n + 2 * B * mx0.m
+        out[f"B{B}"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
+                        "bytes": nbytes}
+    out["workload"] = "llama3-70b gate 28672x8192 packed 2-bit, d=8, bf16 activations; L2 flushed per launch"
+    return out
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+
+def oracle_sample(seed, budget_s, tokens=64, max_linears=7):
+    """The CPU oracle doing the same step (encode, fwd, bwd, packed product) on a bounded sample:
+    all weights of successive linears of the layer, `tokens` of the 16384 tokens."""
+    import numpy as np
+
+    import oracle
+    from paper_2606_10531_gb300 import workloads as wl
+    mats = wl.llama3_8b_layer()
+    flops, spent, used = 0.0, 0.0, []
+    for i, mx in enumerate(mats[:max_linears]):
+        W = wl.draw_W(mx, seed, i)
+        A, b = wl.draw_A(mx, seed, i), wl.draw_b(mx, seed, i)
+        X = wl.bf16_to_f32(wl.draw_X(mx, seed, i, tokens=tokens))
+        dY = wl.bf16_to_f32(wl.draw_dY(mx, seed, i, tokens=tokens))
+        t0 = time.perf_counter()
+        enc = oracle.encode(W, A, b, mx.d)
+        Z = oracle.quantize(enc["latent"].astype(np.float32))
+        oracle.linear_fwd(X, Z, A, b, mx.d)
+        oracle.linear_bwd(X, dY, Z, A, b, mx.d)
+        oracle.gemm_packed2b(X[:GEMV_TOKENS], oracle.pack2b(Z), A, b, mx.d, mx.n)
+        spent += time.perf_counter() - t0
+        flops += 6.0 * tokens * mx.m * mx.n
+        used.append(mx.name)
+        if spent >= budget_s:
+            break
+    return flops / spent / 1e12, spent, used
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ----------------------------------------------------------------------------- main
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        return reference_arm(args, world, rank)
+    if args.case:
+        return profile_case(args)
+
+    import torch
+    import paper_2606_10531_gb300 as lcq
+    from paper_2606_10531_gb300 import build as lcq_build
+    from paper_2606_10531_gb300 import workloads as wl
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=device)
+    lcq_build.build()
+    lcq.lib()
+    pk = peaks()
+
+    layer = [Linear(torch, lcq, wl, mx, args.seed + 7919 * rank, i, device) for i, mx in enumerate(wl.llama3_8b_layer())]
+    step_flops = sum(L.flops() for L in layer)
+
+    def step():
+        for L in layer:
+            L.step(lcq)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    for L in layer:
+        assert L.statuses(lcq) == [0, 0, 0, 0]
+    barrier()
+
+    clocks = ClockSampler(local)
+    time.sleep(0.5)          # let the sampler start before the timed region
+    lcq.lcq_trace_enable(True)
+    launches0 = lcq.lcq_launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    barrier()
+    launches = lcq.lcq_launch_count() - launches0
+    lcq.lcq_trace_enable(False)
+    clk = clocks.stop()
+    elapsed = e0.elapsed_time(e1) / 1e3
+    if world > 1:
+        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed = float(t.item())
+    trace = lcq.lcq_trace_read()
+    for L in layer:
+        assert L.statuses(lcq) == [0, 0, 0, 0]
+
+    value = step_flops * args.steps * world / elapsed / 1e12
+    ms_per_step = elapsed / args.steps * 1e3
+
+    # dominant kernel: the tensor-core GEMM (all three launch kinds share one kernel template)
+    fl = gemm_flops_per_kind(layer)
+    g_launch = sum(trace.get(k, (0, 0.0))[0] for k in fl)
+    g_ms = sum(trace.get(k, (0, 0.0))[1] for k in fl)
+    g_flops = sum(fl.values()) * args.steps
+    achieved = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else None
+    per_launch_flops = g_flops / g_launch if g_launch else None
+    traffic = traffic_from_profile(os.path.join(ROOT, "paper_2606_10531_gb300", "csrc", "gemm_tc.cu"))
+    total_trace_ms = sum(v[1] for v in trace.values())
+    roofline = {"kernel": "gemm_tc (tcgen05/TMEM, TMA) fwd + dX + dW launches", "bound": "tensor",
+                "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+                "frac": (achieved / pk["bf16_sustained"]) if achieved else None,
+                "frac_of_burst_peak": (achieved / pk["bf16"]) if achieved else None,
+                "peak_kind": f"bf16_tflops_sustained ({pk['src']}); kernel timed inside a long step",
+                "traffic": traffic, "flops_per_launch": per_launch_flops, "launches": g_launch,
+                "share_of_kernel_time": g_ms / total_trace_ms if total_trace_ms else None}
+    breakdown = {k: {"launches": v[0], "ms_per_step": v[1] / args.steps} for k, v in trace.items()}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(args.warmup, 3), "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded device generators with the workload's shapes and distributions",
+            "config": {"workload": WORKLOAD, "tokens": 16384, "d": 8, "linears": 7,
+                       "step_flops": step_flops, "l2": "inputs larger than L2 (129 MB); no flush",
+                       "parallelism": f"replicas x{world} (one layer per rank)" if world > 1 else "single GPU",
+                       "precision": "bf16 tensor-core GEMMs, fp32 accumulate; fp32 encode/decode/STE epilogue"},
+            "frac_bf16_peak": value / pk["bf16"], "roofline": roofline, "breakdown": breakdown,
+            "gpu_launches": launches, "clocks": clk}
+
+    if rank == 0 and not args.no_extras:
+        del layer
+        torch.cuda.empty_cache()
+        line["encode"] = time_encode_70b(torch, lcq, wl, args.seed, device, pk)
+        line["packed_decode"] = time_gemv_70b(torch, lcq, wl, args.seed, device, pk)
+        torch.cuda.empty_cache()
+        layer = None
+
+    if not args.no_e2e:
+        line["e2e"] = e2e_arm(torch, lcq, wl, args, device, world, rank)
+
+    if rank == 0 and not args.no_cpu_baseline:
+        v, spent, used = oracle_sample(args.seed, budget_s=10.0)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                "sample": f"oracle step (encode, fwd, bwd, packed product) on linears {used} with "
+                                          f"64 of 16384 tokens; {spent:.1f} s of CPU work"}
+    if world > 1:
+        torch.distributed.barrier()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def e2e_arm(torch, lcq, wl, args, device, world, rank):
+    """Same step through the public API with the step's inputs in pinned host memory: every step copies
+    W, X, dY host->device and reads dA, db, MSE and the packed-product output back to the host."""
+    layer = [Linear(torch, lcq, wl, mx, args.seed + 7919 * rank, i, device)
+             for i, mx in enumerate(wl.llama3_8b_layer())]
+    host = []
+    for L in layer:
+        h = {"W": L.W.cpu().pin_memory(), "X": L.X.cpu().pin_memory(), "dY": L.dY.cpu().pin_memory(),
+             "dA": torch.empty_like(L.dA, device="cpu").pin_memory(),
+             "db": torch.empty_like(L.db, device="cpu").pin_memory(),
+             "mse": torch.empty_like(L.mse, device="cpu").pin_memory(),
+             "Yg": torch.empty_like(L.Yg, device="cpu").pin_memory()}
+        host.append(h)
+    h2d = sum(h["W"].numel() * 4 + h["X"].numel() * 2 + h["dY"].numel() * 2 for h in host)
+    d2h = sum(h["dA"].numel() * 4 + h["db"].numel() * 4 + 8 + h["Yg"].numel() * 2 for h in host)
+
+    def step():
+        for L, h in zip(layer, host):
+            L.W.copy_(h["W"], non_blocking=True)
+            L.X.copy_(h["X"], non_blocking=True)
+            L.dY.copy_(h["dY"], non_blocking=True)
+            L.Xg.copy_(L.X[:GEMV_TOKENS])
+            L.step(lcq)
+            h["dA"].copy_(L.dA, non_blocking=True)
+            h["db"].copy_(L.db, non_blocking=True)
+            h["mse"].copy_(L.mse, non_blocking=True)
+            h["Yg"].copy_(L.Yg, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize()
+    el = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([el], device=device, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        el = float(t.item())
+    flops = sum(L.flops() for L in layer) * args.steps * world
+    del layer, host
+    torch.cuda.empty_cache()
+    return {"value": flops / el / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": el / args.steps * 1e3, "api": "paper_2606_10531_gb300 ctypes binding of liblcq"}
+
+
+def profile_case(args):
+    """One call in a loop on a small case (for ncu captures); prints a one-line summary."""
+    import torch
+    import paper_2606_10531_gb300 as lcq
+    from paper_2606_10531_gb300 import build as lcq_build
+    from paper_2606_10531_gb300 import workloads as wl
+    lcq_build.build()
+    device = torch.device("cuda", 0)
+    if args.case == "linear":
+        L = Linear(torch, lcq, wl, wl.llama3_8b_layer()[0], args.seed, 0, device)
+        lcq.lcq_encode(L.W, L.A, L.b, L.d, L.ws_e, latent=L.P)
+
+        def run():
+            lcq.lcq_linear_fwd(L.X, L.P, L.d, L.A, L.b, L.Y, L.ws_f, packed_saved=L.saved)
+            lcq.lcq_linear_bwd(L.X, L.dY, L.saved, L.m, L.n, L.d, L.A, L.b, L.dP, L.dA, L.db, L.ws_b, dX=L.dX)
+        wss = [L.ws_e, L.ws_f, L.ws_b]
+    elif args.case == "encode":
+        mx = wl.llama3_70b_layer_encode()[4]
+        W, A, b = (wl.torch_W(torch, mx, args.seed, 4, device), wl.torch_A(torch, mx, args.seed, 4, device),
+                   wl.torch_b(torch, mx, args.seed, 4, device))
+        pk_ = torch.empty((mx.m, mx.n // 4), dtype=torch.uint8, device=device)
+        mse = torch.empty(1, dtype=torch.float64, device=device)
+        ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, mx.m, mx.n, mx.d, device)
+
+        def run():
+            lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
+        wss = [ws]
+    else:
+        mx = wl.llama3_70b_gate_decode(GEMV_TOKENS)[0]
+        packed = wl.torch_packed_codes(torch, mx, args.seed, 0, device)
+        A, b = wl.torch_A(torch, mx, args.seed, 0, device), wl.torch_b(torch, mx, args.seed, 0, device)
+        X = wl.torch_X(torch, mx, args.seed, 0, device)
+        Y = torch.empty((mx.N, mx.m), dtype=torch.bfloat16, device=device)
+        ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, mx.N, mx.m, mx.n, mx.d, device)
+
+        def run():
+            lcq.lcq_gemm_packed2b(X, packed, mx.n, mx.d, A, b, Y, ws)
+        wss = [ws]
+    for _ in range(args.warmup + args.steps):
+        run()
+    torch.cuda.synchronize()
+    print(json.dumps({"case": args.case, "iterations": args.warmup + args.steps,
+                      "status": [lcq.lcq_device_status(w) for w in wss]}), flush=True)
+
+
+def reference_arm(args, world, rank):
+    """The CPU oracle as the reference implementation: each step is a bounded sample of the same workload
+    (one linear of the layer, 32 of its 16384 tokens, rotating through the linears)."""
+    if rank != 0:
+        return
+    import numpy as np
+
+    import oracle
+    from paper_2606_10531_gb300 import workloads as wl
+    mats = wl.llama3_8b_layer()
+    tokens = 32
+    cache = {}
+
+    def inputs(i):
+        if i not in cache:
+            mx = mats[i]
+            cache[i] = (mx, wl.draw_W(mx, args.seed, i), wl.draw_A(mx, args.seed, i), wl.draw_b(mx, args.seed, i),
+                        wl.bf16_to_f32(wl.draw_X(mx, args.seed, i, tokens=tokens)),
+                        wl.bf16_to_f32(wl.draw_dY(mx, args.seed, i, tokens=tokens)))
+        return cache[i]
+
+    order = [0, 1, 2, 3]     # q, k, v, o: keeps each step to seconds on the host cores
+
+    def step(k):
+        mx, W, A, b, X, dY = inputs(order[k % len(order)])
+        t0 = time.perf_counter()
+        enc = oracle.encode(W, A, b, mx.d)
+        Z = oracle.quantize(enc["latent"].astype(np.float32))
+        oracle.linear_fwd(X, Z, A, b, mx.d)
+        oracle.linear_bwd(X, dY, Z, A, b, mx.d)
+        oracle.gemm_packed2b(X[:GEMV_TOKENS], oracle.pack2b(Z), A, b, mx.d, mx.n)
+        return time.perf_counter() - t0, 6.0 * tokens * mx.m * mx.n
+
+    for k in range(max(args.warmup, 3)):
+        step(k)
+    tot_t, tot_f = 0.0, 0.0
+    for k in range(args.steps):
+        t, f = step(k)
+        tot_t += t
+        tot_f += f
+    value = tot_f / tot_t / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": tot_t / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic: seeded NumPy draws with the workload's shapes and distributions",
+            "config": {"workload": WORKLOAD, "tokens": 16384, "d": 8, "linears": 7},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                             "sample": f"per step one of the q,k,v,o linears (all weights) with {tokens} of 16384 "
+                                       "tokens: encode, fwd, bwd, packed product"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -178,6 +178,35 @@ const char *lcq_status_string(lcq_status s);
 /* Number of kernels this library has launched in the calling process. */
 uint64_t lcq_launch_count(void);
 
+/*
+ * Kernel tracing with CUDA events (measurement support; not part of the
+ * paper's method). While enabled, every kernel the library launches is
+ * bracketed by two events recorded on the launching stream; records beyond
+ * LCQ_TRACE_CAPACITY are dropped. lcq_trace_enable(1) clears the records and
+ * starts recording, lcq_trace_enable(0) stops. Not thread-safe: trace from one
+ * host thread at a time.
+ */
+#define LCQ_TRACE_CAPACITY 4096
+typedef enum lcq_kernel_kind {
+    LCQ_K_ENCODE = 0,        /* encode stream kernel                         */
+    LCQ_K_QUANT_DECODE = 1,  /* forward prologue: quantize + decode to bf16  */
+    LCQ_K_DECODE = 2,        /* decode packed codes                          */
+    LCQ_K_PACK = 3,          /* pack one-code-per-byte codes                 */
+    LCQ_K_GEMM_FWD = 4,      /* tensor-core GEMM, Y = X W_hat^T              */
+    LCQ_K_GEMM_DX = 5,       /* tensor-core GEMM, dX = dY W_hat              */
+    LCQ_K_GEMM_DW = 6,       /* tensor-core GEMM, dW_hat = dY^T X + dP/dA/db */
+    LCQ_K_REDUCE = 7,        /* fixed-order dA/db reduction                  */
+    LCQ_K_GEMV_PREP = 8,     /* packed product: activation transform         */
+    LCQ_K_GEMV = 9,          /* packed product: main kernel                  */
+    LCQ_K_NUM_KINDS = 10
+} lcq_kernel_kind;
+lcq_status lcq_trace_enable(int on);
+/*
+ * Synchronise on the recorded events and report, for one kernel kind, the
+ * number of recorded launches and the sum of their durations in milliseconds.
+ */
+lcq_status lcq_trace_read(int kind, uint64_t *launches, double *total_ms);
+
 #ifdef __cplusplus
 }
 #endif

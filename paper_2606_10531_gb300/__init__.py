@@ -23,7 +23,10 @@ LCQ_STE_IDENTITY, LCQ_STE_CLIPPED = 0, 1
 
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
-           "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count")
+           "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
+           "lcq_trace_read")
+KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
+                "gemv_prep", "gemv")
 
 
 class LCQError(RuntimeError):
@@ -53,6 +56,8 @@ _SIG = {
     "lcq_device_status": (ctypes.c_int, [_P, _P, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]),
     "lcq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "lcq_launch_count": (ctypes.c_uint64, []),
+    "lcq_trace_enable": (ctypes.c_int, [ctypes.c_int]),
+    "lcq_trace_read": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_double)]),
 }
 
 
@@ -168,3 +173,18 @@ def lcq_device_status(ws, clear: bool = False, stream=None) -> int:
 
 def lcq_launch_count() -> int:
     return int(lib().lcq_launch_count())
+
+
+def lcq_trace_enable(on: bool = True):
+    _check(lib().lcq_trace_enable(int(bool(on))), "lcq_trace_enable")
+
+
+def lcq_trace_read() -> dict:
+    """{kernel kind: (launches, total milliseconds)} of the events recorded since tracing was enabled."""
+    out = {}
+    for k, name in enumerate(KERNEL_KINDS):
+        cnt, ms = ctypes.c_uint64(0), ctypes.c_double(0.0)
+        _check(lib().lcq_trace_read(k, ctypes.byref(cnt), ctypes.byref(ms)), "lcq_trace_read")
+        if cnt.value:
+            out[name] = (int(cnt.value), float(ms.value))
+    return out

@@ -330,12 +330,14 @@ int gemm_grid(int64_t M, int64_t N, int num_sms) {
 
 template <int EPI, int D, bool A_MN, bool B_MN>
 static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, const GemmParams &gp, int grid,
-                              cudaStream_t st) {
+                              int trace_kind, cudaStream_t st) {
     auto k = gemm_kernel<EPI, D, A_MN, B_MN>;
     const int smem = static_cast<int>(sizeof(GemmSmem) + 1024);
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
+    trace_begin(trace_kind, st);
     k<<<grid, kGemmThreads, smem, st>>>(ma, mb, gp);
+    trace_end(trace_kind, st);
     count_launch();
     return cudaGetLastError();
 }
@@ -353,14 +355,14 @@ cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cud
     gp.status = p.status;
     const int grid = gemm_grid(p.M, p.N, num_sms);
     if (epi == EPI_STORE_BF16) {
-        if (!p.a.mn_major && !p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, false>(ma, mb, gp, grid, st);
-        if (!p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, true>(ma, mb, gp, grid, st);
-        if (p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, true, true>(ma, mb, gp, grid, st);
-        return launch_one<EPI_STORE_BF16, 1, true, false>(ma, mb, gp, grid, st);
+        if (!p.a.mn_major && !p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, false>(ma, mb, gp, grid, p.trace_kind, st);
+        if (!p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, true>(ma, mb, gp, grid, p.trace_kind, st);
+        if (p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, true, true>(ma, mb, gp, grid, p.trace_kind, st);
+        return launch_one<EPI_STORE_BF16, 1, true, false>(ma, mb, gp, grid, p.trace_kind, st);
     }
     if (!(p.a.mn_major && p.b.mn_major)) return cudaErrorInvalidValue;
-    if (p.dw.d == 4) return launch_one<EPI_DW, 4, true, true>(ma, mb, gp, grid, st);
-    return launch_one<EPI_DW, 8, true, true>(ma, mb, gp, grid, st);
+    if (p.dw.d == 4) return launch_one<EPI_DW, 4, true, true>(ma, mb, gp, grid, p.trace_kind, st);
+    return launch_one<EPI_DW, 8, true, true>(ma, mb, gp, grid, p.trace_kind, st);
 }
 
 }  // namespace lcq

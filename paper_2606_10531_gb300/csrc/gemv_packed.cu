@@ -248,15 +248,19 @@ size_t packed_gemv_workspace(int64_t N, int64_t n) {
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st) {
     (void)num_sms;
     const int64_t npad = gemv_npad(a.n);
+    trace_begin(LCQ_K_GEMV_PREP, st);
     if (d == 4) gemv_prep_kernel<4><<<static_cast<unsigned>(a.N), 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
     else gemv_prep_kernel<8><<<static_cast<unsigned>(a.N), 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
+    trace_end(LCQ_K_GEMV_PREP, st);
     count_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>((a.m + kGemvRows - 1) / kGemvRows), static_cast<unsigned>((a.N + 15) / 16));
     const bool vec = (a.n % 64) == 0;
+    trace_begin(LCQ_K_GEMV, st);
     if (vec) packed_gemv_kernel<true><<<grid, 32 * kGemvWarps, 0, st>>>(a.packed, a.m, a.n, a.N, a.Xp, npad, a.corr, a.Y);
     else packed_gemv_kernel<false><<<grid, 32 * kGemvWarps, 0, st>>>(a.packed, a.m, a.n, a.N, a.Xp, npad, a.corr, a.Y);
+    trace_end(LCQ_K_GEMV, st);
     count_launch();
     return cudaGetLastError();
 }

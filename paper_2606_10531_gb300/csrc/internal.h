@@ -8,6 +8,9 @@
 namespace lcq {
 
 void count_launch();
+// Record the start / end event of a kernel of the given lcq_kernel_kind on `st` (no-op unless tracing).
+void trace_begin(int kind, cudaStream_t st);
+void trace_end(int kind, cudaStream_t st);
 
 struct EncodeArgs {
     const float *W;
@@ -76,6 +79,7 @@ struct GemmProblem {
     int64_t ldc;
     DwEpilogue dw;
     int32_t *status;
+    int trace_kind;          // lcq_kernel_kind recorded by the tracer
 };
 
 // Number of CTAs the persistent GEMM uses for this problem (partials rows for EPI_DW).

@@ -481,7 +481,9 @@ cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t 
     else k = mse ? encode_kernel<8, true> : encode_kernel<8, false>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
+    trace_begin(LCQ_K_ENCODE, st);
     k<<<grid, kStreamThreads, smem, st>>>(a);
+    trace_end(LCQ_K_ENCODE, st);
     count_launch();
     return cudaGetLastError();
 }
@@ -493,7 +495,9 @@ cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cu
     void (*k)(QuantDecodeArgs) = d == 4 ? quant_decode_kernel<4> : quant_decode_kernel<8>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
+    trace_begin(LCQ_K_QUANT_DECODE, st);
     k<<<grid, kStreamThreads, smem, st>>>(a);
+    trace_end(LCQ_K_QUANT_DECODE, st);
     count_launch();
     return cudaGetLastError();
 }
@@ -503,8 +507,10 @@ cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t 
     int64_t grid = (nslices + 255) / 256;
     if (grid > 8LL * num_sms) grid = 8LL * num_sms;
     if (grid < 1) grid = 1;
+    trace_begin(LCQ_K_DECODE, st);
     if (d == 4) decode_kernel<4><<<static_cast<int>(grid), 256, 0, st>>>(a);
     else decode_kernel<8><<<static_cast<int>(grid), 256, 0, st>>>(a);
+    trace_end(LCQ_K_DECODE, st);
     count_launch();
     return cudaGetLastError();
 }
@@ -514,13 +520,17 @@ cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, 
     int64_t grid = (nslices + 255) / 256;
     if (grid > 8LL * num_sms) grid = 8LL * num_sms;
     if (grid < 1) grid = 1;
+    trace_begin(LCQ_K_PACK, st);
     pack2b_kernel<<<static_cast<int>(grid), 256, 0, st>>>(codes, total, packed);
+    trace_end(LCQ_K_PACK, st);
     count_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_reduce_partials(const float *partials, int nparts, int d, float *dA, float *db, cudaStream_t st) {
+    trace_begin(LCQ_K_REDUCE, st);
     reduce_partials_kernel<<<1, 128, 0, st>>>(partials, nparts, d, dA, db);
+    trace_end(LCQ_K_REDUCE, st);
     count_launch();
     return cudaGetLastError();
 }

@@ -11,6 +11,38 @@ namespace lcq {
 static std::atomic<uint64_t> g_launches{0};
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+// ---------------------------------------------------------------- CUDA-event kernel tracing
+struct TraceRec {
+    int kind;
+    cudaEvent_t start, stop;
+};
+static bool g_trace_on = false;
+static int g_trace_n = 0;
+static TraceRec g_trace[LCQ_TRACE_CAPACITY];
+static bool g_trace_pool_ready = false;
+
+static bool trace_pool() {
+    if (g_trace_pool_ready) return true;
+    for (int i = 0; i < LCQ_TRACE_CAPACITY; ++i) {
+        if (cudaEventCreate(&g_trace[i].start) != cudaSuccess) return false;
+        if (cudaEventCreate(&g_trace[i].stop) != cudaSuccess) return false;
+    }
+    g_trace_pool_ready = true;
+    return true;
+}
+
+void trace_begin(int kind, cudaStream_t st) {
+    if (!g_trace_on || g_trace_n >= LCQ_TRACE_CAPACITY) return;
+    g_trace[g_trace_n].kind = kind;
+    cudaEventRecord(g_trace[g_trace_n].start, st);
+}
+
+void trace_end(int kind, cudaStream_t st) {
+    if (!g_trace_on || g_trace_n >= LCQ_TRACE_CAPACITY || g_trace[g_trace_n].kind != kind) return;
+    cudaEventRecord(g_trace[g_trace_n].stop, st);
+    ++g_trace_n;
+}
+
 static int num_sms_current() {
     static int cache[64] = {0};
     int dev = 0;
@@ -122,6 +154,35 @@ const char *lcq_status_string(lcq_status s) {
 
 uint64_t lcq_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+lcq_status lcq_trace_enable(int on) {
+    if (on) {
+        if (!trace_pool()) return LCQ_ERR_CUDA;
+        g_trace_n = 0;
+        g_trace_on = true;
+    } else {
+        g_trace_on = false;
+    }
+    return LCQ_OK;
+}
+
+lcq_status lcq_trace_read(int kind, uint64_t *launches, double *total_ms) {
+    if (!launches || !total_ms) return LCQ_ERR_NULL;
+    if (kind < 0 || kind >= LCQ_K_NUM_KINDS) return LCQ_ERR_ARG;
+    uint64_t cnt = 0;
+    double tot = 0.0;
+    for (int i = 0; i < g_trace_n; ++i) {
+        if (g_trace[i].kind != kind) continue;
+        if (cudaEventSynchronize(g_trace[i].stop) != cudaSuccess) return LCQ_ERR_CUDA;
+        float ms = 0.0f;
+        if (cudaEventElapsedTime(&ms, g_trace[i].start, g_trace[i].stop) != cudaSuccess) return LCQ_ERR_CUDA;
+        tot += ms;
+        ++cnt;
+    }
+    *launches = cnt;
+    *total_ms = tot;
+    return LCQ_OK;
+}
+
 lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, int clear) {
     if (!ws || !status_out) return LCQ_ERR_NULL;
     cudaStream_t st = as_stream(stream);
@@ -221,6 +282,7 @@ lcq_status lcq_linear_fwd(const uint16_t *X, int64_t N, const float *P, int64_t 
     g.b = {W_hat, n, false};
     g.C = Y; g.ldc = m;
     g.status = &h->status;
+    g.trace_kind = LCQ_K_GEMM_FWD;
     return cuda_status(launch_gemm(g, EPI_STORE_BF16, sms, st));
 }
 
@@ -262,6 +324,7 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
             g.b = {W_hat, n, true};
             g.C = dX; g.ldc = n;
             g.status = &h->status;
+            g.trace_kind = LCQ_K_GEMM_DX;
             LCQ_TRY(cuda_status(launch_gemm(g, EPI_STORE_BF16, sms, st)));
         }
     }
@@ -286,6 +349,7 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
     g.dw.ste_mode = ste;
     g.dw.d = d;
     g.status = &h->status;
+    g.trace_kind = LCQ_K_GEMM_DW;
     LCQ_TRY(cuda_status(launch_gemm(g, EPI_DW, sms, st)));
     return cuda_status(launch_reduce_partials(partials, gemm_grid(m, n, sms), d, dA, db, st));
 }
