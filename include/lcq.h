@@ -50,7 +50,8 @@ typedef enum lcq_status {
     LCQ_ERR_CUDA = 6,        /* a CUDA runtime call or kernel launch failed             */
     LCQ_ERR_SINGULAR = 7,    /* device-detected: A is not invertible (encode)           */
     LCQ_ERR_TIMEOUT = 8,     /* device-detected: a bounded pipeline wait gave up        */
-    LCQ_ERR_ARG = 9          /* any other invalid argument (e.g. latent_scale == 0)     */
+    LCQ_ERR_ARG = 9,         /* any other invalid argument (e.g. latent_scale == 0)     */
+    LCQ_ERR_LIMIT = 10       /* problem larger than the static scratch of a _noalloc call */
 } lcq_status;
 
 /* Operation selector for lcq_workspace_size(). */
@@ -164,6 +165,32 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
 lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
                              int d, const float *A, const float *b, uint16_t *Y,
                              void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * lcq_gemm_packed2b_noalloc - lcq_gemm_packed2b for callers that cannot
+ * allocate device memory. The paper has no counterpart: this entry point
+ * exists for callers that hand all device memory to their own fixed pool at
+ * start-up and must not allocate afterwards (for example a serving process
+ * with a hard memory budget), and for C callers with no device allocator.
+ *
+ * Same arguments and results as lcq_gemm_packed2b, without ws/ws_bytes: the
+ * scratch lives in one static device array of about 1 MiB that every GPU
+ * which loads the library holds until the process exits. The call itself
+ * allocates nothing (no cudaMalloc, cudaFree or allocating library routine).
+ *   - Limits: N <= 16 tokens and n <= 32768; larger problems return
+ *     LCQ_ERR_LIMIT before anything is enqueued.
+ *   - device_status: optional device int32 that receives the call's device
+ *     status word (LCQ_OK or a device-detected error); may be NULL.
+ *   - Every call shares the array and it keeps the last call's contents;
+ *     the call clears what must start at zero. Calls that can overlap on the
+ *     GPU (other streams, other host threads) race on the array.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make it before any
+ *     stream capture.
+ */
+lcq_status lcq_gemm_packed2b_noalloc(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
+                                     int d, const float *A, const float *b, uint16_t *Y,
+                                     int32_t *device_status, void *stream);
 
 /*
  * lcq_device_status - synchronise `stream`, then copy the workspace's device

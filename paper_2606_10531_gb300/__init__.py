@@ -17,14 +17,14 @@ LIB_PATH = os.path.join(PKG_DIR, "liblcq.so")
 LCQ_OK = 0
 STATUS_NAMES = {0: "LCQ_OK", 1: "LCQ_ERR_NULL", 2: "LCQ_ERR_SHAPE", 3: "LCQ_ERR_ALIGN", 4: "LCQ_ERR_UNSUPPORTED",
                 5: "LCQ_ERR_WORKSPACE", 6: "LCQ_ERR_CUDA", 7: "LCQ_ERR_SINGULAR", 8: "LCQ_ERR_TIMEOUT",
-                9: "LCQ_ERR_ARG"}
+                9: "LCQ_ERR_ARG", 10: "LCQ_ERR_LIMIT"}
 LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B = 1, 2, 3, 4
 LCQ_STE_IDENTITY, LCQ_STE_CLIPPED = 0, 1
 
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
-           "lcq_trace_read")
+           "lcq_trace_read", "lcq_gemm_packed2b_noalloc")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -53,6 +53,7 @@ _SIG = {
                                       _P, ctypes.c_size_t, _P]),
     "lcq_gemm_packed2b": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t,
                                          _P]),
+    "lcq_gemm_packed2b_noalloc": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
     "lcq_device_status": (ctypes.c_int, [_P, _P, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]),
     "lcq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "lcq_launch_count": (ctypes.c_uint64, []),
@@ -162,6 +163,15 @@ def lcq_gemm_packed2b(X, packed, n: int, d: int, A, b, Y, ws, stream=None):
     m = packed.shape[0]
     _check(lib().lcq_gemm_packed2b(_ptr(X), N, _ptr(packed), m, n, d, _ptr(A), _ptr(b), _ptr(Y), _ptr(ws),
                                    ws.numel(), _stream(stream)), "lcq_gemm_packed2b")
+
+
+def lcq_gemm_packed2b_noalloc(X, packed, n: int, d: int, A, b, Y, device_status=None, stream=None):
+    """Deployment product with the library's static scratch instead of a workspace (N <= 16, n <= 32768).
+    For callers that must not allocate device memory; overlapping calls race on the shared scratch."""
+    N = X.shape[0]
+    m = packed.shape[0]
+    _check(lib().lcq_gemm_packed2b_noalloc(_ptr(X), N, _ptr(packed), m, n, d, _ptr(A), _ptr(b), _ptr(Y),
+                                           _ptr(device_status), _stream(stream)), "lcq_gemm_packed2b_noalloc")
 
 
 def lcq_device_status(ws, clear: bool = False, stream=None) -> int:

@@ -148,6 +148,7 @@ const char *lcq_status_string(lcq_status s) {
         case LCQ_ERR_SINGULAR: return "A is singular";
         case LCQ_ERR_TIMEOUT: return "device pipeline wait timed out";
         case LCQ_ERR_ARG: return "invalid argument";
+        case LCQ_ERR_LIMIT: return "problem exceeds the static scratch of the allocation-free call";
         default: return "unknown status";
     }
 }
