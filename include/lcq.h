@@ -202,6 +202,9 @@ lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, 
 /* Static description of a status code; never NULL. */
 const char *lcq_status_string(lcq_status s);
 
+/* Text of the CUDA error behind the most recent LCQ_ERR_CUDA in this process ("no error" if none). */
+const char *lcq_last_cuda_error(void);
+
 /* Number of kernels this library has launched in the calling process. */
 uint64_t lcq_launch_count(void);
 
@@ -223,8 +226,8 @@ typedef enum lcq_kernel_kind {
     LCQ_K_GEMM_DX = 5,       /* tensor-core GEMM, dX = dY W_hat              */
     LCQ_K_GEMM_DW = 6,       /* tensor-core GEMM, dW_hat = dY^T X + dP/dA/db */
     LCQ_K_REDUCE = 7,        /* fixed-order dA/db reduction                  */
-    LCQ_K_GEMV_PREP = 8,     /* packed product: activation transform         */
-    LCQ_K_GEMV = 9,          /* packed product: main kernel                  */
+    LCQ_K_GEMV_PREP = 8,     /* reserved (the transform is timed inside GEMV) */
+    LCQ_K_GEMV = 9,          /* packed product: activation transform + main  */
     LCQ_K_NUM_KINDS = 10
 } lcq_kernel_kind;
 lcq_status lcq_trace_enable(int on);

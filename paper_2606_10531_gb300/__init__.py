@@ -24,7 +24,7 @@ LCQ_STE_IDENTITY, LCQ_STE_CLIPPED = 0, 1
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
-           "lcq_trace_read", "lcq_gemm_packed2b_noalloc")
+           "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -32,7 +32,13 @@ KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx
 class LCQError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
-        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)} ({_status_string(status)})")
+        detail = _status_string(status)
+        if status == 6:
+            try:
+                detail += ": " + lib().lcq_last_cuda_error().decode()
+            except Exception:  # noqa: BLE001 - only decorates the message
+                pass
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)} ({detail})")
 
 
 class lcq_opts(ctypes.Structure):
@@ -56,6 +62,7 @@ _SIG = {
     "lcq_gemm_packed2b_noalloc": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
     "lcq_device_status": (ctypes.c_int, [_P, _P, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]),
     "lcq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "lcq_last_cuda_error": (ctypes.c_char_p, []),
     "lcq_launch_count": (ctypes.c_uint64, []),
     "lcq_trace_enable": (ctypes.c_int, [ctypes.c_int]),
     "lcq_trace_read": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_double)]),

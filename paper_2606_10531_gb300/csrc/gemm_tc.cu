@@ -287,16 +287,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
 // ------------------------------------------------------------------ host side
 
 static PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    }
-    return fn;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
 }
 
 // rows x K operand stored K-major ([rows][ld]) or MN-major ([K][ld]); box rows_box x 64.
@@ -333,7 +324,7 @@ static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, cons
                               int trace_kind, cudaStream_t st) {
     auto k = gemm_kernel<EPI, D, A_MN, B_MN>;
     const int smem = static_cast<int>(sizeof(GemmSmem) + 1024);
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), smem);
     if (e != cudaSuccess) return e;
     trace_begin(trace_kind, st);
     k<<<grid, kGemmThreads, smem, st>>>(ma, mb, gp);

@@ -5,11 +5,20 @@
 //
 // so the integer codes themselves are the weight operand and A acts on the few activation rows.
 //
-// prep kernel  (one CTA per token): X' in bf16, written in the column order and scale the
-//              main kernel's register fragments expect, and the per-token constant corr[t].
-// main kernel  streams the codes once from HBM with 16-byte loads, turns each 32-bit word of 16
-//              codes into eight bf16x2 tensor-core fragments with one LOP3 each (no table, no
-//              shared memory) and accumulates with mma.sync m16n8k16 (rows of W x tokens).
+// prep kernel  (256 16-column blocks per CTA): X' in bf16, written in the column order and scale
+//              the main kernel's register fragments expect, and per-CTA partials of the per-token
+//              constant corr[t].
+// main kernel  streams the codes once from HBM, turns each 32-bit word of 16 codes into eight
+//              bf16x2 tensor-core fragments with one LOP3 each (no table) and accumulates with
+//              mma.sync m16n8k16 (16 rows of W x 8 tokens). The codes operand is converted in
+//              registers, so the bandwidth-bound stream never round-trips through a bf16 copy.
+//   tma variant (n % 64 == 0): persistent CTAs; one producer thread streams (rows x 512 columns)
+//              code tiles through an 8-stage shared-memory ring with 2-D TMA copies (128-byte
+//              swizzle, bank-conflict-free fragment reads); eight consumer warps each own a 64-column
+//              slice of every tile and reuse its activation fragments over all rows of the unit.
+//              Launched with programmatic dependent launch so the code stream starts while the
+//              prep kernel still runs; consumers wait for it (griddepcontrol.wait) before reading X'.
+//   generic variant: plain 16-byte loads (byte loads at a ragged row end), any n % 8 == 0.
 //
 // Code -> bf16 conversion: OR-ing a 2-bit field into the mantissa of bf16 128.0 (0x4300) gives
 // the exact value 128 + z * 4^p when the field sits at mantissa bit 2p (p = 0, 1, 2). Word w holds
@@ -22,12 +31,15 @@
 
 namespace lcq {
 
-constexpr int kGemvRowBlocks = 4;                 // 16-row MMA blocks per warp
-constexpr int kGemvRows = 16 * kGemvRowBlocks;    // rows of W per CTA
-constexpr int kGemvWarps = 8;                     // K is split over the CTA's warps
-constexpr int kSuper = 256;                       // columns per warp step (64 bytes per row)
+constexpr int kGemvRowBlocks = 4;                 // generic variant: 16-row MMA blocks per warp
+constexpr int kGemvRows = 16 * kGemvRowBlocks;    // generic variant: rows of W per CTA
+constexpr int kGemvWarps = 8;                     // generic variant: K is split over the CTA's warps
+constexpr int kSuper = 256;                       // generic variant: columns per warp step
+constexpr int kPadCols = 512;                     // X' rows are zero-padded to a multiple of this
+constexpr int kPrepCols = 4096;                   // columns per prep CTA (256 threads x 16)
 
-__host__ __device__ inline int64_t gemv_npad(int64_t n) { return (n + kSuper - 1) / kSuper * kSuper; }
+__host__ __device__ inline int64_t gemv_npad(int64_t n) { return (n + kPadCols - 1) / kPadCols * kPadCols; }
+__host__ __device__ inline int64_t gemv_nprep(int64_t n) { return (gemv_npad(n) + kPrepCols - 1) / kPrepCols; }
 
 // Field position (power-of-4 scale) of fragment register k.
 __device__ __forceinline__ int frag_shift(int k) { return (k % 3 == 2) ? 2 : ((k % 3 == 1) ? 1 : 0); }
@@ -35,8 +47,10 @@ __device__ __forceinline__ int frag_shift(int k) { return (k % 3 == 2) ? 2 : ((k
 template <int D>
 __global__ void __launch_bounds__(256)
 gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const float *__restrict__ A,
-                 const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ corr) {
+                 const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ corrpart) {
     __shared__ float red[2][8];
+    // let the dependent main kernel start streaming codes right away (it waits for our results itself)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t t = blockIdx.x;
     float Am[D * D], bv[D];
 #pragma unroll
@@ -46,7 +60,8 @@ gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const 
     const uint16_t *xrow = X + t * n;
     uint32_t *out = reinterpret_cast<uint32_t *>(Xp + t * npad);
     float S = 0.0f, r = 0.0f;
-    for (int64_t blk = threadIdx.x; blk < npad / 16; blk += blockDim.x) {
+    const int64_t blk = static_cast<int64_t>(blockIdx.y) * 256 + threadIdx.x;
+    if (blk < npad / 16) {
         float xp[16];
         const int64_t c0 = blk * 16;
         if (c0 + 16 <= n) {
@@ -110,9 +125,16 @@ gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const 
     __syncthreads();
     if (threadIdx.x == 0) {
         float s2 = 0.0f, r2 = 0.0f;
-        for (int w = 0; w < static_cast<int>(blockDim.x / 32); ++w) { s2 += red[0][w]; r2 += red[1][w]; }
-        corr[t] = r2 - 128.0f * s2;
+        for (int w = 0; w < 8; ++w) { s2 += red[0][w]; r2 += red[1][w]; }
+        corrpart[t * gridDim.y + blockIdx.y] = r2 - 128.0f * s2;
     }
+}
+
+// corr[t] = sum of the prep CTAs' partials, in a fixed order.
+__device__ __forceinline__ float token_corr(const float *corrpart, int64_t t, int64_t nprep) {
+    float s = 0.0f;
+    for (int64_t c = 0; c < nprep; ++c) s += corrpart[t * nprep + c];
+    return s;
 }
 
 __device__ __forceinline__ uint32_t lop_or_and(uint32_t a, uint32_t mask) {
@@ -136,8 +158,8 @@ __device__ __forceinline__ void codes_to_frags(uint32_t w, uint32_t (&f)[8]) {
 
 __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                                uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+    // not volatile: a pure function of its operands, so independent accumulator chains can be interleaved
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
         "{%0, %1, %2, %3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
@@ -155,8 +177,9 @@ __device__ __forceinline__ uint4 load_codes(const uint8_t *row_ptr, int64_t byte
 template <bool VEC>
 __global__ void __launch_bounds__(32 * kGemvWarps)
 packed_gemv_kernel(const uint8_t *__restrict__ packed, int64_t m, int64_t n, int64_t N, const uint16_t *__restrict__ Xp,
-                   int64_t npad, const float *__restrict__ corr, uint16_t *__restrict__ Y) {
+                   int64_t npad, const float *__restrict__ corrpart, int64_t nprep, uint16_t *__restrict__ Y) {
     __shared__ float red[kGemvWarps][kGemvRows][17];
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane >> 2, tid = lane & 3;
     const int64_t row0 = static_cast<int64_t>(blockIdx.x) * kGemvRows;
@@ -174,9 +197,9 @@ packed_gemv_kernel(const uint8_t *__restrict__ packed, int64_t m, int64_t n, int
 #pragma unroll
             for (int e = 0; e < 4; ++e) acc[i][nt][e] = 0.0f;
 
-    const uint32_t *xp0 = reinterpret_cast<const uint32_t *>(Xp + (tok0 + g) * npad);
-    const uint32_t *xp1 = reinterpret_cast<const uint32_t *>(Xp + (tok0 + g + 8) * npad);
     const bool has0 = g < ntok, has1 = g + 8 < ntok;
+    const uint32_t *xp0 = reinterpret_cast<const uint32_t *>(Xp + (tok0 + (has0 ? g : 0)) * npad);
+    const uint32_t *xp1 = reinterpret_cast<const uint32_t *>(Xp + (tok0 + (has1 ? g + 8 : 0)) * npad);
 
     for (int64_t sc = warp; sc < nsc; sc += kGemvWarps) {
         const int64_t byte0 = sc * 64 + 16 * tid;
@@ -233,35 +256,306 @@ packed_gemv_kernel(const uint8_t *__restrict__ packed, int64_t m, int64_t n, int
         float s = 0.0f;
 #pragma unroll
         for (int w = 0; w < kGemvWarps; ++w) s += red[w][rl][tl];
-        s += corr[tok0 + tl];
+        s += token_corr(corrpart, tok0 + tl, nprep);
         const __nv_bfloat16 h = __float2bfloat16_rn(s);
         Y[(tok0 + tl) * m + row] = *reinterpret_cast<const uint16_t *>(&h);
     }
 }
 
+// ------------------------------------------------------------------ TMA-streamed variant
+
+constexpr int kTmaStages = 8;
+constexpr int kTmaMaxRows = 128;      // rows of W per unit (multiple of 16)
+constexpr int kColGroups = 8;         // 64-column slices of a 512-column tile
+constexpr int kTileCols = 512;        // 128 bytes of codes per row per stage
+
+struct GemvSmem {
+    uint8_t ring[kTmaStages][kTmaMaxRows * 128];
+    float red[kColGroups][kTmaMaxRows][17];
+    uint64_t full[kTmaStages];
+    uint64_t empty[kTmaStages];
+    float corr[16];
+};
+
+struct GemvTmaParams {
+    int64_t m, N, npad, nprep;
+    int R, units, nkc;
+    const uint16_t *Xp;       // [N][npad] (token 0 of this launch)
+    const float *corrpart;    // [N][nprep]
+    uint16_t *Y;              // [N][m]
+    int32_t *status;
+};
+
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+// NT: 8-token MMA tiles (1: N <= 8, 2: N <= 16). CW: consumer warps; with 16 the two warps of a
+// 64-column slice split its rows, doubling the warps available to hide latency.
+template <int NT, int CW>
+__global__ void __launch_bounds__(32 * (CW + 1), 1)
+packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaParams p) {
+    constexpr int kRbPerWarp = (kTmaMaxRows / 16) / (CW / kColGroups);
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    GemvSmem &s = *reinterpret_cast<GemvSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        prefetch_tensormap(&tmC);
+        for (int i = 0; i < kTmaStages; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], CW);
+        }
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- producer: code tiles -> ring
+        if (lane == 0) {
+            const uint32_t bytes = static_cast<uint32_t>(p.R) * 128u;
+            int it = 0;
+            for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
+                for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+                    const int st = it % kTmaStages;
+                    if (!mbar_wait(&s.empty[st], ((it / kTmaStages) & 1) ^ 1, p.status)) return;
+                    mbar_arrive_expect_tx(&s.full[st], bytes);
+                    tma_load_2d(s.ring[st], &tmC, kc * 128, u * p.R, &s.full[st]);
+                }
+            }
+        }
+        return;
+    }
+
+    // -------------------------------------------------------------------- consumers
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // X' and corr partials of the prep kernel
+    const int cw = (warp - 1) % kColGroups;              // 64-column slice
+    const int rb0 = ((warp - 1) / kColGroups) * kRbPerWarp;
+    const int g = lane >> 2, tid = lane & 3;
+    const int ct = threadIdx.x - 32;
+    if (ct < p.N) s.corr[ct] = token_corr(p.corrpart, ct, p.nprep);
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+    const bool has0 = g < p.N, has1 = (g + 8) < p.N;
+    const uint32_t *xp0 = reinterpret_cast<const uint32_t *>(p.Xp + (has0 ? g : 0) * p.npad);
+    const uint32_t *xp1 = reinterpret_cast<const uint32_t *>(p.Xp + (has1 ? g + 8 : 0) * p.npad);
+    const int nrb = p.R / 16;
+    const uint32_t swz = static_cast<uint32_t>((cw ^ g) << 4) + 4u * tid;   // this lane's word in a swizzled row
+
+    // activation fragments of this warp's 64 columns of tile kc (16-column block of this lane's word);
+    // the next tile's fragments are fetched while the current tile is multiplied.
+    auto load_frags = [&](int kc, uint2 (&bq)[4][NT]) {
+        const int64_t blk = static_cast<int64_t>(kc) * (kTileCols / 16) + cw * 4 + tid;
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            bq[h][0] = has0 ? __ldg(reinterpret_cast<const uint2 *>(xp0 + blk * 8 + 2 * h)) : make_uint2(0, 0);
+            if (NT == 2)
+                bq[h][NT - 1] = has1 ? __ldg(reinterpret_cast<const uint2 *>(xp1 + blk * 8 + 2 * h)) : make_uint2(0, 0);
+        }
+    };
+    uint2 bcur[4][NT], bnext[4][NT];
+    load_frags(0, bcur);
+
+    int it = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
+        float acc[kRbPerWarp][NT][4];
+#pragma unroll
+        for (int i = 0; i < kRbPerWarp; ++i)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[i][nt][e] = 0.0f;
+
+        for (int kc = 0; kc < p.nkc; ++kc, ++it) {
+            const int st = it % kTmaStages;
+            load_frags(kc + 1 < p.nkc ? kc + 1 : 0, bnext);
+            if (!mbar_wait(&s.full[st], (it / kTmaStages) & 1, p.status)) { ok = false; break; }
+            const uint32_t base = smem_u32(s.ring[st]) + swz;
+            // row blocks in pairs: two blocks' fragments converted, then their MMAs interleaved (h outer)
+#pragma unroll
+            for (int rp = 0; rp < kRbPerWarp / 2; ++rp) {
+                const int rb = rb0 + 2 * rp;
+                if (rb < nrb) {
+                    const bool second = rb + 1 < nrb;
+                    uint32_t w[2][2];
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        const uint32_t rbase = static_cast<uint32_t>((rb + j) * 16 + g) * 128u;
+                        w[j][0] = (j == 0 || second) ? lds32(base + rbase) : 0u;
+                        w[j][1] = (j == 0 || second) ? lds32(base + rbase + 8u * 128u) : 0u;
+                    }
+                    uint32_t f[2][2][8];
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        codes_to_frags(w[j][0], f[j][0]);
+                        codes_to_frags(w[j][1], f[j][1]);
+                    }
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) {
+                            if (j == 0 || second) {
+#pragma unroll
+                                for (int nt = 0; nt < NT; ++nt)
+                                    mma_bf16_16816(acc[2 * rp + j][nt], f[j][0][2 * h], f[j][1][2 * h],
+                                                   f[j][0][2 * h + 1], f[j][1][2 * h + 1], bcur[h][nt].x,
+                                                   bcur[h][nt].y);
+                            }
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.empty[st]);
+#pragma unroll
+            for (int h = 0; h < 4; ++h)
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) bcur[h][nt] = bnext[h][nt];
+        }
+        if (!ok) break;
+        // cross-slice reduction (fixed order), + corr, bf16 store
+#pragma unroll
+        for (int i = 0; i < kRbPerWarp; ++i) {
+            const int rb = rb0 + i;
+            if (rb < nrb) {
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    s.red[cw][16 * rb + g][nt * 8 + 2 * tid] = acc[i][nt][0];
+                    s.red[cw][16 * rb + g][nt * 8 + 2 * tid + 1] = acc[i][nt][1];
+                    s.red[cw][16 * rb + g + 8][nt * 8 + 2 * tid] = acc[i][nt][2];
+                    s.red[cw][16 * rb + g + 8][nt * 8 + 2 * tid + 1] = acc[i][nt][3];
+                }
+            }
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+        const int64_t row0 = static_cast<int64_t>(u) * p.R;
+        for (int o = ct; o < p.R * p.N; o += 32 * CW) {
+            const int rl = o % p.R, tl = o / p.R;
+            const int64_t row = row0 + rl;
+            if (row >= p.m) continue;
+            float v = 0.0f;
+#pragma unroll
+            for (int w = 0; w < kColGroups; ++w) v += s.red[w][rl][tl];
+            v += s.corr[tl];
+            const __nv_bfloat16 h = __float2bfloat16_rn(v);
+            p.Y[static_cast<int64_t>(tl) * p.m + row] = *reinterpret_cast<const uint16_t *>(&h);
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ host side
+
 size_t packed_gemv_workspace(int64_t N, int64_t n) {
     const size_t xp = static_cast<size_t>(N) * static_cast<size_t>(gemv_npad(n)) * 2;
-    const size_t cr = static_cast<size_t>(N) * 4;
+    const size_t cr = static_cast<size_t>(N) * static_cast<size_t>(gemv_nprep(n)) * 4;
     return ((xp + 255) / 256) * 256 + ((cr + 255) / 256) * 256;
 }
 
+size_t packed_gemv_corr_offset(int64_t N, int64_t n) {
+    const size_t xp = static_cast<size_t>(N) * static_cast<size_t>(gemv_npad(n)) * 2;
+    return ((xp + 255) / 256) * 256;
+}
+
+// Rows per unit for the TMA variant: balance the units over the persistent CTAs.
+static int choose_rows(int64_t m, int ctas) {
+    int best = 64;
+    double best_eff = -1.0;
+    for (int R = kTmaMaxRows; R >= 64; R -= 16) {
+        const int64_t units = (m + R - 1) / R;
+        const int64_t rounds = (units + ctas - 1) / ctas;
+        const double eff = static_cast<double>(units) / static_cast<double>(rounds * (units < ctas ? units : ctas));
+        const double rows_eff = static_cast<double>(m) / static_cast<double>(units * R);
+        const double e = eff * rows_eff;
+        if (e > best_eff + 1e-9) { best_eff = e; best = R; }
+    }
+    return best;
+}
+
+static bool make_codes_map(CUtensorMap *map, const uint8_t *packed, int64_t m, int64_t n, int R) {
+    void *fnp = tensor_map_encoder();
+    if (!fnp) return false;
+    auto enc = reinterpret_cast<CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                             const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                             CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                             CUtensorMapFloatOOBfill)>(fnp);
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(n / 4), static_cast<cuuint64_t>(m)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(n / 4)};
+    cuuint32_t box[2] = {128, static_cast<cuuint32_t>(R)};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(packed), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k, std::forward<Args>(args)...);
+}
+
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st) {
-    (void)num_sms;
-    const int64_t npad = gemv_npad(a.n);
-    trace_begin(LCQ_K_GEMV_PREP, st);
-    if (d == 4) gemv_prep_kernel<4><<<static_cast<unsigned>(a.N), 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
-    else gemv_prep_kernel<8><<<static_cast<unsigned>(a.N), 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
-    trace_end(LCQ_K_GEMV_PREP, st);
+    const int64_t npad = gemv_npad(a.n), nprep = gemv_nprep(a.n);
+    trace_begin(LCQ_K_GEMV, st);
+    dim3 pgrid(static_cast<unsigned>(a.N), static_cast<unsigned>(nprep));
+    if (d == 4) gemv_prep_kernel<4><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
+    else gemv_prep_kernel<8><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
     count_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dim3 grid(static_cast<unsigned>((a.m + kGemvRows - 1) / kGemvRows), static_cast<unsigned>((a.N + 15) / 16));
-    const bool vec = (a.n % 64) == 0;
-    trace_begin(LCQ_K_GEMV, st);
-    if (vec) packed_gemv_kernel<true><<<grid, 32 * kGemvWarps, 0, st>>>(a.packed, a.m, a.n, a.N, a.Xp, npad, a.corr, a.Y);
-    else packed_gemv_kernel<false><<<grid, 32 * kGemvWarps, 0, st>>>(a.packed, a.m, a.n, a.N, a.Xp, npad, a.corr, a.Y);
+    if (a.n % 64 == 0 && a.m >= 16) {
+        const int R = choose_rows(a.m, num_sms);
+        CUtensorMap map;
+        if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
+        const int units = static_cast<int>((a.m + R - 1) / R);
+        const int grid = units < num_sms ? units : num_sms;
+        const size_t smem = sizeof(GemvSmem) + 1024;
+        for (int64_t t0 = 0; t0 < a.N; t0 += 16) {
+            GemvTmaParams p;
+            p.m = a.m;
+            p.N = (a.N - t0) < 16 ? (a.N - t0) : 16;
+            p.npad = npad;
+            p.nprep = nprep;
+            p.R = R;
+            p.units = units;
+            p.nkc = static_cast<int>(npad / kTileCols);
+            p.Xp = a.Xp + t0 * npad;
+            p.corrpart = a.corr + t0 * nprep;
+            p.Y = a.Y + t0 * a.m;
+            p.status = a.status;
+            const bool two = p.N > 8;
+            auto k = two ? packed_gemv_tma_kernel<2, 8> : packed_gemv_tma_kernel<1, 16>;
+            const int threads = two ? 32 * 9 : 32 * 17;
+            e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            e = launch_pdl(k, dim3(grid), dim3(threads), smem, st, map, p);
+            count_launch();
+            if (e != cudaSuccess) return e;
+        }
+    } else {
+        dim3 grid(static_cast<unsigned>((a.m + kGemvRows - 1) / kGemvRows), static_cast<unsigned>((a.N + 15) / 16));
+        const bool vec = (a.n % 64) == 0;
+        if (vec)
+            e = launch_pdl(packed_gemv_kernel<true>, grid, dim3(32 * kGemvWarps), 0, st, a.packed, a.m, a.n, a.N,
+                           static_cast<const uint16_t *>(a.Xp), npad, static_cast<const float *>(a.corr), nprep, a.Y);
+        else
+            e = launch_pdl(packed_gemv_kernel<false>, grid, dim3(32 * kGemvWarps), 0, st, a.packed, a.m, a.n, a.N,
+                           static_cast<const uint16_t *>(a.Xp), npad, static_cast<const float *>(a.corr), nprep, a.Y);
+        count_launch();
+        if (e != cudaSuccess) return e;
+    }
     trace_end(LCQ_K_GEMV, st);
-    count_launch();
     return cudaGetLastError();
 }
 

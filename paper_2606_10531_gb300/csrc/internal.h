@@ -8,6 +8,10 @@
 namespace lcq {
 
 void count_launch();
+// cuTensorMapEncodeTiled from the driver (looked up once); nullptr if unavailable.
+void *tensor_map_encoder();
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per kernel and device.
+cudaError_t ensure_dynamic_smem(const void *fn, int bytes);
 // Record the start / end event of a kernel of the given lcq_kernel_kind on `st` (no-op unless tracing).
 void trace_begin(int kind, cudaStream_t st);
 void trace_end(int kind, cudaStream_t st);
@@ -93,11 +97,12 @@ struct PackedGemvArgs {
     const uint8_t *packed;   // [m][n/4]
     const float *A, *b;
     uint16_t *Y;             // [N][m] bf16
-    uint16_t *Xp;            // workspace: transformed activations
-    float *corr;             // workspace: per-token constant
+    uint16_t *Xp;            // workspace: transformed activations [N][npad]
+    float *corr;             // workspace: per-token constant, partial sums [N][nprep]
     int32_t *status;
 };
 size_t packed_gemv_workspace(int64_t N, int64_t n);
+size_t packed_gemv_corr_offset(int64_t N, int64_t n);
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);
 
 }  // namespace lcq

@@ -14,12 +14,12 @@
 
 namespace lcq {
 
-constexpr int kChunk = 4096;                 // fp32 weights per stage (16 KB)
-constexpr int kStages = 4;
-constexpr int kComputeWarps = 8;
+constexpr int kComputeWarps = 11;                                // + 1 producer = 12 warps, 3 per SM sub-partition
+constexpr int kPerThread = 16;                                   // weights per compute thread per stage
+constexpr int kChunk = 32 * kComputeWarps * kPerThread;          // fp32 weights per stage (22 KB)
+constexpr int kStages = 6;                                       // 132 KB ring
 constexpr int kStreamThreads = 32 * (1 + kComputeWarps);
-constexpr int kPerThread = kChunk / (32 * kComputeWarps);   // 16
-static_assert(kPerThread == 16, "each compute thread owns 16 weights");
+constexpr float kRoundMagic = 12582912.0f;                       // 1.5 * 2^23
 
 struct StreamSmem {
     float buf[kStages][kChunk];
@@ -27,9 +27,9 @@ struct StreamSmem {
     uint64_t empty[kStages];
     float Ainv[64];
     float A[64];
+    float M[64];        // A^T A (encode MSE)
     float b[8];
     double gj[8][16];
-    float red[kComputeWarps];
     double dred[kComputeWarps];
     int singular;
 };
@@ -54,8 +54,8 @@ __device__ void stream_producer(StreamSmem &s, const float *src, int64_t total, 
     }
 }
 
-// One warp: A^{-1} by Gauss-Jordan elimination with partial pivoting in fp64,
-// rounded to fp32. Sets s.singular if a pivot is (relatively) zero.
+// One warp: A^{-1} by Gauss-Jordan elimination with partial pivoting in fp64, rounded to fp32,
+// and M = A^T A. Sets s.singular if a pivot is (relatively) zero.
 template <int D>
 __device__ void invert_warp(StreamSmem &s) {
     const int lane = threadIdx.x & 31;
@@ -66,11 +66,16 @@ __device__ void invert_warp(StreamSmem &s) {
         s.gj[r][c] = v;
         if (c < D) amax = fmax(amax, fabs(v));
     }
+    for (int e = lane; e < D * D; e += 32) {
+        const int i = e / D, j = e % D;
+        double acc = 0.0;
+        for (int r = 0; r < D; ++r) acc += static_cast<double>(s.A[r * D + i]) * static_cast<double>(s.A[r * D + j]);
+        s.M[e] = static_cast<float>(acc);
+    }
     for (int o = 16; o; o >>= 1) amax = fmax(amax, __shfl_xor_sync(0xffffffffu, amax, o));
     __syncwarp();
     int singular = !(amax > 0.0) || !isfinite(amax);
     for (int c = 0; c < D && !singular; ++c) {
-        // pivot search over rows c..D-1
         double best = -1.0;
         int prow = c;
         for (int r = c; r < D; ++r) {
@@ -90,10 +95,7 @@ __device__ void invert_warp(StreamSmem &s) {
         __syncwarp();
         double f[4];
         int cnt = 0;
-        for (int e = lane; e < D * 2 * D; e += 32, ++cnt) {
-            const int r = e / (2 * D);
-            f[cnt] = s.gj[r][c];
-        }
+        for (int e = lane; e < D * 2 * D; e += 32, ++cnt) f[cnt] = s.gj[e / (2 * D)][c];
         __syncwarp();
         cnt = 0;
         for (int e = lane; e < D * 2 * D; e += 32, ++cnt) {
@@ -110,33 +112,70 @@ __device__ void invert_warp(StreamSmem &s) {
 }
 
 // ------------------------------------------------------------------ encode
+//
+// Per group (d weights): v = w - b; u = A^{-1} v (packed fp32x2 FMAs over pairs of rows of A^{-1});
+// z = clip(round_half_even(u), 0, 3) taken on the fp32 pipe: t = u + 1.5*2^23 rounds u to an
+// integer (round to nearest even), clamping t to [1.5*2^23, 1.5*2^23 + 3] clamps the integer,
+// whose value is then the low two bits of t (NaN -> 0: fmaxf drops the NaN).
+// Squared residual ||w - (A z + b)||^2 = ||A (u - z)||^2 = e^T (A^T A) e with e = u - z.
+
+// Packing without extracting the codes: bits(tc) = kMagicBits + z, so summing bits(tc_k) * 4^k over the
+// 16 codes of a thread (mod 2^32) gives the packed word plus kMagicBits * (4^0 + ... + 4^15), removed once.
+constexpr uint32_t kMagicBits = 0x4B400000u;                       // bits of 1.5 * 2^23
+constexpr uint32_t kPackBias = kMagicBits * 0x55555555u;           // kMagicBits * sum_{k<16} 4^k (mod 2^32)
 
 template <int D, bool kMse>
-__device__ __forceinline__ void encode_group(const float *w, const float (&Ai)[D * D], const float (&Am)[D * D],
-                                             const float (&bv)[D], uint32_t (&z)[D], float (&u)[D], float &sq) {
+__device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)[D / 2][D], const float (&Mu)[D * (D + 1) / 2],
+                                             const float2 (&bv2)[D / 2], uint32_t &zacc, int zshift, float (&u)[D],
+                                             float &sq) {
     float v[D];
 #pragma unroll
-    for (int j = 0; j < D; ++j) v[j] = w[j] - bv[j];
+    for (int j = 0; j < D / 2; ++j) {
+        const float2 r = __fadd2_rn(make_float2(w[2 * j], w[2 * j + 1]), bv2[j]);   // w - b (bv2 holds -b)
+        v[2 * j] = r.x;
+        v[2 * j + 1] = r.y;
+    }
+    float2 u2[D / 2];
 #pragma unroll
-    for (int k = 0; k < D; ++k) {
-        float acc = 0.0f;
+    for (int kp = 0; kp < D / 2; ++kp) {
+        float2 acc = make_float2(0.0f, 0.0f);
 #pragma unroll
-        for (int j = 0; j < D; ++j) acc = fmaf(Ai[k * D + j], v[j], acc);
-        u[k] = acc;
-        z[k] = round_clamp3(acc);
+        for (int j = 0; j < D; ++j) acc = __ffma2_rn(Ai2[kp][j], make_float2(v[j], v[j]), acc);
+        u2[kp] = acc;
+        u[2 * kp] = acc.x;
+        u[2 * kp + 1] = acc.y;
+    }
+    float e[D];
+#pragma unroll
+    for (int kp = 0; kp < D / 2; ++kp) {
+        const float2 t = __fadd2_rn(u2[kp], make_float2(kRoundMagic, kRoundMagic));
+        const float tc0 = fminf(fmaxf(t.x, kRoundMagic), kRoundMagic + 3.0f);
+        const float tc1 = fminf(fmaxf(t.y, kRoundMagic), kRoundMagic + 3.0f);
+        zacc += __float_as_uint(tc0) << (zshift + 4 * kp);
+        zacc += __float_as_uint(tc1) << (zshift + 4 * kp + 2);
+        if (kMse) {
+            const float2 zf = __fadd2_rn(make_float2(tc0, tc1), make_float2(-kRoundMagic, -kRoundMagic));
+            const float2 ee = __ffma2_rn(zf, make_float2(-1.0f, -1.0f), u2[kp]);
+            e[2 * kp] = ee.x;
+            e[2 * kp + 1] = ee.y;
+        }
     }
     if (kMse) {
+        // e^T M e with the upper triangle of M (off-diagonal terms pre-doubled)
+        float q = 0.0f;
+        int idx = 0;
 #pragma unroll
-        for (int j = 0; j < D; ++j) {
-            float r = v[j];
+        for (int i = 0; i < D; ++i) {
+            float si = 0.0f;
 #pragma unroll
-            for (int k = 0; k < D; ++k) r = fmaf(-Am[j * D + k], static_cast<float>(z[k]), r);
-            sq = fmaf(r, r, sq);
+            for (int j = i; j < D; ++j) si = fmaf(Mu[idx++], e[j], si);
+            q = fmaf(e[i], si, q);
         }
+        sq += q;
     }
 }
 
-template <int D, bool kMse>
+template <int D, bool kMse, bool kLatent>
 __global__ void __launch_bounds__(kStreamThreads, 1)
 encode_kernel(EncodeArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -164,11 +203,21 @@ encode_kernel(EncodeArgs a) {
     compute_bar();
     if (s.singular && blockIdx.x == 0 && threadIdx.x == 32) set_status(a.status, LCQ_ERR_SINGULAR);
 
-    float Ai[D * D], Am[D * D], bv[D];
+    float2 Ai2[D / 2][D], bv2[D / 2];
+    float Mu[D * (D + 1) / 2];
 #pragma unroll
-    for (int i = 0; i < D * D; ++i) { Ai[i] = s.Ainv[i]; Am[i] = s.A[i]; }
+    for (int kp = 0; kp < D / 2; ++kp)
 #pragma unroll
-    for (int i = 0; i < D; ++i) bv[i] = s.b[i];
+        for (int j = 0; j < D; ++j) Ai2[kp][j] = make_float2(s.Ainv[(2 * kp) * D + j], s.Ainv[(2 * kp + 1) * D + j]);
+    {
+        int idx = 0;
+#pragma unroll
+        for (int i = 0; i < D; ++i)
+#pragma unroll
+            for (int j = i; j < D; ++j) Mu[idx++] = (i == j ? 1.0f : 2.0f) * s.M[i * D + j];
+    }
+#pragma unroll
+    for (int i = 0; i < D / 2; ++i) bv2[i] = make_float2(-s.b[2 * i], -s.b[2 * i + 1]);
 
     const int t = threadIdx.x - 32;
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
@@ -183,57 +232,51 @@ encode_kernel(EncodeArgs a) {
         if (off < cnt) {
             const int valid = static_cast<int>((cnt - off) < kPerThread ? (cnt - off) : kPerThread);
             const float *src = s.buf[st] + off;
-            float w[kPerThread];
-#pragma unroll
-            for (int q = 0; q < kPerThread / 4; ++q) {
-                const float4 f = (q * 4 < valid) ? reinterpret_cast<const float4 *>(src)[q] : make_float4(0, 0, 0, 0);
-                w[4 * q] = f.x; w[4 * q + 1] = f.y; w[4 * q + 2] = f.z; w[4 * q + 3] = f.w;
-            }
-            uint32_t zz[kPerThread];
-            float uu[kPerThread];
+            const int64_t gidx = base + off;   // flat weight index, multiple of 16
+            uint32_t p = 0;
+            // every group of the slice is computed (a ragged tail reads stale shared memory that is
+            // neither stored nor summed): valid is a multiple of d
 #pragma unroll
             for (int g = 0; g < kPerThread / D; ++g) {
-                uint32_t z[D];
+                float w[D];
+#pragma unroll
+                for (int q = 0; q < D / 4; ++q) {
+                    const float4 f = reinterpret_cast<const float4 *>(src + g * D)[q];
+                    w[4 * q] = f.x; w[4 * q + 1] = f.y; w[4 * q + 2] = f.z; w[4 * q + 3] = f.w;
+                }
                 float u[D];
                 float gsq = 0.0f;
-                encode_group<D, kMse>(w + g * D, Ai, Am, bv, z, u, gsq);
-                if (g * D < valid) sq += gsq;
+                encode_group<D, kMse>(w, Ai2, Mu, bv2, p, 2 * g * D, u, gsq);
+                if (g * D < valid) {
+                    sq += gsq;
+                    if (kLatent) {
+                        float4 *dst = reinterpret_cast<float4 *>(a.latent + gidx + g * D);
 #pragma unroll
-                for (int k = 0; k < D; ++k) { zz[g * D + k] = z[k]; uu[g * D + k] = u[k]; }
+                        for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+                    }
+                }
             }
-            const int64_t gidx = base + off;   // flat weight index, multiple of 16
+            p -= kPackBias;
             if (valid == kPerThread) {
-                if (a.packed) {
-                    uint32_t p = 0;
-#pragma unroll
-                    for (int k = 0; k < kPerThread; ++k) p |= zz[k] << (2 * k);
-                    *reinterpret_cast<uint32_t *>(a.packed + gidx / 4) = p;
-                }
+                if (a.packed) *reinterpret_cast<uint32_t *>(a.packed + gidx / 4) = p;
                 if (a.codes) {
-                    uint4 q;
-                    q.x = zz[0] | (zz[1] << 8) | (zz[2] << 16) | (zz[3] << 24);
-                    q.y = zz[4] | (zz[5] << 8) | (zz[6] << 16) | (zz[7] << 24);
-                    q.z = zz[8] | (zz[9] << 8) | (zz[10] << 16) | (zz[11] << 24);
-                    q.w = zz[12] | (zz[13] << 8) | (zz[14] << 16) | (zz[15] << 24);
-                    *reinterpret_cast<uint4 *>(a.codes + gidx) = q;
-                }
-                if (a.latent) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.latent + gidx);
+                    // spread 2-bit fields to bytes: byte k of word q = code 4q + k
+                    uint32_t ww[4];
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) dst[q] = make_float4(uu[4 * q], uu[4 * q + 1], uu[4 * q + 2], uu[4 * q + 3]);
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t f = (p >> (8 * q)) & 0xFFu;
+                        ww[q] = (f & 3u) | (((f >> 2) & 3u) << 8) | (((f >> 4) & 3u) << 16) | (((f >> 6) & 3u) << 24);
+                    }
+                    *reinterpret_cast<uint4 *>(a.codes + gidx) = make_uint4(ww[0], ww[1], ww[2], ww[3]);
                 }
             } else {
 #pragma unroll
                 for (int k = 0; k < kPerThread; k += 4) {
                     if (k < valid) {
-                        if (a.packed)
-                            a.packed[(gidx + k) / 4] =
-                                static_cast<uint8_t>(zz[k] | (zz[k + 1] << 2) | (zz[k + 2] << 4) | (zz[k + 3] << 6));
+                        if (a.packed) a.packed[(gidx + k) / 4] = static_cast<uint8_t>((p >> (2 * k)) & 0xFFu);
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            if (a.codes) a.codes[gidx + k + e] = static_cast<uint8_t>(zz[k + e]);
-                            if (a.latent) a.latent[gidx + k + e] = uu[k + e];
-                        }
+                        for (int e = 0; e < 4; ++e)
+                            if (a.codes) a.codes[gidx + k + e] = static_cast<uint8_t>((p >> (2 * (k + e))) & 3u);
                     }
                 }
             }
@@ -462,24 +505,28 @@ __global__ void reduce_partials_kernel(const float *__restrict__ partials, int n
 
 static int stream_grid(int64_t total, int num_sms) {
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
-    int64_t g = 2LL * num_sms;
+    int64_t g = num_sms;   // persistent: one CTA (a 144 KB ring) per SM
     if (nchunks < g) g = nchunks;
     return static_cast<int>(g < 1 ? 1 : g);
 }
 
-size_t encode_partials_offset() { return 256; }
-
-int encode_max_blocks(int num_sms) { return 2 * num_sms; }
+int encode_max_blocks(int num_sms) { return num_sms; }
 
 cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t st) {
     const int64_t total = a.m * a.n;
     const int grid = stream_grid(total, num_sms);
     const size_t smem = sizeof(StreamSmem);
     const bool mse = a.mse != nullptr;
+    const bool lat = a.latent != nullptr;
     void (*k)(EncodeArgs) = nullptr;
-    if (d == 4) k = mse ? encode_kernel<4, true> : encode_kernel<4, false>;
-    else k = mse ? encode_kernel<8, true> : encode_kernel<8, false>;
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (d == 4) {
+        k = mse ? (lat ? encode_kernel<4, true, true> : encode_kernel<4, true, false>)
+                : (lat ? encode_kernel<4, false, true> : encode_kernel<4, false, false>);
+    } else {
+        k = mse ? (lat ? encode_kernel<8, true, true> : encode_kernel<8, true, false>)
+                : (lat ? encode_kernel<8, false, true> : encode_kernel<8, false, false>);
+    }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     trace_begin(LCQ_K_ENCODE, st);
     k<<<grid, kStreamThreads, smem, st>>>(a);
@@ -493,7 +540,7 @@ cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cu
     const int grid = stream_grid(total, num_sms);
     const size_t smem = sizeof(StreamSmem);
     void (*k)(QuantDecodeArgs) = d == 4 ? quant_decode_kernel<4> : quant_decode_kernel<8>;
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     trace_begin(LCQ_K_QUANT_DECODE, st);
     k<<<grid, kStreamThreads, smem, st>>>(a);

@@ -2,6 +2,7 @@
 // See include/lcq.h for the contract of every entry point.
 #include <atomic>
 #include <cstring>
+#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
@@ -41,6 +42,39 @@ void trace_end(int kind, cudaStream_t st) {
     if (!g_trace_on || g_trace_n >= LCQ_TRACE_CAPACITY || g_trace[g_trace_n].kind != kind) return;
     cudaEventRecord(g_trace[g_trace_n].stop, st);
     ++g_trace_n;
+}
+
+void *tensor_map_encoder() {
+    static std::once_flag once;
+    static void *fn = nullptr;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = p;
+    });
+    return fn;
+}
+
+cudaError_t ensure_dynamic_smem(const void *fn, int bytes) {
+    struct Entry {
+        const void *fn;
+        int dev, bytes;
+    };
+    static std::mutex mu;
+    static Entry done[256];
+    static int ndone = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < ndone; ++i)
+        if (done[i].fn == fn && done[i].dev == dev && done[i].bytes >= bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && ndone < 256) done[ndone++] = {fn, dev, bytes};
+    return e;
 }
 
 static int num_sms_current() {
@@ -89,7 +123,13 @@ static lcq_status check_ws(void *ws, size_t ws_bytes, size_t need) {
     return LCQ_OK;
 }
 
-static lcq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LCQ_OK : LCQ_ERR_CUDA; }
+static std::atomic<int> g_last_cuda_error{0};
+
+static lcq_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return LCQ_OK;
+    g_last_cuda_error.store(static_cast<int>(e), std::memory_order_relaxed);
+    return LCQ_ERR_CUDA;
+}
 
 static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste) {
     float s = 1.0f;
@@ -154,6 +194,11 @@ const char *lcq_status_string(lcq_status s) {
 }
 
 uint64_t lcq_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char *lcq_last_cuda_error(void) {
+    const int e = g_last_cuda_error.load(std::memory_order_relaxed);
+    return e == 0 ? "no error" : cudaGetErrorString(static_cast<cudaError_t>(e));
+}
 
 lcq_status lcq_trace_enable(int on) {
     if (on) {
@@ -372,7 +417,7 @@ lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed
     PackedGemvArgs a;
     a.X = X; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
     a.Xp = reinterpret_cast<uint16_t *>(base);
-    a.corr = reinterpret_cast<float *>(base + align256(static_cast<size_t>(N) * ((n + 255) / 256 * 256) * 2));
+    a.corr = reinterpret_cast<float *>(base + packed_gemv_corr_offset(N, n));
     a.status = &h->status;
     return cuda_status(launch_packed_gemv(a, d, num_sms_current(), st));
 }
