@@ -243,7 +243,8 @@ def test_linear_empty_tokens_gives_zero_gradients():
 # ----------------------------------------------------------------------------- deployment product
 
 @pytest.mark.parametrize("N", [1, 4, 16, 17, 40])
-@pytest.mark.parametrize("m,n,d", [(200, 512, 8), (64, 1024, 4), (70, 200, 4), (8, 8, 8)])
+@pytest.mark.parametrize("m,n,d", [(200, 512, 8), (64, 1024, 4), (70, 200, 4), (8, 8, 8), (1000, 4096, 8),
+                                   (300, 8192, 4)])
 def test_gemm_packed2b_matches_oracle(N, m, n, d):
     torch = T()
     rng = np.random.default_rng(N * 1000 + m + n + d)
