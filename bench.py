@@ -318,9 +318,8 @@ def cpu_cores():
 
 def main():
     args = parse()
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2606_10531_gb300 import dist as lcq_dist
+    rank, local, world = lcq_dist.rank_world()
 
     if args.impl == "reference":
         return reference_arm(args, world, rank)
@@ -336,9 +335,7 @@ def main():
         raise SystemExit("bench.py needs a CUDA GPU")
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=device)
+    lcq_dist.init("nccl", device)
     lcq_build.build()
     lcq.lib()
     pk = peaks()
@@ -352,8 +349,7 @@ def main():
 
     def barrier():
         torch.cuda.synchronize()
-        if world > 1:
-            torch.distributed.barrier()
+        lcq_dist.barrier()
         torch.cuda.synchronize()
 
     for _ in range(max(args.warmup, 3)):
@@ -376,11 +372,7 @@ def main():
     launches = lcq.lcq_launch_count() - launches0
     lcq.lcq_trace_enable(False)
     clk = clocks.stop()
-    elapsed = e0.elapsed_time(e1) / 1e3
-    if world > 1:
-        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = lcq_dist.max_over_ranks(e0.elapsed_time(e1) / 1e3, device)
     trace = lcq.lcq_trace_read()
     for L in layer:
         assert L.statuses(lcq) == [0, 0, 0, 0]
@@ -433,12 +425,10 @@ def main():
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                                 "sample": f"oracle step (encode, fwd, bwd, packed product) on linears {used} with "
                                           f"64 of 16384 tokens; {spent:.1f} s of CPU work"}
-    if world > 1:
-        torch.distributed.barrier()
+    lcq_dist.barrier()
     if rank == 0:
         print(json.dumps(line), flush=True)
-    if world > 1:
-        torch.distributed.destroy_process_group()
+    lcq_dist.finalize()
 
 
 def e2e_arm(torch, lcq, wl, args, device, world, rank):
@@ -470,20 +460,16 @@ def e2e_arm(torch, lcq, wl, args, device, world, rank):
             h["Yg"].copy_(L.Yg, non_blocking=True)
         torch.cuda.current_stream().synchronize()
 
+    from paper_2606_10531_gb300 import dist as lcq_dist
     for _ in range(max(args.warmup, 3)):
         step()
     torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
+    lcq_dist.barrier()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         step()
     torch.cuda.synchronize()
-    el = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([el], device=device, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        el = float(t.item())
+    el = lcq_dist.max_over_ranks(time.perf_counter() - t0, device)
     flops = sum(L.flops() for L in layer) * args.steps * world
     del layer, host
     torch.cuda.empty_cache()

@@ -199,6 +199,16 @@ lcq_status lcq_gemm_packed2b_noalloc(const uint16_t *X, int64_t N, const uint8_t
  */
 lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, int clear);
 
+/*
+ * lcq_selftest_wait_timeout - exercise the bounded-wait error path on the GPU
+ * (measurement and reliability support; the paper has no counterpart). One
+ * CTA waits on an mbarrier phase that nothing completes, using the same
+ * bounded wait as every pipeline of the library; after about 2 seconds it gives
+ * up, sets LCQ_ERR_TIMEOUT in the workspace status word and returns, leaving
+ * the context usable. ws: at least 256 bytes of device memory.
+ */
+lcq_status lcq_selftest_wait_timeout(void *ws, void *stream);
+
 /* Static description of a status code; never NULL. */
 const char *lcq_status_string(lcq_status s);
 

@@ -24,7 +24,7 @@ LCQ_STE_IDENTITY, LCQ_STE_CLIPPED = 0, 1
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
-           "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error")
+           "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -63,6 +63,7 @@ _SIG = {
     "lcq_device_status": (ctypes.c_int, [_P, _P, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]),
     "lcq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "lcq_last_cuda_error": (ctypes.c_char_p, []),
+    "lcq_selftest_wait_timeout": (ctypes.c_int, [_P, _P]),
     "lcq_launch_count": (ctypes.c_uint64, []),
     "lcq_trace_enable": (ctypes.c_int, [ctypes.c_int]),
     "lcq_trace_read": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_double)]),
@@ -186,6 +187,11 @@ def lcq_device_status(ws, clear: bool = False, stream=None) -> int:
     _check(lib().lcq_device_status(_ptr(ws), _stream(stream), ctypes.byref(out), int(bool(clear))),
            "lcq_device_status")
     return int(out.value)
+
+
+def lcq_selftest_wait_timeout(ws, stream=None):
+    """Run the bounded-wait self-test kernel (about 2 s); the workspace status then reads LCQ_ERR_TIMEOUT."""
+    _check(lib().lcq_selftest_wait_timeout(_ptr(ws), _stream(stream)), "lcq_selftest_wait_timeout")
 
 
 def lcq_launch_count() -> int:

@@ -501,6 +501,25 @@ __global__ void reduce_partials_kernel(const float *__restrict__ partials, int n
     }
 }
 
+// ------------------------------------------------------------------ bounded-wait self-test
+
+// One thread waits on an mbarrier whose phase nothing completes: mbar_wait gives up after its
+// time limit, records LCQ_ERR_TIMEOUT and the kernel returns normally.
+__global__ void wait_timeout_selftest_kernel(int32_t *status) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+        (void)mbar_wait(&bar, 0, status);
+    }
+}
+
+cudaError_t launch_wait_timeout_selftest(int32_t *status, cudaStream_t st) {
+    wait_timeout_selftest_kernel<<<1, 32, 0, st>>>(status);
+    count_launch();
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ host launchers
 
 static int stream_grid(int64_t total, int num_sms) {

@@ -243,6 +243,13 @@ lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, 
     return LCQ_OK;
 }
 
+lcq_status lcq_selftest_wait_timeout(void *ws, void *stream) {
+    if (!ws) return LCQ_ERR_NULL;
+    if (reinterpret_cast<uintptr_t>(ws) & 255u) return LCQ_ERR_ALIGN;
+    Header *h = static_cast<Header *>(ws);
+    return cuda_status(launch_wait_timeout_selftest(&h->status, as_stream(stream)));
+}
+
 lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, uint8_t *packed,
                       uint8_t *codes, float *latent, double *mse, void *ws, size_t ws_bytes, void *stream) {
     LCQ_TRY(check_common(m, n, d));

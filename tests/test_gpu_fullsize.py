@@ -1,0 +1,132 @@
+"""Parity at the full sizes of the benchmarked workloads, through the same C-ABI calls bench.py makes.
+
+The oracle cannot recompute every output of these layers in seconds, so each test checks what it
+can exactly: the quantized codes over the whole matrix, sampled rows of every product computed one
+by one in fp64, and the weight-gradient sums through identities that hold at any size:
+    db[j]    = sum_t rowsum(dY)[t] * sum_g X[t, g*d + j]
+    dA[j][k] = sum_{t,g} X[t, g*d + j] * (dY Z)[t, g*d + k]
+Tolerances are those of the small parity tests (2e-2 of max|ref| for bf16 products and gradients)."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2606_10531_gb300 as lcq
+from paper_2606_10531_gb300 import workloads as wl
+from tests.gpu_util import TOL_BF16, dev, dev_bf16, empty_bf16, host_bf16, max_rel
+
+pytestmark = pytest.mark.gpu
+
+SEED = 0
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_10531_gb300 import build
+    build.build()
+    lcq.lib()
+
+
+def _latent_chunked(W, A, b, d, rows=2048):
+    out = np.empty(W.shape, dtype=np.float32)
+    for r0 in range(0, W.shape[0], rows):
+        out[r0:r0 + rows] = oracle.latent(W[r0:r0 + rows], A, b, d).astype(np.float32)
+    return out
+
+
+def _check_linear(mx, index):
+    import torch
+    m, n, d, N = mx.m, mx.n, mx.d, mx.N
+    W = wl.draw_W(mx, SEED, index)
+    A, b = wl.draw_A(mx, SEED, index), wl.draw_b(mx, SEED, index)
+    Xb, dYb = wl.draw_X(mx, SEED, index), wl.draw_dY(mx, SEED, index)
+    P = _latent_chunked(W, A, b, d)
+    del W
+    Z = oracle.quantize(P)
+
+    Xd, dYd, Ad, bd = dev_bf16(Xb), dev_bf16(dYb), dev(A), dev(b)
+    Y = empty_bf16(N, m)
+    saved = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    wsf = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d)
+    lcq.lcq_linear_fwd(Xd, dev(P), d, Ad, bd, Y, wsf, packed_saved=saved)
+    assert np.array_equal(saved.cpu().numpy(), oracle.pack2b(Z)), "integer weights differ"
+    dX = empty_bf16(N, n)
+    dP = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    dA = torch.empty((d, d), dtype=torch.float32, device="cuda")
+    db = torch.empty(d, dtype=torch.float32, device="cuda")
+    wsb = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, N, m, n, d)
+    lcq.lcq_linear_bwd(Xd, dYd, saved, m, n, d, Ad, bd, dP, dA, db, wsb, dX=dX)
+    assert lcq.lcq_device_status(wsf) == 0 and lcq.lcq_device_status(wsb) == 0
+
+    X, dY = wl.bf16_to_f32(Xb).astype(np.float64), wl.bf16_to_f32(dYb).astype(np.float64)
+    W_hat = oracle.decode(Z, A, b, d)
+    rng = np.random.default_rng(1234 + index)
+    toks = rng.choice(N, 8, replace=False)
+    rows = rng.choice(m, 8, replace=False)
+    # sampled rows of Y = X W_hat^T and dX = dY W_hat
+    Yg, dXg = host_bf16(Y), host_bf16(dX)
+    assert max_rel(Yg[toks], X[toks] @ W_hat.T) <= TOL_BF16
+    assert max_rel(dXg[toks], dY[toks] @ W_hat) <= TOL_BF16
+    # sampled rows of dP = (dY^T X)_g A
+    dW_rows = dY[:, rows].T @ X                                    # 8 x n
+    dP_ref = (dW_rows.reshape(8, n // d, d) @ A.astype(np.float64)).reshape(8, n)
+    assert max_rel(dP.cpu().numpy()[rows], dP_ref) <= TOL_BF16
+    # db, dA through their row-sum identities (any size)
+    rho = dY.sum(axis=1)
+    sig = X.reshape(N, n // d, d).sum(axis=1)
+    assert max_rel(db.cpu().numpy(), rho @ sig) <= TOL_BF16
+    T = (wl.bf16_to_f32(dYb) @ Z.astype(np.float32)).astype(np.float64)      # dY Z, N x n
+    dA_ref = np.einsum("tgj,tgk->jk", X.reshape(N, n // d, d), T.reshape(N, n // d, d))
+    assert max_rel(dA.cpu().numpy(), dA_ref) <= TOL_BF16
+
+
+def test_llama3_8b_gate_fwd_bwd_full_size():
+    mats = wl.llama3_8b_layer()
+    _check_linear(mats[4], 4)         # gate 14336 x 4096, d = 8, 16384 tokens
+
+
+def test_llama2_7b_gate_fwd_bwd_full_size_d4_outliers():
+    mats = wl.llama2_7b_projections(d=4)
+    _check_linear(mats[4], 4)         # gate 11008 x 4096, d = 4, 4096 tokens, 1% outlier channels x20
+
+
+@pytest.mark.parametrize("B", [1, 4, 16])
+def test_llama3_70b_gate_packed_product_full_size(B):
+    mx = wl.llama3_70b_gate_decode(B)[0]
+    packed = wl.draw_packed_codes(mx, SEED, 0)
+    A, b = wl.draw_A(mx, SEED, 0), wl.draw_b(mx, SEED, 0)
+    Xb = wl.draw_X(mx, SEED, B)
+    Y = empty_bf16(B, mx.m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, B, mx.m, mx.n, mx.d)
+    lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(packed), mx.n, mx.d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    rows = np.random.default_rng(99 + B).choice(mx.m, 64, replace=False)
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), packed[rows], A, b, mx.d, mx.n)   # B x 64
+    assert max_rel(host_bf16(Y)[:, rows], ref) <= TOL_BF16
+
+
+def test_llama3_70b_gate_bulk_encode_full_size():
+    import torch
+    mx = wl.llama3_70b_layer_encode()[4]       # gate 28672 x 8192, heavy-tailed, d = 8
+    W = wl.draw_W(mx, SEED, 4)
+    A, b = wl.draw_A(mx, SEED, 4), wl.draw_b(mx, SEED, 4)
+    packed = torch.empty((mx.m, mx.n // 4), dtype=torch.uint8, device="cuda")
+    mse = torch.empty(1, dtype=torch.float64, device="cuda")
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, mx.m, mx.n, mx.d)
+    lcq.lcq_encode(dev(W), dev(A), dev(b), mx.d, ws, packed=packed, mse=mse)
+    assert lcq.lcq_device_status(ws) == 0
+    got = packed.cpu().numpy()
+    sq, mismatch, near = 0.0, 0, 0
+    for r0 in range(0, mx.m, 2048):
+        ref = oracle.encode(W[r0:r0 + 2048], A, b, mx.d)
+        z = oracle.unpack2b(got[r0:r0 + 2048], mx.n)
+        keep = ~ref["near"]
+        mismatch += int(np.sum((z != ref["codes"]) & keep))
+        near += int(np.sum(ref["near"]))
+        sq += ref["mse"] * z.size
+    assert mismatch == 0
+    ref_mse = sq / (mx.m * mx.n)
+    assert abs(mse.item() - ref_mse) <= 1e-4 * ref_mse
+    print(f"near-boundary codes excluded: {near} of {mx.m * mx.n}")

@@ -256,3 +256,22 @@ def test_gemm_packed2b_matches_oracle(N, m, n, d):
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
     lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
+
+
+# ----------------------------------------------------------------------------- failure detection
+
+def test_bounded_wait_reports_timeout_and_context_stays_usable():
+    """A wait on a flag nothing sets gives up after its limit and reports LCQ_ERR_TIMEOUT (8)."""
+    import time
+    torch = T()
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    t0 = time.time()
+    lcq.lcq_selftest_wait_timeout(ws)
+    assert lcq.lcq_device_status(ws, clear=True) == 8
+    assert 1.0 < time.time() - t0 < 30.0
+    assert lcq.lcq_device_status(ws) == 0
+    # the context still works: a normal call afterwards
+    Z = np.random.default_rng(1).integers(0, 4, (4, 16)).astype(np.uint8)
+    packed = torch.empty((4, 4), dtype=torch.uint8, device="cuda")
+    lcq.lcq_pack2b(dev(Z), packed)
+    assert np.array_equal(packed.cpu().numpy(), oracle.pack2b(Z))
