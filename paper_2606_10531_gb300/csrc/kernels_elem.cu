@@ -119,28 +119,50 @@ __device__ void invert_warp(StreamSmem &s) {
 // whose value is then the low two bits of t (NaN -> 0: fmaxf drops the NaN).
 // Squared residual ||w - (A z + b)||^2 = ||A (u - z)||^2 = e^T (A^T A) e with e = u - z.
 
-// Packing without extracting the codes: bits(tc) = kMagicBits + z, so summing bits(tc_k) * 4^k over the
-// 16 codes of a thread (mod 2^32) gives the packed word plus kMagicBits * (4^0 + ... + 4^15), removed once.
-constexpr uint32_t kMagicBits = 0x4B400000u;                       // bits of 1.5 * 2^23
-constexpr uint32_t kPackBias = kMagicBits * 0x55555555u;           // kMagicBits * sum_{k<16} 4^k (mod 2^32)
+// Insert the two low bits of `src` (the code: tc = 1.5*2^23 + z) into `dst` at bit `pos` (ALU pipe).
+__device__ __forceinline__ uint32_t bfi2(uint32_t src, uint32_t dst, int pos) {
+    uint32_t r;
+    asm("bfi.b32 %0, %1, %2, %3, 2;" : "=r"(r) : "r"(src), "r"(dst), "r"(pos));
+    return r;
+}
+
+// Upper triangle of M = A^T A in the order the paired quadratic form consumes it (see quad_form).
+template <int D>
+struct QuadCoef {
+    float2 pair[D * D / 4];   // (Mu[i][j], Mu[i+1][j]) for even i, j = i+1..D-1
+    float diag[D / 2];        // Mu[i][i] for even i
+};
+
+// q = e^T M e = sum_i e_i s_i with s_i = M_ii e_i + 2 sum_{j>i} M_ij e_j, rows taken in pairs (i, i+1) so
+// that every column j > i feeds both rows with one packed fp32x2 FMA.
+template <int D>
+__device__ __forceinline__ float quad_form(const QuadCoef<D> &c, const float (&e)[D]) {
+    float2 eb[D];
+#pragma unroll
+    for (int j = 0; j < D; ++j) eb[j] = make_float2(e[j], e[j]);
+    float2 q2 = make_float2(0.0f, 0.0f);
+    int idx = 0;
+#pragma unroll
+    for (int i = 0; i < D; i += 2) {
+        float2 s2 = make_float2(c.diag[i / 2] * e[i], 0.0f);
+#pragma unroll
+        for (int j = i + 1; j < D; ++j) s2 = __ffma2_rn(c.pair[idx++], eb[j], s2);
+        q2 = __ffma2_rn(make_float2(e[i], e[i + 1]), s2, q2);
+    }
+    return q2.x + q2.y;
+}
 
 template <int D, bool kMse>
-__device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)[D / 2][D], const float (&Mu)[D * (D + 1) / 2],
-                                             const float2 (&bv2)[D / 2], uint32_t &zacc, int zshift, float (&u)[D],
+__device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)[D / 2][D], const QuadCoef<D> &qc,
+                                             const float2 (&c2)[D / 2], uint32_t &zacc, int zshift, float (&u)[D],
                                              float &sq) {
-    float v[D];
-#pragma unroll
-    for (int j = 0; j < D / 2; ++j) {
-        const float2 r = __fadd2_rn(make_float2(w[2 * j], w[2 * j + 1]), bv2[j]);   // w - b (bv2 holds -b)
-        v[2 * j] = r.x;
-        v[2 * j + 1] = r.y;
-    }
+    // u = A^{-1} w + c with c = -A^{-1} b
     float2 u2[D / 2];
 #pragma unroll
     for (int kp = 0; kp < D / 2; ++kp) {
-        float2 acc = make_float2(0.0f, 0.0f);
+        float2 acc = c2[kp];
 #pragma unroll
-        for (int j = 0; j < D; ++j) acc = __ffma2_rn(Ai2[kp][j], make_float2(v[j], v[j]), acc);
+        for (int j = 0; j < D; ++j) acc = __ffma2_rn(Ai2[kp][j], make_float2(w[j], w[j]), acc);
         u2[kp] = acc;
         u[2 * kp] = acc.x;
         u[2 * kp + 1] = acc.y;
@@ -151,8 +173,8 @@ __device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)
         const float2 t = __fadd2_rn(u2[kp], make_float2(kRoundMagic, kRoundMagic));
         const float tc0 = fminf(fmaxf(t.x, kRoundMagic), kRoundMagic + 3.0f);
         const float tc1 = fminf(fmaxf(t.y, kRoundMagic), kRoundMagic + 3.0f);
-        zacc += __float_as_uint(tc0) << (zshift + 4 * kp);
-        zacc += __float_as_uint(tc1) << (zshift + 4 * kp + 2);
+        zacc = bfi2(__float_as_uint(tc0), zacc, zshift + 4 * kp);
+        zacc = bfi2(__float_as_uint(tc1), zacc, zshift + 4 * kp + 2);
         if (kMse) {
             const float2 zf = __fadd2_rn(make_float2(tc0, tc1), make_float2(-kRoundMagic, -kRoundMagic));
             const float2 ee = __ffma2_rn(zf, make_float2(-1.0f, -1.0f), u2[kp]);
@@ -160,19 +182,7 @@ __device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)
             e[2 * kp + 1] = ee.y;
         }
     }
-    if (kMse) {
-        // e^T M e with the upper triangle of M (off-diagonal terms pre-doubled)
-        float q = 0.0f;
-        int idx = 0;
-#pragma unroll
-        for (int i = 0; i < D; ++i) {
-            float si = 0.0f;
-#pragma unroll
-            for (int j = i; j < D; ++j) si = fmaf(Mu[idx++], e[j], si);
-            q = fmaf(e[i], si, q);
-        }
-        sq += q;
-    }
+    if (kMse) sq += quad_form<D>(qc, e);
 }
 
 template <int D, bool kMse, bool kLatent>
@@ -203,21 +213,33 @@ encode_kernel(EncodeArgs a) {
     compute_bar();
     if (s.singular && blockIdx.x == 0 && threadIdx.x == 32) set_status(a.status, LCQ_ERR_SINGULAR);
 
-    float2 Ai2[D / 2][D], bv2[D / 2];
-    float Mu[D * (D + 1) / 2];
+    float2 Ai2[D / 2][D], c2[D / 2];
+    QuadCoef<D> qc;
 #pragma unroll
     for (int kp = 0; kp < D / 2; ++kp)
 #pragma unroll
         for (int j = 0; j < D; ++j) Ai2[kp][j] = make_float2(s.Ainv[(2 * kp) * D + j], s.Ainv[(2 * kp + 1) * D + j]);
+#pragma unroll
+    for (int kp = 0; kp < D / 2; ++kp) {
+        float c0 = 0.0f, c1 = 0.0f;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            c0 = fmaf(-s.Ainv[(2 * kp) * D + j], s.b[j], c0);
+            c1 = fmaf(-s.Ainv[(2 * kp + 1) * D + j], s.b[j], c1);
+        }
+        c2[kp] = make_float2(c0, c1);
+    }
     {
         int idx = 0;
 #pragma unroll
-        for (int i = 0; i < D; ++i)
+        for (int i = 0; i < D; i += 2) {
+            qc.diag[i / 2] = s.M[i * D + i];
+            // row i gets 2*M[i][j] for j > i; row i+1 gets M[i+1][i+1] at j = i+1, 2*M[i+1][j] beyond
 #pragma unroll
-            for (int j = i; j < D; ++j) Mu[idx++] = (i == j ? 1.0f : 2.0f) * s.M[i * D + j];
+            for (int j = i + 1; j < D; ++j)
+                qc.pair[idx++] = make_float2(2.0f * s.M[i * D + j], (j == i + 1 ? 1.0f : 2.0f) * s.M[(i + 1) * D + j]);
+        }
     }
-#pragma unroll
-    for (int i = 0; i < D / 2; ++i) bv2[i] = make_float2(-s.b[2 * i], -s.b[2 * i + 1]);
 
     const int t = threadIdx.x - 32;
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
@@ -246,7 +268,7 @@ encode_kernel(EncodeArgs a) {
                 }
                 float u[D];
                 float gsq = 0.0f;
-                encode_group<D, kMse>(w, Ai2, Mu, bv2, p, 2 * g * D, u, gsq);
+                encode_group<D, kMse>(w, Ai2, qc, c2, p, 2 * g * D, u, gsq);
                 if (g * D < valid) {
                     sq += gsq;
                     if (kLatent) {
@@ -256,7 +278,7 @@ encode_kernel(EncodeArgs a) {
                     }
                 }
             }
-            p -= kPackBias;
+
             if (valid == kPerThread) {
                 if (a.packed) *reinterpret_cast<uint32_t *>(a.packed + gidx / 4) = p;
                 if (a.codes) {
