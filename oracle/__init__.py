@@ -8,6 +8,7 @@ Pinned by tests/test_oracle_pins.py; every function has at least one pin that
 does not re-derive it from its own formula (closed forms, brute force,
 finite differences, hand-worked fixtures in tests/golden/).
 """
-from .lcvq import (BITS, ZMAX, SingularMatrix, brute_nearest, decode, encode, gemm_packed2b,  # noqa: F401
+from .lcvq import (BITS, DGE_GRAD_MAX, DGE_K, ZMAX, SingularMatrix, brute_nearest, decode, dge_f,  # noqa: F401
+                   dge_fprime, dge_grad, encode, gemm_packed2b,
                    init_codebook, inverse, latent, linear_bwd, linear_fwd, mse, near_boundary,
                    pack2b, quantize, round_clamp, unpack2b)

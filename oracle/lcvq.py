@@ -142,8 +142,36 @@ def linear_fwd(X, Z, A, b, d: int) -> np.ndarray:
     return _f64(X) @ decode(Z, A, b, d).T
 
 
+DGE_K = 5.0          # sharpness k of the differentiable gradient estimator (Sec. 4.4)
+DGE_GRAD_MAX = 3.0   # reading: cap on f'(x), which diverges at the rounding boundary (parity unpinned)
+
+
+def dge_f(x, k: float = DGE_K, delta: float = 1.0):
+    """Differentiable surrogate of rounding on one interval (Sec. 3.3, Eq. dge):
+    f(x) = delta/2 * (1 + sign(2x/delta - 1) * |2x/delta - 1|^(1/k))."""
+    y = 2.0 * _f64(x) / delta - 1.0
+    return delta / 2.0 * (1.0 + np.sign(y) * np.abs(y) ** (1.0 / k))
+
+
+def dge_fprime(x, k: float = DGE_K, delta: float = 1.0):
+    """f'(x) = (1/k) * |2x/delta - 1|^(1/k - 1) (Sec. 3.3); infinite at x = delta/2."""
+    y = np.abs(2.0 * _f64(x) / delta - 1.0)
+    with np.errstate(divide="ignore"):
+        return (1.0 / k) * y ** (1.0 / k - 1.0)
+
+
+def dge_grad(V, k: float = DGE_K, grad_max: float = DGE_GRAD_MAX):
+    """dz/dv of the DGE surrogate of clip(round(v), 0, 3) with delta = 1 (reading):
+    on [0, 3) v = n + x with x = v - floor(v), the surrogate is n + f(x) and its slope f'(x),
+    capped at grad_max; outside [0, 3) clip(round(.)) is flat and the slope is 0."""
+    V64 = _f64(V)
+    x = V64 - np.floor(V64)
+    g = np.minimum(dge_fprime(x, k), grad_max)
+    return np.where((V64 >= 0.0) & (V64 < ZMAX), g, 0.0)
+
+
 def linear_bwd(X, dY, Z, A, b, d: int, P=None, s: float = 1.0, t: float = 0.0,
-               ste: str = "identity") -> dict:
+               ste: str = "identity", dge_k: float = DGE_K, dge_grad_max: float = DGE_GRAD_MAX) -> dict:
     """Gradients of L with dL/dY = dY through Y = X W_hat^T, W_hat = decode(Z).
 
     The layer is linear in X, A, B and in z treated as a real vector, so:
@@ -154,7 +182,8 @@ def linear_bwd(X, dY, Z, A, b, d: int, P=None, s: float = 1.0, t: float = 0.0,
         dB     = sum_{r,g} dw_hat_{r,g}
     and the straight-through estimator dW_z/dW_p = 1 (Sec. 3.3) gives
     dP = dZ / s; with ste="clipped" the gradient is zeroed where
-    P/s + t lies outside [-1/2, 2^b - 1/2].
+    P/s + t lies outside [-1/2, 2^b - 1/2]; with ste="dge" it is scaled by the
+    slope of the differentiable gradient estimator at v = P/s + t (dge_grad).
     """
     X64, dY64, A64 = _f64(X), _f64(dY), _f64(A)
     What = decode(Z, A, b, d)
@@ -172,6 +201,12 @@ def linear_bwd(X, dY, Z, A, b, d: int, P=None, s: float = 1.0, t: float = 0.0,
         P32 = np.asarray(P, dtype=np.float32)
         V = ((P32 * (np.float32(1.0) / np.float32(s))).astype(np.float32) + np.float32(t)).astype(np.float64)
         dP = np.where((V >= -0.5) & (V <= ZMAX + 0.5), dP, 0.0)
+    elif ste == "dge":
+        if P is None:
+            raise ValueError("ste='dge' needs P")
+        P32 = np.asarray(P, dtype=np.float32)
+        V = ((P32 * (np.float32(1.0) / np.float32(s))).astype(np.float32) + np.float32(t)).astype(np.float64)
+        dP = dP * dge_grad(V, dge_k, dge_grad_max)
     elif ste != "identity":
         raise ValueError(f"unknown ste mode {ste!r}")
     return {"dX": dX, "dP": dP, "dA": dA, "db": db, "dW_hat": dWhat}

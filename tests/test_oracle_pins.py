@@ -297,3 +297,44 @@ def test_pack_unpack_round_trip():
     P = oracle.pack2b(Z)
     assert P.shape == (7, 16)
     assert np.array_equal(oracle.unpack2b(P, 64), Z)
+
+
+# ----------------------------------------------------------------------------- DGE (Sec. 3.3, Eq. dge)
+
+def test_dge_surrogate_endpoints_and_slope_closed_forms(golden_dir):
+    """f(0) = 0, f(delta/2) = delta/2, f(delta) = delta; f'(0) = f'(delta) = 1/k; f' = df/dx."""
+    for k in (1.0, 3.0, 5.0):
+        for delta in (1.0, 2.0):
+            assert math.isclose(oracle.dge_f(0.0, k, delta), 0.0, abs_tol=1e-15)
+            assert math.isclose(oracle.dge_f(delta / 2, k, delta), delta / 2, abs_tol=1e-15)
+            assert math.isclose(oracle.dge_f(delta, k, delta), delta, rel_tol=1e-15)
+            assert math.isclose(oracle.dge_fprime(0.0, k, delta), 1.0 / k, rel_tol=1e-15)
+            assert math.isclose(oracle.dge_fprime(delta, k, delta), 1.0 / k, rel_tol=1e-15)
+            for x in (0.1 * delta, 0.3 * delta, 0.7 * delta, 0.95 * delta):
+                h = 1e-6 * delta
+                fd = (oracle.dge_f(x + h, k, delta) - oracle.dge_f(x - h, k, delta)) / (2 * h)
+                assert math.isclose(oracle.dge_fprime(x, k, delta), fd, rel_tol=1e-6)
+    # the slope diverges at the boundary (the reason the implementation caps it)
+    assert np.isinf(oracle.dge_fprime(0.5, 5.0))
+
+
+def test_dge_with_k1_is_the_identity_estimator_inside_the_range():
+    """k = 1 makes f(x) = x, slope 1: DGE reduces to the straight-through estimator on [0, 3)."""
+    v = np.array([-0.7, -0.1, 0.0, 0.4, 1.5, 2.9, 3.0, 3.6])
+    g = oracle.dge_grad(v, k=1.0, grad_max=10.0)
+    assert list(g) == [0.0, 0.0, 1.0, 1.0, 1.0, 1.0, 0.0, 0.0]
+    d, N, m, n = 4, 2, 3, 8
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    P = RNG.uniform(0.01, 2.99, (m, n)).astype(np.float32)
+    X, dY = RNG.normal(size=(N, n)), RNG.normal(size=(N, m))
+    Z = oracle.quantize(P)
+    ste = oracle.linear_bwd(X, dY, Z, A, b, d)["dP"]
+    dge = oracle.linear_bwd(X, dY, Z, A, b, d, P=P, ste="dge", dge_k=1.0, dge_grad_max=10.0)["dP"]
+    np.testing.assert_allclose(dge, ste, rtol=1e-15)
+
+
+def test_dge_slope_is_periodic_and_capped():
+    v = np.array([0.2, 1.2, 2.2, 0.5, 1.5, 0.49999])
+    g = oracle.dge_grad(v, k=5.0, grad_max=3.0)
+    np.testing.assert_allclose(g[:3], g[0], rtol=1e-12)
+    assert g[3] == 3.0 and g[4] == 3.0 and g[5] == 3.0
