@@ -62,18 +62,27 @@ typedef enum lcq_op {
     LCQ_OP_GEMM_PACKED2B = 4
 } lcq_op;
 
-/* Straight-through estimator variants for dP (Sec. 3.3). */
+/* Gradient estimators for dP through the rounding (Sec. 3.3). */
 typedef enum lcq_ste_mode {
     LCQ_STE_IDENTITY = 0, /* dW_z/dW_p = 1 everywhere (the paper's STE)                  */
-    LCQ_STE_CLIPPED = 1   /* zero where P/s + t lies outside [-1/2, 7/2]                 */
+    LCQ_STE_CLIPPED = 1,  /* zero where P/s + t lies outside [-1/2, 7/2]                 */
+    LCQ_STE_DGE = 2       /* differentiable gradient estimator (Eq. dge), see lcq_opts */
 } lcq_ste_mode;
 
-/* Options of the training calls. NULL means {1, 0, LCQ_STE_IDENTITY}. */
+/*
+ * Options of the training calls. NULL means {1, 0, LCQ_STE_IDENTITY, 0, 5, 3}.
+ * LCQ_STE_DGE scales dP by the slope of the estimator at v = P/s + t: on [0, 3),
+ * with x = v - floor(v) (interval delta = 1), min(dge_grad_max, (1/k)|2x - 1|^(1/k - 1));
+ * 0 outside [0, 3). dge_k and dge_grad_max <= 0 select the defaults k = 5 (the
+ * paper's setting) and a cap of 3 (the paper does not state a cap).
+ */
 typedef struct lcq_opts {
     float latent_scale;   /* s: integer weights are clip(round(P/s + t), 0, 3); must be != 0 */
     float latent_offset;  /* t                                                                 */
     int32_t ste_mode;     /* lcq_ste_mode                                                      */
     int32_t reserved;     /* must be 0                                                         */
+    float dge_k;          /* DGE sharpness k                                                   */
+    float dge_grad_max;   /* DGE slope cap                                                     */
 } lcq_opts;
 
 /*
@@ -143,7 +152,7 @@ lcq_status lcq_linear_fwd(const uint16_t *X, int64_t N, const float *P, int64_t 
  *   dA[j][k] = sum_{r,g} dW_hat[r, g*d + j] * z[r, g*d + k]     [d][d] fp32
  *   db[j]    = sum_{r,g} dW_hat[r, g*d + j]                     [d] fp32
  * X [N][n] bf16, dY [N][m] bf16, packed_saved [m][n/4] from lcq_linear_fwd,
- * P [m][n] fp32 (read only in CLIPPED mode; may be NULL otherwise).
+ * P [m][n] fp32 (read only in CLIPPED and DGE modes; may be NULL otherwise).
  * dX may be NULL (skips the dX GEMM). dA and db are overwritten, not
  * accumulated; the sums are taken in a fixed order (bitwise reproducible).
  * Needs lcq_workspace_size(LCQ_OP_LINEAR_BWD, N, m, n, d).

@@ -19,7 +19,7 @@ STATUS_NAMES = {0: "LCQ_OK", 1: "LCQ_ERR_NULL", 2: "LCQ_ERR_SHAPE", 3: "LCQ_ERR_
                 5: "LCQ_ERR_WORKSPACE", 6: "LCQ_ERR_CUDA", 7: "LCQ_ERR_SINGULAR", 8: "LCQ_ERR_TIMEOUT",
                 9: "LCQ_ERR_ARG", 10: "LCQ_ERR_LIMIT"}
 LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B = 1, 2, 3, 4
-LCQ_STE_IDENTITY, LCQ_STE_CLIPPED = 0, 1
+LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
@@ -43,7 +43,8 @@ class LCQError(RuntimeError):
 
 class lcq_opts(ctypes.Structure):
     _fields_ = [("latent_scale", ctypes.c_float), ("latent_offset", ctypes.c_float),
-                ("ste_mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("ste_mode", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("dge_k", ctypes.c_float), ("dge_grad_max", ctypes.c_float)]
 
 
 _P = ctypes.c_void_p
@@ -115,8 +116,8 @@ def _stream(stream):
     return ctypes.c_void_p(stream.cuda_stream)
 
 
-def _opts(latent_scale=1.0, latent_offset=0.0, ste_mode=LCQ_STE_IDENTITY):
-    return lcq_opts(float(latent_scale), float(latent_offset), int(ste_mode), 0)
+def _opts(latent_scale=1.0, latent_offset=0.0, ste_mode=LCQ_STE_IDENTITY, dge_k=0.0, dge_grad_max=0.0):
+    return lcq_opts(float(latent_scale), float(latent_offset), int(ste_mode), 0, float(dge_k), float(dge_grad_max))
 
 
 # ----------------------------------------------------------------------------- entry points
@@ -158,9 +159,10 @@ def lcq_linear_fwd(X, P, d: int, A, b, Y, ws, packed_saved=None, latent_scale=1.
 
 
 def lcq_linear_bwd(X, dY, packed_saved, m: int, n: int, d: int, A, b, dP, dA, db, ws, dX=None, P=None,
-                   latent_scale=1.0, latent_offset=0.0, ste_mode=LCQ_STE_IDENTITY, stream=None):
+                   latent_scale=1.0, latent_offset=0.0, ste_mode=LCQ_STE_IDENTITY, dge_k=0.0, dge_grad_max=0.0,
+                   stream=None):
     N = X.shape[0]
-    o = _opts(latent_scale, latent_offset, ste_mode)
+    o = _opts(latent_scale, latent_offset, ste_mode, dge_k, dge_grad_max)
     _check(lib().lcq_linear_bwd(_ptr(X), _ptr(dY), _ptr(packed_saved), _ptr(P), N, m, n, d, _ptr(A), _ptr(b),
                                 ctypes.byref(o), _ptr(dX), _ptr(dP), _ptr(dA), _ptr(db), _ptr(ws), ws.numel(),
                                 _stream(stream)), "lcq_linear_bwd")

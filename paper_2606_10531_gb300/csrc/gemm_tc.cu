@@ -240,6 +240,17 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                                 const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
                                 if (!(u >= -0.5f && u <= 3.5f)) out[k] = 0.0f;
                             }
+                        } else if (p.dw.ste_mode == LCQ_STE_DGE) {
+                            // slope of the differentiable gradient estimator (Eq. dge) at v, delta = 1
+#pragma unroll
+                            for (int k = 0; k < D; ++k) {
+                                const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
+                                const float x = u - floorf(u);
+                                const float y = fabsf(2.0f * x - 1.0f);
+                                float gs = fminf(p.dw.dge_cap, p.dw.dge_inv_k * exp2f(p.dw.dge_exp * log2f(y)));
+                                if (!(u >= 0.0f && u < 3.0f)) gs = 0.0f;
+                                out[k] *= gs;
+                            }
                         }
 #pragma unroll
                         for (int k = 0; k < D; k += 4)

@@ -75,6 +75,9 @@ struct DwEpilogue {
     float inv_s, t;
     int ste_mode;
     int d;
+    float dge_inv_k;         // 1/k
+    float dge_exp;           // 1/k - 1
+    float dge_cap;
 };
 
 struct GemmProblem {

@@ -131,8 +131,9 @@ static lcq_status cuda_status(cudaError_t e) {
     return LCQ_ERR_CUDA;
 }
 
-static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste) {
-    float s = 1.0f;
+static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste, float *dge_k = nullptr,
+                          float *dge_cap = nullptr) {
+    float s = 1.0f, k = 5.0f, cap = 3.0f;
     t = 0.0f;
     ste = LCQ_STE_IDENTITY;
     if (o) {
@@ -140,10 +141,14 @@ static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste) {
         t = o->latent_offset;
         ste = o->ste_mode;
         if (o->reserved != 0) return LCQ_ERR_ARG;
+        if (o->dge_k > 0.0f) k = o->dge_k;
+        if (o->dge_grad_max > 0.0f) cap = o->dge_grad_max;
     }
-    if (!(s != 0.0f) || !isfinite(s) || !isfinite(t)) return LCQ_ERR_ARG;
-    if (ste != LCQ_STE_IDENTITY && ste != LCQ_STE_CLIPPED) return LCQ_ERR_UNSUPPORTED;
+    if (!(s != 0.0f) || !isfinite(s) || !isfinite(t) || !isfinite(k) || !isfinite(cap)) return LCQ_ERR_ARG;
+    if (ste != LCQ_STE_IDENTITY && ste != LCQ_STE_CLIPPED && ste != LCQ_STE_DGE) return LCQ_ERR_UNSUPPORTED;
     inv_s = 1.0f / s;
+    if (dge_k) *dge_k = k;
+    if (dge_cap) *dge_cap = cap;
     return LCQ_OK;
 }
 
@@ -344,13 +349,13 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
                           uint16_t *dX, float *dP, float *dA, float *db, void *ws, size_t ws_bytes, void *stream) {
     LCQ_TRY(check_common(m, n, d));
     if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
-    float inv_s, t;
+    float inv_s, t, dge_k, dge_cap;
     int ste;
-    LCQ_TRY(opts_of(opts, inv_s, t, ste));
+    LCQ_TRY(opts_of(opts, inv_s, t, ste, &dge_k, &dge_cap));
     LCQ_TRY(check_tensor(X, N * n));
     LCQ_TRY(check_tensor(dY, N * m));
     LCQ_TRY(check_tensor(packed_saved, m * n));
-    LCQ_TRY(check_tensor(P, m * n, ste == LCQ_STE_CLIPPED));
+    LCQ_TRY(check_tensor(P, m * n, ste != LCQ_STE_IDENTITY));
     LCQ_TRY(check_tensor(dX, N * n, false));
     LCQ_TRY(check_tensor(dP, m * n));
     if (!A || !b || !dA || !db) return LCQ_ERR_NULL;
@@ -394,7 +399,10 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
     g.b = {X, n, true};
     g.dw.packed = packed_saved;
     g.dw.A = A;
-    g.dw.P = ste == LCQ_STE_CLIPPED ? P : nullptr;
+    g.dw.P = ste != LCQ_STE_IDENTITY ? P : nullptr;
+    g.dw.dge_inv_k = 1.0f / dge_k;
+    g.dw.dge_exp = 1.0f / dge_k - 1.0f;
+    g.dw.dge_cap = dge_cap;
     g.dw.dP = dP;
     g.dw.partials = partials;
     g.dw.inv_s = inv_s;

@@ -77,7 +77,7 @@ def test_encode_validation(L):
 
 
 def test_linear_validation(L):
-    o = lcq.lcq_opts(1.0, 0.0, 0, 0)
+    o = lcq.lcq_opts(1.0, 0.0, 0, 0, 0.0, 0.0)
     big = 1 << 30
     fwd = lambda **k: L.lcq_linear_fwd(k.get("X", FAKE), k.get("N", 4), k.get("P", FAKE), k.get("m", 8),  # noqa: E731
                                        k.get("n", 16), k.get("d", 8), FAKE, FAKE, k.get("o", ctypes.byref(o)),
@@ -87,14 +87,16 @@ def test_linear_validation(L):
     assert fwd(X=None) == NULL
     assert fwd(Y=FAKE + 2) == ALIGN
     assert fwd(ws_bytes=8) == WS
-    bad = lcq.lcq_opts(0.0, 0.0, 0, 0)
+    bad = lcq.lcq_opts(0.0, 0.0, 0, 0, 0.0, 0.0)
     assert fwd(o=ctypes.byref(bad)) == ARG
-    bad_mode = lcq.lcq_opts(1.0, 0.0, 7, 0)
+    bad_mode = lcq.lcq_opts(1.0, 0.0, 7, 0, 0.0, 0.0)
     assert fwd(o=ctypes.byref(bad_mode)) == UNSUP
     bwd = lambda **k: L.lcq_linear_bwd(FAKE, FAKE, FAKE, k.get("P", None), 4, 8, 16, 8, FAKE, FAKE,  # noqa: E731
                                        k.get("o", None), None, FAKE, k.get("dA", FAKE), FAKE, FAKE, big, None)
-    clipped = lcq.lcq_opts(1.0, 0.0, 1, 0)
+    clipped = lcq.lcq_opts(1.0, 0.0, 1, 0, 0.0, 0.0)
     assert bwd(o=ctypes.byref(clipped)) == NULL     # CLIPPED needs P
+    dge = lcq.lcq_opts(1.0, 0.0, 2, 0, 5.0, 3.0)
+    assert bwd(o=ctypes.byref(dge)) == NULL         # DGE needs P
     assert bwd(dA=None) == NULL
 
 

@@ -170,13 +170,13 @@ def _linear_inputs(N, m, n, d, seed):
 
 
 @pytest.mark.parametrize("N,m,n,d", LINEAR_CASES)
-@pytest.mark.parametrize("ste", ["identity", "clipped"])
+@pytest.mark.parametrize("ste", ["identity", "clipped", "dge"])
 def test_linear_fwd_bwd_match_oracle(N, m, n, d, ste):
     torch = T()
     P, A, b, Xb, dYb = _linear_inputs(N, m, n, d, seed=N * 31 + m + n + d)
     X, dY = wl.bf16_to_f32(Xb), wl.bf16_to_f32(dYb)
     s, t = (1.0, 0.0) if ste == "identity" else (0.5, 0.75)
-    mode = lcq.LCQ_STE_IDENTITY if ste == "identity" else lcq.LCQ_STE_CLIPPED
+    mode = {"identity": lcq.LCQ_STE_IDENTITY, "clipped": lcq.LCQ_STE_CLIPPED, "dge": lcq.LCQ_STE_DGE}[ste]
     Z = oracle.quantize(P, s, t)
     Yref = oracle.linear_fwd(X, Z, A, b, d)
     g = oracle.linear_bwd(X, dY, Z, A, b, d, P=P, s=s, t=t, ste=ste)
