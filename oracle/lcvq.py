@@ -250,6 +250,16 @@ def init_codebook(G, bits: int = BITS):
     return A, B
 
 
+def init_latent(Z, m: int, n: int, bits: int = BITS):
+    """Latent (proxy) weights from integer weights, Eq. xavier_preprocess: W_p = s (W_z - t) with
+    s = 2a/(2^b - 1), t = (2^b - 1)/2, a = sqrt(6/(m+n)). Returns (W_p fp64, s, t)."""
+    a = np.sqrt(6.0 / (m + n))
+    L = (1 << bits) - 1
+    s = 2.0 * a / L
+    t = L / 2.0
+    return s * (_f64(Z) - t), s, t
+
+
 def brute_nearest(W, A, b, d: int):
     """Exhaustive nearest codeword over all 4^d codewords (Eq. vq_assign on Eq. lc_codebook).
 

@@ -338,3 +338,22 @@ def test_dge_slope_is_periodic_and_capped():
     g = oracle.dge_grad(v, k=5.0, grad_max=3.0)
     np.testing.assert_allclose(g[:3], g[0], rtol=1e-12)
     assert g[3] == 3.0 and g[4] == 3.0 and g[5] == 3.0
+
+
+# ----------------------------------------------------------------------------- initialisation (N2)
+
+def test_xavier_preprocess_constants_and_levels(golden_dir):
+    c = read_keyed("xavier_constants.txt")
+    m, n = int(c["m"][0]), int(c["n"][0])
+    P, s, t = oracle.init_latent(np.array([[0, 1, 2, 3]]), m, n)
+    assert math.isclose(s, c["s"][0], rel_tol=1e-14) and t == c["t"][0]
+    a = c["a"][0]
+    np.testing.assert_allclose(P[0], [-a, -a / 3, a / 3, a], rtol=1e-14)
+
+
+def test_xavier_preprocess_preserves_the_integer_weights():
+    """Sec. 3.4: quantizing the preprocessed latents with the same (s, t) returns the integer weights."""
+    for (m, n) in ((4096, 4096), (14336, 4096), (1024, 4096)):
+        Z = RNG.integers(0, 4, (16, 64)).astype(np.uint8)
+        P, s, t = oracle.init_latent(Z, m, n)
+        assert np.array_equal(oracle.quantize(P.astype(np.float32), s, t), Z)
