@@ -202,6 +202,24 @@ lcq_status lcq_gemm_packed2b_noalloc(const uint16_t *X, int64_t N, const uint8_t
                                      int32_t *device_status, void *stream);
 
 /*
+ * lcq_init_codebook - codebook initialisation of Sec. 2.2 Eq. init_ab for b = 2:
+ *   A = s G,  b = -s G mu 1,  mu = (2^b - 1)/2 = 1.5,  s = sqrt(12 / (2^{2b} - 1)) = sqrt(0.8)
+ * G [d][d] fp32 (a random orthogonal matrix chosen by the caller), A [d][d] and b [d] fp32 outputs;
+ * all device pointers. Over all 4^d codewords the codebook then has mean 0 and covariance G G^T.
+ */
+lcq_status lcq_init_codebook(const float *G, int d, float *A, float *b, void *stream);
+
+/*
+ * lcq_init_latent - latent (proxy) weights from integer weights, Sec. 3.4 Eq. xavier_preprocess:
+ *   P = s (z - t),  s = 2a / (2^b - 1),  t = (2^b - 1) / 2,  a = sqrt(6 / (m + n))
+ * packed [m][n/4] uint8 codes in, P [m][n] fp32 out (device). *s_out and *t_out (host, may be NULL)
+ * receive s and t as used (fp32): passing them as lcq_opts.latent_scale / latent_offset makes
+ * lcq_linear_fwd quantize P back to exactly the same codes.
+ */
+lcq_status lcq_init_latent(const uint8_t *packed, int64_t m, int64_t n, float *P, float *s_out, float *t_out,
+                           void *stream);
+
+/*
  * lcq_device_status - synchronise `stream`, then copy the workspace's device
  * status word (LCQ_OK or a device-detected lcq_status) to *status_out and,
  * if clear != 0, reset it to LCQ_OK.

@@ -24,7 +24,8 @@ LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
-           "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout")
+           "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout",
+           "lcq_init_codebook", "lcq_init_latent")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -65,6 +66,9 @@ _SIG = {
     "lcq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "lcq_last_cuda_error": (ctypes.c_char_p, []),
     "lcq_selftest_wait_timeout": (ctypes.c_int, [_P, _P]),
+    "lcq_init_codebook": (ctypes.c_int, [_P, ctypes.c_int, _P, _P, _P]),
+    "lcq_init_latent": (ctypes.c_int, [_P, _I64, _I64, _P, ctypes.POINTER(ctypes.c_float),
+                                       ctypes.POINTER(ctypes.c_float), _P]),
     "lcq_launch_count": (ctypes.c_uint64, []),
     "lcq_trace_enable": (ctypes.c_int, [ctypes.c_int]),
     "lcq_trace_read": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_double)]),
@@ -194,6 +198,19 @@ def lcq_device_status(ws, clear: bool = False, stream=None) -> int:
 def lcq_selftest_wait_timeout(ws, stream=None):
     """Run the bounded-wait self-test kernel (about 2 s); the workspace status then reads LCQ_ERR_TIMEOUT."""
     _check(lib().lcq_selftest_wait_timeout(_ptr(ws), _stream(stream)), "lcq_selftest_wait_timeout")
+
+
+def lcq_init_codebook(G, d: int, A, b, stream=None):
+    _check(lib().lcq_init_codebook(_ptr(G), d, _ptr(A), _ptr(b), _stream(stream)), "lcq_init_codebook")
+
+
+def lcq_init_latent(packed, n: int, P, stream=None):
+    """Writes P = s (z - t) (Eq. xavier_preprocess); returns (s, t) for lcq_linear_fwd's latent affine."""
+    m = packed.shape[0]
+    s_, t_ = ctypes.c_float(0.0), ctypes.c_float(0.0)
+    _check(lib().lcq_init_latent(_ptr(packed), m, n, _ptr(P), ctypes.byref(s_), ctypes.byref(t_), _stream(stream)),
+           "lcq_init_latent")
+    return float(s_.value), float(t_.value)
 
 
 def lcq_launch_count() -> int:

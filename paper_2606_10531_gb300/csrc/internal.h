@@ -52,6 +52,9 @@ cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cu
 cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, int num_sms, cudaStream_t st);
 cudaError_t launch_wait_timeout_selftest(int32_t *status, cudaStream_t st);
+cudaError_t launch_init_codebook(const float *G, int d, float *A, float *b, cudaStream_t st);
+cudaError_t launch_init_latent(const uint8_t *packed, int64_t total, float s, float t, float *P, int num_sms,
+                               cudaStream_t st);
 cudaError_t launch_reduce_partials(const float *partials, int nparts, int d, float *dA, float *db, cudaStream_t st);
 
 // ---------------------------------------------------------------- tensor-core GEMM

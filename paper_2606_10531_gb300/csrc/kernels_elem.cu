@@ -523,6 +523,66 @@ __global__ void reduce_partials_kernel(const float *__restrict__ partials, int n
     }
 }
 
+// ------------------------------------------------------------------ initialisation (Eq. init_ab, Eq. xavier_preprocess)
+
+__global__ void init_codebook_kernel(const float *__restrict__ G, int d, float *A, float *b) {
+    const float sc = sqrtf(12.0f / 15.0f);   // s = sqrt(12 / (2^{2b} - 1)), b = 2
+    const int i = threadIdx.x;
+    if (i < d * d) A[i] = sc * G[i];
+    if (i < d) {
+        float acc = 0.0f;
+        for (int k = 0; k < d; ++k) acc += G[i * d + k];
+        b[i] = -sc * 1.5f * acc;             // -s G (mu 1), mu = 1.5
+    }
+}
+
+__global__ void __launch_bounds__(256)
+init_latent_kernel(const uint8_t *__restrict__ packed, int64_t total, float s, float t, float *__restrict__ P) {
+    const int64_t nslices = (total + 15) / 16;
+    for (int64_t sl = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; sl < nslices;
+         sl += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gidx = sl * 16;
+        const int valid = static_cast<int>((total - gidx) < 16 ? (total - gidx) : 16);
+        uint32_t w = 0;
+        if (valid == 16) {
+            w = __ldg(reinterpret_cast<const uint32_t *>(packed + gidx / 4));
+        } else {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (k < valid / 4) w |= static_cast<uint32_t>(packed[gidx / 4 + k]) << (8 * k);
+        }
+        float v[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = s * (static_cast<float>((w >> (2 * k)) & 3u) - t);
+        if (valid == 16) {
+            float4 *dst = reinterpret_cast<float4 *>(P + gidx);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        } else {
+#pragma unroll
+            for (int k = 0; k < 16; ++k)
+                if (k < valid) P[gidx + k] = v[k];
+        }
+    }
+}
+
+cudaError_t launch_init_codebook(const float *G, int d, float *A, float *b, cudaStream_t st) {
+    init_codebook_kernel<<<1, 64, 0, st>>>(G, d, A, b);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_init_latent(const uint8_t *packed, int64_t total, float s, float t, float *P, int num_sms,
+                               cudaStream_t st) {
+    const int64_t nslices = (total + 15) / 16;
+    int64_t grid = (nslices + 255) / 256;
+    if (grid > 8LL * num_sms) grid = 8LL * num_sms;
+    if (grid < 1) grid = 1;
+    init_latent_kernel<<<static_cast<int>(grid), 256, 0, st>>>(packed, total, s, t, P);
+    count_launch();
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ bounded-wait self-test
 
 // One thread waits on an mbarrier whose phase nothing completes: mbar_wait gives up after its

@@ -248,6 +248,28 @@ lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, 
     return LCQ_OK;
 }
 
+lcq_status lcq_init_codebook(const float *G, int d, float *A, float *b, void *stream) {
+    if (d != 4 && d != 8) return LCQ_ERR_UNSUPPORTED;
+    if (!G || !A || !b) return LCQ_ERR_NULL;
+    return cuda_status(launch_init_codebook(G, d, A, b, as_stream(stream)));
+}
+
+lcq_status lcq_init_latent(const uint8_t *packed, int64_t m, int64_t n, float *P, float *s_out, float *t_out,
+                           void *stream) {
+    if (m < 0 || n < 0 || n % 4 != 0) return LCQ_ERR_SHAPE;
+    if (m + n == 0) return LCQ_ERR_SHAPE;
+    const double a = sqrt(6.0 / static_cast<double>(m + n));
+    const float s = static_cast<float>(2.0 * a / 3.0);
+    const float t = 1.5f;
+    if (s_out) *s_out = s;
+    if (t_out) *t_out = t;
+    const int64_t mn = m * n;
+    if (mn == 0) return LCQ_OK;
+    LCQ_TRY(check_tensor(packed, mn));
+    LCQ_TRY(check_tensor(P, mn));
+    return cuda_status(launch_init_latent(packed, mn, s, t, P, num_sms_current(), as_stream(stream)));
+}
+
 lcq_status lcq_selftest_wait_timeout(void *ws, void *stream) {
     if (!ws) return LCQ_ERR_NULL;
     if (reinterpret_cast<uintptr_t>(ws) & 255u) return LCQ_ERR_ALIGN;

@@ -275,3 +275,41 @@ def test_bounded_wait_reports_timeout_and_context_stays_usable():
     packed = torch.empty((4, 4), dtype=torch.uint8, device="cuda")
     lcq.lcq_pack2b(dev(Z), packed)
     assert np.array_equal(packed.cpu().numpy(), oracle.pack2b(Z))
+
+
+# ----------------------------------------------------------------------------- initialisation
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_init_codebook_matches_oracle(d):
+    torch = T()
+    G = np.linalg.qr(np.random.default_rng(40 + d).normal(size=(d, d)))[0].astype(np.float32)
+    A = torch.empty((d, d), dtype=torch.float32, device="cuda")
+    b = torch.empty(d, dtype=torch.float32, device="cuda")
+    lcq.lcq_init_codebook(dev(G), d, A, b)
+    Aref, bref = oracle.init_codebook(G.astype(np.float64))
+    np.testing.assert_allclose(A.cpu().numpy(), Aref, rtol=1e-6, atol=1e-7)
+    np.testing.assert_allclose(b.cpu().numpy(), bref, rtol=1e-5, atol=1e-6)
+
+
+@pytest.mark.parametrize("m,n", [(4096, 4096), (37, 24), (300, 1028)])
+def test_init_latent_matches_oracle_and_requantizes_to_the_same_codes(m, n):
+    torch = T()
+    d = 4
+    Z = np.random.default_rng(m + n).integers(0, 4, (m, n)).astype(np.uint8)
+    packed = dev(oracle.pack2b(Z))
+    P = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    s, t = lcq.lcq_init_latent(packed, n, P)
+    Pref, sref, tref = oracle.init_latent(Z, m, n)
+    assert abs(s - sref) <= 1e-7 * sref and t == tref
+    np.testing.assert_allclose(P.cpu().numpy(), Pref, rtol=2e-7, atol=1e-9)
+    # forward quantization with the returned (s, t) gives back exactly the integer weights
+    if n % 8 == 0:
+        A = dev(np.eye(d, dtype=np.float32))
+        bz = dev(np.zeros(d, np.float32))
+        N = 1
+        X = torch.zeros((N, n), dtype=torch.bfloat16, device="cuda")
+        Y = torch.empty((N, m), dtype=torch.bfloat16, device="cuda")
+        saved = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+        ws = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d)
+        lcq.lcq_linear_fwd(X, P, d, A, bz, Y, ws, packed_saved=saved, latent_scale=s, latent_offset=t)
+        assert np.array_equal(saved.cpu().numpy(), oracle.pack2b(Z))
