@@ -9,6 +9,7 @@ does not re-derive it from its own formula (closed forms, brute force,
 finite differences, hand-worked fixtures in tests/golden/).
 """
 from .lcvq import (BITS, DGE_GRAD_MAX, DGE_K, ZMAX, SingularMatrix, brute_nearest, decode, dge_f,  # noqa: F401
-                   dge_fprime, dge_grad, encode, gemm_packed2b, init_latent,
+                   dge_fprime, dge_grad, encode, gemm_packed2b, gemm_packed2b_hadamard, hadamard_block,
+                   hadamard_rotate, init_latent,
                    init_codebook, inverse, latent, linear_bwd, linear_fwd, mse, near_boundary,
                    pack2b, quantize, round_clamp, unpack2b)

@@ -260,6 +260,31 @@ def init_latent(Z, m: int, n: int, bits: int = BITS):
     return s * (_f64(Z) - t), s, t
 
 
+def hadamard_block(n: int, max_block: int = 32768) -> int:
+    """Block size of the incoherence rotation (reading): the largest power of two dividing n, at most max_block."""
+    bsz = 1
+    while n % (bsz * 2) == 0 and bsz * 2 <= max_block:
+        bsz *= 2
+    return bsz
+
+
+def hadamard_rotate(M, n: int):
+    """Right-multiply the rows of M by the normalized block-diagonal Walsh-Hadamard matrix H of size n
+    (blocks of hadamard_block(n)); H is symmetric and orthogonal (Sec. 2.2 incoherence processing, reading)."""
+    import scipy.linalg
+    bsz = hadamard_block(n)
+    Hb = scipy.linalg.hadamard(bsz).astype(np.float64) / np.sqrt(bsz)
+    M64 = _f64(M)
+    rows = M64.shape[0]
+    return (M64.reshape(rows, n // bsz, bsz) @ Hb).reshape(rows, n)
+
+
+def gemm_packed2b_hadamard(X, packed, A, b, d: int, n: int) -> np.ndarray:
+    """Deployment product with online rotation of the activations: Y = (X H) W_hat^T, where the
+    codes encode the rotated weights W H (App. Inference Speed: Hadamard transform, then the product)."""
+    return gemm_packed2b(hadamard_rotate(X, n), packed, A, b, d, n)
+
+
 def brute_nearest(W, A, b, d: int):
     """Exhaustive nearest codeword over all 4^d codewords (Eq. vq_assign on Eq. lc_codebook).
 

@@ -357,3 +357,32 @@ def test_xavier_preprocess_preserves_the_integer_weights():
         Z = RNG.integers(0, 4, (16, 64)).astype(np.uint8)
         P, s, t = oracle.init_latent(Z, m, n)
         assert np.array_equal(oracle.quantize(P.astype(np.float32), s, t), Z)
+
+
+# ----------------------------------------------------------------------------- Hadamard rotation (N3)
+
+def test_hadamard_blocks_are_the_largest_power_of_two_dividing_n():
+    assert [oracle.hadamard_block(n) for n in (8, 24, 4096, 8192, 11008, 14336, 28672)] == \
+        [8, 8, 4096, 8192, 256, 2048, 4096]
+
+
+@pytest.mark.parametrize("n", [8, 24, 64, 96])
+def test_hadamard_rotation_is_orthogonal_and_self_inverse(n):
+    X = RNG.normal(size=(3, n))
+    Xr = oracle.hadamard_rotate(X, n)
+    np.testing.assert_allclose(np.linalg.norm(Xr, axis=1), np.linalg.norm(X, axis=1), rtol=1e-12)
+    np.testing.assert_allclose(oracle.hadamard_rotate(Xr, n), X, atol=1e-12)
+    # the first row of a Sylvester block is constant: column 0 of each block is the block mean times sqrt(bsz)
+    bsz = oracle.hadamard_block(n)
+    np.testing.assert_allclose(Xr[:, 0], X[:, :bsz].sum(axis=1) / np.sqrt(bsz), rtol=1e-12)
+
+
+def test_rotation_cancels_through_the_product():
+    """Rotating the activations and the weights by the same orthogonal H leaves Y unchanged:
+    gemm_packed2b_hadamard(X H, codes) = gemm_packed2b(X, codes) since H H = I."""
+    d, m, n = 4, 5, 32
+    A, b = config_like_A(d, RNG), RNG.normal(0, 1e-3, d)
+    Z = RNG.integers(0, 4, (m, n)).astype(np.uint8)
+    X = RNG.normal(size=(2, n))
+    np.testing.assert_allclose(oracle.gemm_packed2b_hadamard(oracle.hadamard_rotate(X, n), oracle.pack2b(Z), A, b, d, n),
+                               oracle.gemm_packed2b(X, oracle.pack2b(Z), A, b, d, n), rtol=1e-12, atol=1e-14)
