@@ -282,8 +282,70 @@ def time_gemv_70b(torch, lcq, wl, seed, device, pk):
         nbytes = mx0.m * mx0.n / 4 + 2 * B * mx0.n + 2 * B * mx0.m
         out[f"B{B}"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
                         "bytes": nbytes, "eager_us_l2_flushed": statistics.median(eager) * 1e6}
+    # the paper's deployment path: online Hadamard rotation of the activations, then the product (1 token)
+    X = wl.torch_X(torch, wl.llama3_70b_gate_decode(1)[0], seed + 2000, 1, device)
+    Y = torch.empty((1, mx0.m), dtype=torch.bfloat16, device=device)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, 1, mx0.m, mx0.n, mx0.d, device)
+    for c in range(ncopies):
+        lcq.lcq_gemm_packed2b_hadamard(X, packs[c], mx0.n, mx0.d, A, b, Y, ws)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for i in range(calls):
+            lcq.lcq_gemm_packed2b_hadamard(X, packs[i % ncopies], mx0.n, mx0.d, A, b, Y, ws)
+    graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(replays):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    t = e0.elapsed_time(e1) * 1e-3 / (replays * calls)
+    nbytes = mx0.m * mx0.n / 4 + 2 * mx0.n + 2 * mx0.m
+    out["B1_hadamard"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
+                          "bytes": nbytes}
+    assert lcq.lcq_device_status(ws) == 0
+    del graph
     out["workload"] = ("llama3-70b gate 28672x8192 packed 2-bit, d=8, bf16 activations; CUDA-graph replay of 24 "
-                       "calls over 6 code copies (352 MB > L2)")
+                       "calls over 6 code copies (352 MB > L2); B1_hadamard adds the online rotation")
+    return out
+
+
+def time_training_sets(torch, lcq, wl, seed, device, pk):
+    """fwd+bwd of the other training workloads: Llama-2-7B projections (4096 tokens, 1% outlier channels)
+    at d = 4 and d = 8, and the single 512x512 oracle-sized layer (64 tokens, latency)."""
+    out = {}
+    sets = [("llama2_7b_projections_d4", wl.llama2_7b_projections(4), 5),
+            ("llama2_7b_projections_d8", wl.llama2_7b_projections(8), 5),
+            ("tiny_layer_512x512_64tok", wl.tiny_layer(), 200)]
+    for name, mats, iters in sets:
+        layer = [Linear(torch, lcq, wl, mx, seed + 3000, i, device) for i, mx in enumerate(mats)]
+        for L in layer:
+            lcq.lcq_encode(L.W, L.A, L.b, L.d, L.ws_e, latent=L.P)
+
+        def run():
+            for L in layer:
+                lcq.lcq_linear_fwd(L.X, L.P, L.d, L.A, L.b, L.Y, L.ws_f, packed_saved=L.saved)
+                lcq.lcq_linear_bwd(L.X, L.dY, L.saved, L.m, L.n, L.d, L.A, L.b, L.dP, L.dA, L.db, L.ws_b, dX=L.dX)
+
+        for _ in range(3):
+            run()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(iters):
+            run()
+        e1.record()
+        torch.cuda.synchronize()
+        t = e0.elapsed_time(e1) * 1e-3 / iters
+        fl = sum(L.flops() for L in layer)
+        for L in layer:
+            assert L.statuses(lcq)[1:3] == [0, 0]
+        out[name] = {"ms_per_fwd_bwd": t * 1e3, "TFLOP/s": fl / t / 1e12, "frac_bf16_peak": fl / t / 1e12 / pk["bf16"],
+                     "tokens": mats[0].N, "linears": len(mats)}
+        del layer
+        torch.cuda.empty_cache()
     return out
 
 
@@ -424,6 +486,7 @@ def main():
         torch.cuda.empty_cache()
         line["encode"] = time_encode_70b(torch, lcq, wl, args.seed, device, pk)
         line["packed_decode"] = time_gemv_70b(torch, lcq, wl, args.seed, device, pk)
+        line["other_training_workloads"] = time_training_sets(torch, lcq, wl, args.seed, device, pk)
         torch.cuda.empty_cache()
         layer = None
 

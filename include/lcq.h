@@ -59,7 +59,8 @@ typedef enum lcq_op {
     LCQ_OP_ENCODE = 1,
     LCQ_OP_LINEAR_FWD = 2,
     LCQ_OP_LINEAR_BWD = 3,
-    LCQ_OP_GEMM_PACKED2B = 4
+    LCQ_OP_GEMM_PACKED2B = 4,
+    LCQ_OP_GEMM_PACKED2B_HADAMARD = 5
 } lcq_op;
 
 /* Gradient estimators for dP through the rounding (Sec. 3.3). */
@@ -200,6 +201,26 @@ lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed
 lcq_status lcq_gemm_packed2b_noalloc(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
                                      int d, const float *A, const float *b, uint16_t *Y,
                                      int32_t *device_status, void *stream);
+
+/*
+ * lcq_hadamard - incoherence rotation of Sec. 2.2 (Hadamard transform following QuIP#), read as a
+ * normalized block-diagonal Walsh-Hadamard matrix H whose block is the largest power of two dividing
+ * n (at most 32768): out[r] = in[r] H for each of `rows` rows of length n (fp32, device; in may equal
+ * out). H is symmetric and orthogonal, so rotating twice restores the input. Used to rotate weights
+ * before lcq_encode when the deployment product rotates the activations (lcq_gemm_packed2b_hadamard).
+ */
+lcq_status lcq_hadamard(const float *in, int64_t rows, int64_t n, float *out, void *stream);
+
+/*
+ * lcq_gemm_packed2b_hadamard - deployment product with online rotation of the activations
+ * (App. Inference Speed: Hadamard transform, then the fused affine-dequant product):
+ *   Y = (X H) W_hat^T, with the codes encoding the rotated weights W H (see lcq_hadamard).
+ * Arguments as lcq_gemm_packed2b; needs lcq_workspace_size(LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d).
+ * The rotated activations are kept in fp32.
+ */
+lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
+                                      int d, const float *A, const float *b, uint16_t *Y,
+                                      void *ws, size_t ws_bytes, void *stream);
 
 /*
  * lcq_init_codebook - codebook initialisation of Sec. 2.2 Eq. init_ab for b = 2:

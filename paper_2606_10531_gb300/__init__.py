@@ -18,14 +18,14 @@ LCQ_OK = 0
 STATUS_NAMES = {0: "LCQ_OK", 1: "LCQ_ERR_NULL", 2: "LCQ_ERR_SHAPE", 3: "LCQ_ERR_ALIGN", 4: "LCQ_ERR_UNSUPPORTED",
                 5: "LCQ_ERR_WORKSPACE", 6: "LCQ_ERR_CUDA", 7: "LCQ_ERR_SINGULAR", 8: "LCQ_ERR_TIMEOUT",
                 9: "LCQ_ERR_ARG", 10: "LCQ_ERR_LIMIT"}
-LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B = 1, 2, 3, 4
+LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B, LCQ_OP_GEMM_PACKED2B_HADAMARD = 1, 2, 3, 4, 5
 LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
            "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout",
-           "lcq_init_codebook", "lcq_init_latent")
+           "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -67,6 +67,9 @@ _SIG = {
     "lcq_last_cuda_error": (ctypes.c_char_p, []),
     "lcq_selftest_wait_timeout": (ctypes.c_int, [_P, _P]),
     "lcq_init_codebook": (ctypes.c_int, [_P, ctypes.c_int, _P, _P, _P]),
+    "lcq_hadamard": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
+    "lcq_gemm_packed2b_hadamard": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P,
+                                                  ctypes.c_size_t, _P]),
     "lcq_init_latent": (ctypes.c_int, [_P, _I64, _I64, _P, ctypes.POINTER(ctypes.c_float),
                                        ctypes.POINTER(ctypes.c_float), _P]),
     "lcq_launch_count": (ctypes.c_uint64, []),
@@ -198,6 +201,18 @@ def lcq_device_status(ws, clear: bool = False, stream=None) -> int:
 def lcq_selftest_wait_timeout(ws, stream=None):
     """Run the bounded-wait self-test kernel (about 2 s); the workspace status then reads LCQ_ERR_TIMEOUT."""
     _check(lib().lcq_selftest_wait_timeout(_ptr(ws), _stream(stream)), "lcq_selftest_wait_timeout")
+
+
+def lcq_hadamard(inp, out, stream=None):
+    rows, n = inp.shape
+    _check(lib().lcq_hadamard(_ptr(inp), rows, n, _ptr(out), _stream(stream)), "lcq_hadamard")
+
+
+def lcq_gemm_packed2b_hadamard(X, packed, n: int, d: int, A, b, Y, ws, stream=None):
+    N = X.shape[0]
+    m = packed.shape[0]
+    _check(lib().lcq_gemm_packed2b_hadamard(_ptr(X), N, _ptr(packed), m, n, d, _ptr(A), _ptr(b), _ptr(Y), _ptr(ws),
+                                            ws.numel(), _stream(stream)), "lcq_gemm_packed2b_hadamard")
 
 
 def lcq_init_codebook(G, d: int, A, b, stream=None):

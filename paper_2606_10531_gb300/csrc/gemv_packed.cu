@@ -44,9 +44,10 @@ __host__ __device__ inline int64_t gemv_nprep(int64_t n) { return (gemv_npad(n) 
 // Field position (power-of-4 scale) of fragment register k.
 __device__ __forceinline__ int frag_shift(int k) { return (k % 3 == 2) ? 2 : ((k % 3 == 1) ? 1 : 0); }
 
-template <int D>
+// X is bf16 [N][n] (uint16 bit patterns) or, with F32IN, fp32 [N][n] (rotated activations).
+template <int D, bool F32IN>
 __global__ void __launch_bounds__(256)
-gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const float *__restrict__ A,
+gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const float *__restrict__ A,
                  const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ corrpart) {
     __shared__ float red[2][8];
     // let the dependent main kernel start streaming codes right away (it waits for our results itself)
@@ -57,7 +58,11 @@ gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const 
     for (int i = 0; i < D * D; ++i) Am[i] = __ldg(A + i);
 #pragma unroll
     for (int i = 0; i < D; ++i) bv[i] = __ldg(b + i);
-    const uint16_t *xrow = X + t * n;
+    const uint16_t *xrow = static_cast<const uint16_t *>(Xv) + t * n;
+    const float *frow = static_cast<const float *>(Xv) + t * n;
+    auto xval = [&](int64_t c) -> float {
+        return F32IN ? frow[c] : __uint_as_float(static_cast<uint32_t>(xrow[c]) << 16);
+    };
     uint32_t *out = reinterpret_cast<uint32_t *>(Xp + t * npad);
     float S = 0.0f, r = 0.0f;
     const int64_t blk = static_cast<int64_t>(blockIdx.y) * 256 + threadIdx.x;
@@ -66,13 +71,22 @@ gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const 
         const int64_t c0 = blk * 16;
         if (c0 + 16 <= n) {
             float x[16];
-            const uint4 *src = reinterpret_cast<const uint4 *>(xrow + c0);
-            const uint4 u0 = __ldg(src), u1 = __ldg(src + 1);
-            const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+            if (F32IN) {
+                const float4 *src = reinterpret_cast<const float4 *>(frow + c0);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                x[2 * i] = __uint_as_float(w[i] << 16);
-                x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+                for (int q = 0; q < 4; ++q) {
+                    const float4 f = __ldg(src + q);
+                    x[4 * q] = f.x; x[4 * q + 1] = f.y; x[4 * q + 2] = f.z; x[4 * q + 3] = f.w;
+                }
+            } else {
+                const uint4 *src = reinterpret_cast<const uint4 *>(xrow + c0);
+                const uint4 u0 = __ldg(src), u1 = __ldg(src + 1);
+                const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    x[2 * i] = __uint_as_float(w[i] << 16);
+                    x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+                }
             }
 #pragma unroll
             for (int g = 0; g < 16 / D; ++g) {
@@ -92,14 +106,10 @@ gemv_prep_kernel(const uint16_t *__restrict__ X, int64_t n, int64_t npad, const 
             for (int64_t g0 = c0; g0 < n; g0 += D) {
                 for (int k = 0; k < D; ++k) {
                     float acc = 0.0f;
-                    for (int j = 0; j < D; ++j) {
-                        const float xv = __uint_as_float(static_cast<uint32_t>(xrow[g0 + j]) << 16);
-                        acc = fmaf(xv, Am[j * D + k], acc);
-                    }
+                    for (int j = 0; j < D; ++j) acc = fmaf(xval(g0 + j), Am[j * D + k], acc);
                     xp[g0 - c0 + k] = acc;
                 }
-                for (int j = 0; j < D; ++j)
-                    r = fmaf(__uint_as_float(static_cast<uint32_t>(xrow[g0 + j]) << 16), bv[j], r);
+                for (int j = 0; j < D; ++j) r = fmaf(xval(g0 + j), bv[j], r);
             }
         }
         uint32_t words[8];
@@ -447,6 +457,63 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
 
 // ------------------------------------------------------------------ host side
 
+// ------------------------------------------------------------------ block Walsh-Hadamard rotation
+//
+// out[r, blk*B + j] = (1/sqrt(B)) sum_i in[r, blk*B + i] * H_B[i][j] (Sylvester H, symmetric):
+// one CTA per (row, block) transforms the block in shared memory (log2 B butterfly stages).
+// in may equal out (each block is read whole before it is written).
+
+template <typename InT>
+__global__ void __launch_bounds__(1024)
+hadamard_kernel(const InT *__restrict__ in, int64_t n, int bsz, float *out) {
+    extern __shared__ float hbuf[];
+    const int64_t row = blockIdx.x;
+    const int64_t base = row * n + static_cast<int64_t>(blockIdx.y) * bsz;
+    for (int i = threadIdx.x; i < bsz; i += blockDim.x) {
+        if constexpr (sizeof(InT) == 2)
+            hbuf[i] = __uint_as_float(static_cast<uint32_t>(in[base + i]) << 16);
+        else
+            hbuf[i] = in[base + i];
+    }
+    __syncthreads();
+    for (int h = 1; h < bsz; h <<= 1) {
+        for (int p = threadIdx.x; p < bsz / 2; p += blockDim.x) {
+            const int i = (p / h) * 2 * h + (p % h);
+            const float u = hbuf[i], v = hbuf[i + h];
+            hbuf[i] = u + v;
+            hbuf[i + h] = u - v;
+        }
+        __syncthreads();
+    }
+    const float scale = rsqrtf(static_cast<float>(bsz));
+    for (int i = threadIdx.x; i < bsz; i += blockDim.x) out[base + i] = hbuf[i] * scale;
+}
+
+int hadamard_block_size(int64_t n) {
+    int bsz = 1;
+    while (n % (2 * bsz) == 0 && 2 * bsz <= 32768) bsz *= 2;
+    return bsz;
+}
+
+cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t n, float *out, cudaStream_t st) {
+    const int bsz = hadamard_block_size(n);
+    const int threads = bsz / 2 < 1024 ? (bsz / 2 < 32 ? 32 : bsz / 2) : 1024;
+    const size_t smem = static_cast<size_t>(bsz) * 4;
+    dim3 grid(static_cast<unsigned>(rows), static_cast<unsigned>(n / bsz));
+    cudaError_t e;
+    if (in_bf16) {
+        e = ensure_dynamic_smem(reinterpret_cast<const void *>(hadamard_kernel<uint16_t>), static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        hadamard_kernel<uint16_t><<<grid, threads, smem, st>>>(static_cast<const uint16_t *>(in), n, bsz, out);
+    } else {
+        e = ensure_dynamic_smem(reinterpret_cast<const void *>(hadamard_kernel<float>), static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        hadamard_kernel<float><<<grid, threads, smem, st>>>(static_cast<const float *>(in), n, bsz, out);
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
 size_t packed_gemv_workspace(int64_t N, int64_t n) {
     const size_t xp = static_cast<size_t>(N) * static_cast<size_t>(gemv_npad(n)) * 2;
     const size_t cr = static_cast<size_t>(N) * static_cast<size_t>(gemv_nprep(n)) * 4;
@@ -509,8 +576,13 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
     const int64_t npad = gemv_npad(a.n), nprep = gemv_nprep(a.n);
     trace_begin(LCQ_K_GEMV, st);
     dim3 pgrid(static_cast<unsigned>(a.N), static_cast<unsigned>(nprep));
-    if (d == 4) gemv_prep_kernel<4><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
-    else gemv_prep_kernel<8><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
+    if (a.Xf) {
+        if (d == 4) gemv_prep_kernel<4, true><<<pgrid, 256, 0, st>>>(a.Xf, a.n, npad, a.A, a.b, a.Xp, a.corr);
+        else gemv_prep_kernel<8, true><<<pgrid, 256, 0, st>>>(a.Xf, a.n, npad, a.A, a.b, a.Xp, a.corr);
+    } else {
+        if (d == 4) gemv_prep_kernel<4, false><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
+        else gemv_prep_kernel<8, false><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
+    }
     count_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;

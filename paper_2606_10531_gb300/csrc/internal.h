@@ -100,6 +100,7 @@ cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cud
 // ---------------------------------------------------------------- packed 2-bit GEMV / small GEMM
 struct PackedGemvArgs {
     const uint16_t *X;       // [N][n] bf16
+    const float *Xf;         // [N][n] fp32 activations used instead of X when not NULL
     int64_t N, m, n;
     const uint8_t *packed;   // [m][n/4]
     const float *A, *b;
@@ -111,5 +112,8 @@ struct PackedGemvArgs {
 size_t packed_gemv_workspace(int64_t N, int64_t n);
 size_t packed_gemv_corr_offset(int64_t N, int64_t n);
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);
+// Row-wise normalized block Walsh-Hadamard rotation (block = largest power of two dividing n, <= 32768).
+int hadamard_block_size(int64_t n);
+cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t n, float *out, cudaStream_t st);
 
 }  // namespace lcq

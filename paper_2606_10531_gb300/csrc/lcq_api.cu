@@ -176,6 +176,8 @@ size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d) {
             return kHeader + align256(mn * 2) + align256(sizeof(float) * kMaxGemmCtas * (d * d + d));
         case LCQ_OP_GEMM_PACKED2B:
             return kHeader + packed_gemv_workspace(N, n);
+        case LCQ_OP_GEMM_PACKED2B_HADAMARD:
+            return kHeader + align256(static_cast<size_t>(N) * static_cast<size_t>(n) * 4) + packed_gemv_workspace(N, n);
         default:
             return 0;
     }
@@ -246,6 +248,42 @@ lcq_status lcq_device_status(const void *ws, void *stream, int32_t *status_out, 
         if (cudaStreamSynchronize(st) != cudaSuccess) return LCQ_ERR_CUDA;
     }
     return LCQ_OK;
+}
+
+lcq_status lcq_hadamard(const float *in, int64_t rows, int64_t n, float *out, void *stream) {
+    if (rows < 0 || n < 0 || n % 8 != 0) return LCQ_ERR_SHAPE;
+    if (rows * n == 0) return LCQ_OK;
+    LCQ_TRY(check_tensor(in, rows * n));
+    LCQ_TRY(check_tensor(out, rows * n));
+    return cuda_status(launch_hadamard(in, false, rows, n, out, as_stream(stream)));
+}
+
+lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
+                                      int d, const float *A, const float *b, uint16_t *Y, void *ws, size_t ws_bytes,
+                                      void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    LCQ_TRY(check_tensor(X, N * n));
+    LCQ_TRY(check_tensor(packed, m * n));
+    LCQ_TRY(check_tensor(Y, N * m));
+    if (!A || !b) return LCQ_ERR_NULL;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    if (N * m == 0) return LCQ_OK;
+    if (n == 0) return cuda_status(cudaMemsetAsync(Y, 0, sizeof(uint16_t) * N * m, st));
+    Header *h = static_cast<Header *>(ws);
+    float *Xr = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kHeader);
+    uint8_t *base = static_cast<uint8_t *>(ws) + kHeader + align256(static_cast<size_t>(N) * static_cast<size_t>(n) * 4);
+    trace_begin(LCQ_K_GEMV, st);
+    const cudaError_t e = launch_hadamard(X, true, N, n, Xr, st);
+    trace_end(LCQ_K_GEMV, st);
+    LCQ_TRY(cuda_status(e));
+    PackedGemvArgs a;
+    a.X = X; a.Xf = Xr; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
+    a.Xp = reinterpret_cast<uint16_t *>(base);
+    a.corr = reinterpret_cast<float *>(base + packed_gemv_corr_offset(N, n));
+    a.status = &h->status;
+    return cuda_status(launch_packed_gemv(a, d, num_sms_current(), st));
 }
 
 lcq_status lcq_init_codebook(const float *G, int d, float *A, float *b, void *stream) {
@@ -452,7 +490,7 @@ lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed
     Header *h = static_cast<Header *>(ws);
     uint8_t *base = static_cast<uint8_t *>(ws) + kHeader;
     PackedGemvArgs a;
-    a.X = X; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
+    a.X = X; a.Xf = nullptr; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
     a.Xp = reinterpret_cast<uint16_t *>(base);
     a.corr = reinterpret_cast<float *>(base + packed_gemv_corr_offset(N, n));
     a.status = &h->status;

@@ -313,3 +313,30 @@ def test_init_latent_matches_oracle_and_requantizes_to_the_same_codes(m, n):
         ws = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d)
         lcq.lcq_linear_fwd(X, P, d, A, bz, Y, ws, packed_saved=saved, latent_scale=s, latent_offset=t)
         assert np.array_equal(saved.cpu().numpy(), oracle.pack2b(Z))
+
+
+# ----------------------------------------------------------------------------- Hadamard rotation
+
+@pytest.mark.parametrize("rows,n", [(3, 8), (5, 96), (2, 8192), (4, 14336)])
+def test_hadamard_rotation_matches_oracle(rows, n):
+    torch = T()
+    X = np.random.default_rng(rows + n).normal(size=(rows, n)).astype(np.float32)
+    out = torch.empty((rows, n), dtype=torch.float32, device="cuda")
+    lcq.lcq_hadamard(dev(X), out)
+    np.testing.assert_allclose(out.cpu().numpy(), oracle.hadamard_rotate(X, n), rtol=1e-4, atol=1e-5)
+    lcq.lcq_hadamard(out, out)                    # in place, and H H = I
+    np.testing.assert_allclose(out.cpu().numpy(), X, rtol=1e-4, atol=1e-5)
+
+
+@pytest.mark.parametrize("N", [1, 16])
+@pytest.mark.parametrize("m,n,d", [(200, 512, 8), (70, 200, 4), (300, 8192, 8)])
+def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
+    rng = np.random.default_rng(N * 7 + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    Xb = wl.bf16_bits(rng.normal(0, 1, (N, n)).astype(np.float32))
+    ref = oracle.gemm_packed2b_hadamard(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)
+    lcq.lcq_gemm_packed2b_hadamard(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert max_rel(host_bf16(Y), ref) <= TOL_BF16
