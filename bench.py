@@ -49,7 +49,8 @@ def parse():
     ap.add_argument("--case", choices=["linear", "encode", "gemv"], default=None,
                     help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
                          "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
-                         "28672 x 8192, gemv = 70B gate at 16 tokens")
+                         "28672 x 8192, gemv = 70B gate at --tokens tokens")
+    ap.add_argument("--tokens", type=int, default=None, help="tokens of the gemv profiling case (default 16)")
     return ap.parse_args()
 
 
@@ -226,7 +227,7 @@ def time_encode_70b(torch, lcq, wl, seed, device, pk):
 
 
 def time_gemv_70b(torch, lcq, wl, seed, device, pk):
-    """Packed 2-bit product of the Llama-3-70B gate projection (28672 x 8192, d = 8) at 1/4/16 tokens.
+    """Packed 2-bit product of the Llama-3-70B gate projection (28672 x 8192, d = 8) at 1/2/4/16 tokens.
 
     Decode-style measurement (the paper times decoding under CUDA Graphs): 24 back-to-back calls are
     captured in one CUDA graph, rotating over 6 copies of the packed codes (352 MB > L2) so every call
@@ -239,7 +240,7 @@ def time_gemv_70b(torch, lcq, wl, seed, device, pk):
     b = wl.torch_b(torch, mx0, seed + 2000, 0, device).contiguous()
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=device)
     out = {}
-    for B in (1, 4, 16):
+    for B in (1, 2, 4, 16):
         X = wl.torch_X(torch, wl.llama3_70b_gate_decode(B)[0], seed + 2000, B, device)
         Y = torch.empty((B, mx0.m), dtype=torch.bfloat16, device=device)
         ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, B, mx0.m, mx0.n, mx0.d, device)
@@ -578,7 +579,7 @@ def profile_case(args):
             lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
         wss = [ws]
     else:
-        mx = wl.llama3_70b_gate_decode(GEMV_TOKENS)[0]
+        mx = wl.llama3_70b_gate_decode(args.tokens or GEMV_TOKENS)[0]
         packed = wl.torch_packed_codes(torch, mx, args.seed, 0, device)
         A, b = wl.torch_A(torch, mx, args.seed, 0, device), wl.torch_b(torch, mx, args.seed, 0, device)
         X = wl.torch_X(torch, mx, args.seed, 0, device)

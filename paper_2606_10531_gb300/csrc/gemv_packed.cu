@@ -44,12 +44,89 @@ __host__ __device__ inline int64_t gemv_nprep(int64_t n) { return (gemv_npad(n) 
 // Field position (power-of-4 scale) of fragment register k.
 __device__ __forceinline__ int frag_shift(int k) { return (k % 3 == 2) ? 2 : ((k % 3 == 1) ? 1 : 0); }
 
-// X is bf16 [N][n] (uint16 bit patterns) or, with F32IN, fp32 [N][n] (rotated activations).
+// The 16 activations of the block starting at column c0 of token row t (zero past n; n % 8 == 0).
+// X is bf16 [N][n] (uint16 bit patterns) or, with f32in, fp32 [N][n] (rotated activations).
+__device__ __forceinline__ void load_block(const void *__restrict__ Xv, bool f32in, int64_t n, int64_t t, int64_t c0,
+                                           float (&x)[16]) {
+    if (c0 + 16 <= n) {
+        if (f32in) {
+            const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(Xv) + t * n + c0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float4 f = __ldg(src + q);
+                x[4 * q] = f.x; x[4 * q + 1] = f.y; x[4 * q + 2] = f.z; x[4 * q + 3] = f.w;
+            }
+        } else {
+            const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(Xv) + t * n + c0);
+            const uint4 u0 = __ldg(src), u1 = __ldg(src + 1);
+            const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                x[2 * i] = __uint_as_float(w[i] << 16);
+                x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+            }
+        }
+    } else {
+        // ragged end, 8 columns at a time
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const bool in = c0 + 8 * h < n;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int64_t c = c0 + 8 * h + i;
+                x[8 * h + i] = !in ? 0.0f
+                               : f32in ? static_cast<const float *>(Xv)[t * n + c]
+                                       : __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t *>(Xv)[t * n + c]) << 16);
+            }
+        }
+    }
+}
+
+// X' = X_g A of one 16-column block (groups of D columns), and the block's share r of sum_g X_g . b.
+template <int D>
+__device__ __forceinline__ void xform_block(const float (&x)[16], const float (&Am)[D * D], const float (&bv)[D],
+                                            float (&xp)[16], float &r) {
+#pragma unroll
+    for (int g = 0; g < 16 / D; ++g) {
+#pragma unroll
+        for (int k = 0; k < D; ++k) {
+            float acc = 0.0f;
+#pragma unroll
+            for (int j = 0; j < D; ++j) acc = fmaf(x[g * D + j], Am[j * D + k], acc);
+            xp[g * D + k] = acc;
+        }
+#pragma unroll
+        for (int j = 0; j < D; ++j) r = fmaf(x[g * D + j], bv[j], r);
+    }
+}
+
+template <int D, bool F32IN>
+__device__ __forceinline__ void prep_block(const void *__restrict__ Xv, int64_t n, int64_t t, int64_t c0,
+                                           const float (&Am)[D * D], const float (&bv)[D], float (&xp)[16],
+                                           float &r) {
+    float x[16];
+    load_block(Xv, F32IN, n, t, c0, x);
+    xform_block<D>(x, Am, bv, xp, r);
+}
+
+// Per-CTA sum of v over the 256 threads, written by thread 0 (fixed order).
+__device__ __forceinline__ void block_sum_256(float v, float *out) {
+    __shared__ float red[8];
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float s = 0.0f;
+        for (int w = 0; w < 8; ++w) s += red[w];
+        *out = s;
+    }
+}
+
 template <int D, bool F32IN>
 __global__ void __launch_bounds__(256)
 gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const float *__restrict__ A,
                  const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ corrpart) {
-    __shared__ float red[2][8];
     // let the dependent main kernel start streaming codes right away (it waits for our results itself)
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t t = blockIdx.x;
@@ -58,60 +135,12 @@ gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const flo
     for (int i = 0; i < D * D; ++i) Am[i] = __ldg(A + i);
 #pragma unroll
     for (int i = 0; i < D; ++i) bv[i] = __ldg(b + i);
-    const uint16_t *xrow = static_cast<const uint16_t *>(Xv) + t * n;
-    const float *frow = static_cast<const float *>(Xv) + t * n;
-    auto xval = [&](int64_t c) -> float {
-        return F32IN ? frow[c] : __uint_as_float(static_cast<uint32_t>(xrow[c]) << 16);
-    };
     uint32_t *out = reinterpret_cast<uint32_t *>(Xp + t * npad);
     float S = 0.0f, r = 0.0f;
     const int64_t blk = static_cast<int64_t>(blockIdx.y) * 256 + threadIdx.x;
     if (blk < npad / 16) {
         float xp[16];
-        const int64_t c0 = blk * 16;
-        if (c0 + 16 <= n) {
-            float x[16];
-            if (F32IN) {
-                const float4 *src = reinterpret_cast<const float4 *>(frow + c0);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float4 f = __ldg(src + q);
-                    x[4 * q] = f.x; x[4 * q + 1] = f.y; x[4 * q + 2] = f.z; x[4 * q + 3] = f.w;
-                }
-            } else {
-                const uint4 *src = reinterpret_cast<const uint4 *>(xrow + c0);
-                const uint4 u0 = __ldg(src), u1 = __ldg(src + 1);
-                const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    x[2 * i] = __uint_as_float(w[i] << 16);
-                    x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-                }
-            }
-#pragma unroll
-            for (int g = 0; g < 16 / D; ++g) {
-#pragma unroll
-                for (int k = 0; k < D; ++k) {
-                    float acc = 0.0f;
-#pragma unroll
-                    for (int j = 0; j < D; ++j) acc = fmaf(x[g * D + j], Am[j * D + k], acc);
-                    xp[g * D + k] = acc;
-                }
-#pragma unroll
-                for (int j = 0; j < D; ++j) r = fmaf(x[g * D + j], bv[j], r);
-            }
-        } else {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) xp[i] = 0.0f;
-            for (int64_t g0 = c0; g0 < n; g0 += D) {
-                for (int k = 0; k < D; ++k) {
-                    float acc = 0.0f;
-                    for (int j = 0; j < D; ++j) acc = fmaf(xval(g0 + j), Am[j * D + k], acc);
-                    xp[g0 - c0 + k] = acc;
-                }
-                for (int j = 0; j < D; ++j) r = fmaf(xval(g0 + j), bv[j], r);
-            }
-        }
+        prep_block<D, F32IN>(Xv, n, t, blk * 16, Am, bv, xp, r);
         uint32_t words[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
@@ -126,18 +155,7 @@ gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const flo
         dst[0] = make_uint4(words[0], words[1], words[2], words[3]);
         dst[1] = make_uint4(words[4], words[5], words[6], words[7]);
     }
-    for (int o = 16; o; o >>= 1) {
-        S += __shfl_xor_sync(0xffffffffu, S, o);
-        r += __shfl_xor_sync(0xffffffffu, r, o);
-    }
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) { red[0][warp] = S; red[1][warp] = r; }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        float s2 = 0.0f, r2 = 0.0f;
-        for (int w = 0; w < 8; ++w) { s2 += red[0][w]; r2 += red[1][w]; }
-        corrpart[t * gridDim.y + blockIdx.y] = r2 - 128.0f * s2;
-    }
+    block_sum_256(r - 128.0f * S, corrpart + t * gridDim.y + blockIdx.y);
 }
 
 // corr[t] = sum of the prep CTAs' partials, in a fixed order.
@@ -455,6 +473,268 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
     }
 }
 
+// ------------------------------------------------------------------ integer (dp2a) variant, one token
+//
+// With one token a tensor-core MMA spends most of its width on padding, and the fragment conversion
+// costs more than the product. This variant works on the CUDA cores instead: a code word of 16
+// columns is split into four byte-spread words with one shift and four ANDs,
+//   s0 = w & 0x03030303 (columns 0,4,8,12)       s1 = w & 0x0C0C0C0C (columns 1,5,9,13, times 4)
+//   s2 = (w >> 4) & 0x03030303 (columns 2,6,...)  s3 = (w >> 4) & 0x0C0C0C0C (columns 3,7,..., times 4)
+// and each dp2a multiplies two of those bytes with two int16 activations (exact int32 sums).
+//
+// Activations: the consumer warps compute X' = X_g A themselves (no separate prep kernel) and store
+// it in shared memory as int16 with one scale for the token, s = max|X| * max_k sum_j |A[j][k]| /
+// 32767, a bound on max|X'| known before X' is formed. Column c of a 16-column block holds
+// round(X'[c] / s) for c % 4 in {0, 2} and round(X'[c] / (4 s)) for c % 4 in {1, 3} (those codes
+// arrive multiplied by 4). The eight 32-bit words of a block hold the column pairs (0,4) (8,12)
+// (1,5) (9,13) (2,6) (10,14) (3,7) (11,15), the pairs one dp2a multiplies with bytes (0,1) or (2,3)
+// of a spread code word; a 512-column tile stores the first halves of its 32 blocks, then the second
+// halves (conflict-free 16-byte reads).
+//
+// Codes: one producer thread streams (R rows x 512 columns) tiles through a TMA ring (128-byte
+// swizzle). Lane l owns code word l (16 columns) of rows warp + CW j (CW consumer warps), so a warp
+// reads one whole 128-byte row per load, and the lane's position in a swizzled row is the same for
+// all its rows (CW is a multiple of 8). The int32 sums run over the whole unit and are added over the
+// 32 lanes of a row with exact integer warp reductions (two accumulators, each over half the row's
+// columns: below 2^31 for n <= 32768), then scaled once.
+//
+// Launched with programmatic dependent launch: the code stream starts while the previous kernel in
+// the stream finishes; the consumers wait for it (griddepcontrol.wait) before reading X.
+
+constexpr int kDpMaxTokens = 1;            // two tokens measured slower than the tensor-core kernel
+constexpr int kDpWarps = 16;               // consumer warps (a multiple of 8)
+constexpr int64_t kDpMaxN = 32768;         // integer row sums stay below 2^31
+constexpr size_t kDpSmemLimit = 227 * 1024;
+
+struct GemvDpParams {
+    const void *X;            // [n] bf16 bit patterns, or fp32 when f32in
+    const float *A, *b;
+    int64_t m, n;
+    int d, f32in;
+    int R, units, nkc, stages;
+    uint16_t *Y;              // [m]
+    int32_t *status;
+};
+
+// Shared-memory layout of the dp kernel (offsets from the 1024-byte aligned base).
+struct DpSmemLayout {
+    size_t xq, red, ab, bars, total;
+};
+__host__ __device__ inline DpSmemLayout dp_smem_layout(int R, int stages, int nkc) {
+    DpSmemLayout L;
+    L.xq = static_cast<size_t>(stages) * static_cast<size_t>(R) * 128;
+    L.red = L.xq + static_cast<size_t>(nkc) * 1024;
+    L.ab = L.red + 2 * kDpWarps * 4;                                 // per-warp max|X| and sum X_g . b
+    L.bars = (L.ab + (64 + 8 + 1) * 4 + 15) / 16 * 16;               // A (d x d), b (d), max_k sum_j |A|
+    L.total = L.bars + 2 * kTmaStages * 8;
+    return L;
+}
+
+__device__ __forceinline__ int32_t dp2a_lo(uint32_t a, uint32_t b, int32_t c) {
+    int32_t d;
+    asm("dp2a.lo.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+__device__ __forceinline__ int32_t dp2a_hi(uint32_t a, uint32_t b, int32_t c) {
+    int32_t d;
+    asm("dp2a.hi.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+// acc0/acc1 += the 16 columns of code word w times one 16-column block (two uint4) of activations.
+__device__ __forceinline__ void dp_word(uint32_t w, const uint4 &xa, const uint4 &xb, int32_t &acc0, int32_t &acc1) {
+    const uint32_t w4 = w >> 4;
+    const uint32_t s0 = w & 0x03030303u, s1 = w & 0x0C0C0C0Cu, s2 = w4 & 0x03030303u, s3 = w4 & 0x0C0C0C0Cu;
+    acc0 = dp2a_lo(xa.x, s0, acc0);
+    acc1 = dp2a_hi(xa.y, s0, acc1);
+    acc0 = dp2a_lo(xa.z, s1, acc0);
+    acc1 = dp2a_hi(xa.w, s1, acc1);
+    acc0 = dp2a_lo(xb.x, s2, acc0);
+    acc1 = dp2a_hi(xb.y, s2, acc1);
+    acc0 = dp2a_lo(xb.z, s3, acc0);
+    acc1 = dp2a_hi(xb.w, s3, acc1);
+}
+
+// int16 activations of one 16-column block (lane l of tile `tile`): X' = X_g A, scaled by inv
+// (times 1/4 for columns c % 4 in {1, 3}), stored in the pair order of dp_word. Returns the block's
+// share of sum_g X_g . b added to r.
+template <int D>
+__device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *ab_s, uint8_t *xq_s, float inv, int tile,
+                                            int lane, float &r) {
+    const float(&Am)[D * D] = *reinterpret_cast<const float(*)[D * D]>(ab_s);
+    const float(&bv)[D] = *reinterpret_cast<const float(*)[D]>(ab_s + D * D);
+    float xp[16];
+    xform_block<D>(x, Am, bv, xp, r);
+    constexpr int kFirst[8] = {0, 8, 1, 9, 2, 10, 3, 11};
+    uint32_t words[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int cc = kFirst[k];
+        const float f = (cc & 1) ? 0.25f * inv : inv;
+        const int lo = max(-32767, min(32767, __float2int_rn(xp[cc] * f)));
+        const int hi = max(-32767, min(32767, __float2int_rn(xp[cc + 4] * f)));
+        words[k] = (static_cast<uint32_t>(lo) & 0xFFFFu) | (static_cast<uint32_t>(hi) << 16);
+    }
+    uint4 *dst = reinterpret_cast<uint4 *>(xq_s + static_cast<size_t>(tile) * 1024);
+    dst[lane] = make_uint4(words[0], words[1], words[2], words[3]);
+    dst[32 + lane] = make_uint4(words[4], words[5], words[6], words[7]);
+}
+
+__device__ __forceinline__ float absmax16(const float (&x)[16], float mx) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) mx = fmaxf(mx, fabsf(x[i]));
+    return mx;
+}
+
+// RPT: rows per thread per tile (a unit has R = kDpWarps * RPT rows).
+template <int RPT>
+__global__ void __launch_bounds__(32 * (kDpWarps + 1), 1)
+packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParams p) {
+    constexpr int CW = kDpWarps;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const DpSmemLayout L = dp_smem_layout(p.R, p.stages, p.nkc);
+    float *red_s = reinterpret_cast<float *>(base + L.red);   // [2][CW]: max|X|, then sum X_g . b
+    float *ab_s = reinterpret_cast<float *>(base + L.ab);
+    uint64_t *full = reinterpret_cast<uint64_t *>(base + L.bars);
+    uint64_t *empty = full + kTmaStages;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t stage_bytes = static_cast<uint32_t>(p.R) * 128u;
+    if (threadIdx.x == 0) {
+        prefetch_tensormap(&tmC);
+        for (int i = 0; i < p.stages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], CW);
+        }
+        fence_barrier_init();
+    }
+    __syncthreads();
+    // the next kernel in the stream may start launching; it waits for our completion before it
+    // reads anything we write
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- producer: code tiles -> ring
+        if (lane == 0) {
+            int st = 0;
+            uint32_t ph = 0;
+            for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
+                for (int kc = 0; kc < p.nkc; ++kc) {
+                    if (!mbar_wait(&empty[st], ph ^ 1, p.status)) return;
+                    mbar_arrive_expect_tx(&full[st], stage_bytes);
+                    tma_load_2d(base + static_cast<size_t>(st) * stage_bytes, &tmC, kc * 128, u * p.R, &full[st]);
+                    if (++st == p.stages) { st = 0; ph ^= 1; }
+                }
+            }
+        }
+        return;
+    }
+
+    // -------------------------------------------------------------------- consumers
+    const int cw = warp - 1, ct = threadIdx.x - 32;
+    const auto bar_consumers = [] { asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory"); };
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // X comes from the previous kernel
+    float scale, corr;
+    {
+        // pass 1: A, b to shared memory; max|X| per warp. Lane l of warp cw reads the 16-column block l
+        // of tiles cw, cw + CW, ...; the first block stays in registers for pass 2.
+        const int D = p.d;
+        if (ct < D * D + D) ab_s[ct] = ct < D * D ? __ldg(p.A + ct) : __ldg(p.b + (ct - D * D));
+        const bool f32in = p.f32in != 0;
+        float x0[16];
+        float mx = 0.0f;
+        if (cw < p.nkc) {
+            load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(cw) * 32 + lane) * 16, x0);
+            mx = absmax16(x0, mx);
+        }
+        for (int tile = cw + CW; tile < p.nkc; tile += CW) {
+            float x[16];
+            load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(tile) * 32 + lane) * 16, x);
+            mx = absmax16(x, mx);
+        }
+        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if (lane == 0) red_s[cw] = mx;
+        bar_consumers();
+        // pass 2: the token's scale s = max|X| * max_k sum_j |A[j][k]| / 32767 (a bound on max|X'|),
+        // then X' -> int16
+        float xmax = 0.0f, acol = 0.0f;
+        for (int w = 0; w < CW; ++w) xmax = fmaxf(xmax, red_s[w]);
+        for (int k = 0; k < D; ++k) {
+            float cs = 0.0f;
+            for (int j = 0; j < D; ++j) cs += fabsf(ab_s[j * D + k]);
+            acol = fmaxf(acol, cs);
+        }
+        const float bound = xmax * acol;
+        scale = bound / 32767.0f;
+        const float inv = bound > 0.0f ? 32767.0f / bound : 0.0f;
+        uint8_t *xq_s = base + L.xq;
+        float r = 0.0f;
+        if (cw < p.nkc) {
+            if (D == 8) dp_quantize<8>(x0, ab_s, xq_s, inv, cw, lane, r);
+            else dp_quantize<4>(x0, ab_s, xq_s, inv, cw, lane, r);
+        }
+        for (int tile = cw + CW; tile < p.nkc; tile += CW) {
+            float x[16];
+            load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(tile) * 32 + lane) * 16, x);
+            if (D == 8) dp_quantize<8>(x, ab_s, xq_s, inv, tile, lane, r);
+            else dp_quantize<4>(x, ab_s, xq_s, inv, tile, lane, r);
+        }
+        for (int o = 16; o; o >>= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+        if (lane == 0) red_s[CW + cw] = r;
+        bar_consumers();
+        corr = 0.0f;
+        for (int w = 0; w < CW; ++w) corr += red_s[CW + w];
+    }
+
+    // this lane's word in any of its rows: 16-byte chunk (lane / 4) ^ (row % 8), row % 8 = warp % 8
+    const int lane_word = (((lane >> 2) ^ (cw & 7)) << 2) + (lane & 3);
+    const uint32_t *ring_w = reinterpret_cast<const uint32_t *>(base) + cw * 32 + lane_word;
+    const uint4 *xq_v = reinterpret_cast<const uint4 *>(base + L.xq) + lane;
+    int st = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
+        int32_t acc[RPT][2];
+#pragma unroll
+        for (int j = 0; j < RPT; ++j) acc[j][0] = acc[j][1] = 0;
+
+        for (int kc = 0; kc < p.nkc; ++kc) {
+            // this lane's 16 activation columns of tile kc (fetched before waiting for the code tile)
+            const uint4 xa = xq_v[kc * 64], xb = xq_v[kc * 64 + 32];
+            if (!mbar_wait(&full[st], ph, p.status)) { ok = false; break; }
+            const uint32_t *tile = ring_w + static_cast<size_t>(st) * (RPT * CW * 32);
+            uint32_t w[RPT];
+#pragma unroll
+            for (int j = 0; j < RPT; ++j) w[j] = tile[j * CW * 32];
+#pragma unroll
+            for (int j = 0; j < RPT; ++j) dp_word(w[j], xa, xb, acc[j][0], acc[j][1]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[st]);
+            if (++st == p.stages) { st = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        // sum the 32 lanes of each row (exact integer warp reductions: each accumulator covers half the
+        // row's columns, below 2^31 for n <= 32768), scale, + corr, bf16 store
+        const int64_t row0 = static_cast<int64_t>(u) * p.R + cw;
+#pragma unroll
+        for (int j = 0; j < RPT; ++j) {
+            const int32_t s0 = __reduce_add_sync(0xffffffffu, acc[j][0]);
+            const int32_t s1 = __reduce_add_sync(0xffffffffu, acc[j][1]);
+            const int64_t row = row0 + static_cast<int64_t>(CW) * j;
+            if (lane == 0 && row < p.m) {
+                const float v = static_cast<float>(static_cast<int64_t>(s0) + static_cast<int64_t>(s1));
+                const __nv_bfloat16 h = __float2bfloat16_rn(fmaf(v, scale, corr));
+                p.Y[row] = *reinterpret_cast<const uint16_t *>(&h);
+            }
+        }
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 // ------------------------------------------------------------------ block Walsh-Hadamard rotation
@@ -525,16 +805,36 @@ size_t packed_gemv_corr_offset(int64_t N, int64_t n) {
     return ((xp + 255) / 256) * 256;
 }
 
-// Rows per unit for the TMA variant: balance the units over the persistent CTAs.
-static int choose_rows(int64_t m, int ctas) {
+// Rows per unit for the TMA variants: balance the units over the persistent CTAs (R a multiple of step).
+static int choose_rows(int64_t m, int ctas, int step = 16) {
     int best = 64;
     double best_eff = -1.0;
-    for (int R = kTmaMaxRows; R >= 64; R -= 16) {
+    for (int R = kTmaMaxRows; R >= 64; R -= step) {
         const int64_t units = (m + R - 1) / R;
         const int64_t rounds = (units + ctas - 1) / ctas;
         const double eff = static_cast<double>(units) / static_cast<double>(rounds * (units < ctas ? units : ctas));
         const double rows_eff = static_cast<double>(m) / static_cast<double>(units * R);
         const double e = eff * rows_eff;
+        if (e > best_eff + 1e-9) { best_eff = e; best = R; }
+    }
+    return best;
+}
+
+// Rows per thread per tile the dp2a kernel is instantiated for (a unit has kDpWarps * RPT rows).
+static const int kDpRpts[] = {16, 12, 8, 6, 4, 3, 2, 1};
+
+// Rows per unit for the dp2a variant: balance the units over the CTAs, and prefer all SMs busy.
+static int choose_rows_dp(int64_t m, int ctas) {
+    int best = kDpWarps;
+    double best_eff = -1.0;
+    for (int rpt : kDpRpts) {
+        const int R = kDpWarps * rpt;
+        const int64_t units = (m + R - 1) / R;
+        const int64_t rounds = (units + ctas - 1) / ctas;
+        const double eff = static_cast<double>(units) / static_cast<double>(rounds * (units < ctas ? units : ctas));
+        const double rows_eff = static_cast<double>(m) / static_cast<double>(units * R);
+        const double busy = static_cast<double>(units < ctas ? units : ctas) / static_cast<double>(ctas);
+        const double e = eff * rows_eff * busy;
         if (e > best_eff + 1e-9) { best_eff = e; best = R; }
     }
     return best;
@@ -572,9 +872,65 @@ static cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t
     return cudaLaunchKernelEx(&cfg, k, std::forward<Args>(args)...);
 }
 
+// dp2a variant for one token. Leaves `done` false (and launches nothing) when the activations do
+// not fit in shared memory next to a ring of at least three stages.
+static cudaError_t launch_packed_gemv_dp(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, bool &done) {
+    done = false;
+    const int nkc = static_cast<int>(gemv_npad(a.n) / kTileCols);
+    const int R = choose_rows_dp(a.m, num_sms);
+    int stages = kTmaStages;
+    while (stages >= 3 && dp_smem_layout(R, stages, nkc).total + 1024 > kDpSmemLimit) --stages;
+    if (stages < 3) return cudaSuccess;
+    CUtensorMap map;
+    if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
+    GemvDpParams p;
+    p.X = a.Xf ? static_cast<const void *>(a.Xf) : static_cast<const void *>(a.X);
+    p.A = a.A;
+    p.b = a.b;
+    p.m = a.m;
+    p.n = a.n;
+    p.d = d;
+    p.f32in = a.Xf != nullptr;
+    p.R = R;
+    p.units = static_cast<int>((a.m + R - 1) / R);
+    p.nkc = nkc;
+    p.stages = stages;
+    p.Y = a.Y;
+    p.status = a.status;
+    const int grid = p.units < num_sms ? p.units : num_sms;
+    const size_t smem = dp_smem_layout(R, stages, nkc).total + 1024;
+    void (*k)(const CUtensorMap, const GemvDpParams) = nullptr;
+    switch (R / kDpWarps) {
+        case 16: k = packed_gemv_dp_kernel<16>; break;
+        case 12: k = packed_gemv_dp_kernel<12>; break;
+        case 8: k = packed_gemv_dp_kernel<8>; break;
+        case 6: k = packed_gemv_dp_kernel<6>; break;
+        case 4: k = packed_gemv_dp_kernel<4>; break;
+        case 3: k = packed_gemv_dp_kernel<3>; break;
+        case 2: k = packed_gemv_dp_kernel<2>; break;
+        default: k = packed_gemv_dp_kernel<1>; break;
+    }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(k, dim3(grid), dim3(32 * (kDpWarps + 1)), smem, st, map, p);
+    count_launch();
+    if (e != cudaSuccess) return e;
+    done = true;
+    return cudaSuccess;
+}
+
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st) {
     const int64_t npad = gemv_npad(a.n), nprep = gemv_nprep(a.n);
     trace_begin(LCQ_K_GEMV, st);
+    if (a.n % 64 == 0 && a.n <= kDpMaxN && a.m >= 16 && a.N == kDpMaxTokens) {
+        bool done = false;
+        const cudaError_t e = launch_packed_gemv_dp(a, d, num_sms, st, done);
+        if (e != cudaSuccess) return e;
+        if (done) {
+            trace_end(LCQ_K_GEMV, st);
+            return cudaGetLastError();
+        }
+    }
     dim3 pgrid(static_cast<unsigned>(a.N), static_cast<unsigned>(nprep));
     if (a.Xf) {
         if (d == 4) gemv_prep_kernel<4, true><<<pgrid, 256, 0, st>>>(a.Xf, a.n, npad, a.A, a.b, a.Xp, a.corr);

@@ -242,7 +242,7 @@ def test_linear_empty_tokens_gives_zero_gradients():
 
 # ----------------------------------------------------------------------------- deployment product
 
-@pytest.mark.parametrize("N", [1, 4, 16, 17, 40])
+@pytest.mark.parametrize("N", [1, 2, 3, 4, 5, 16, 17, 40])
 @pytest.mark.parametrize("m,n,d", [(200, 512, 8), (64, 1024, 4), (70, 200, 4), (8, 8, 8), (1000, 4096, 8),
                                    (300, 8192, 4)])
 def test_gemm_packed2b_matches_oracle(N, m, n, d):
@@ -256,6 +256,56 @@ def test_gemm_packed2b_matches_oracle(N, m, n, d):
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
     lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
+
+
+# One token with n % 64 == 0 takes the integer (dp2a) kernel: activations as int16 with one scale
+# per token (a bound on max|X'|), exact int32 sums. Its only errors are the int16 rounding (at most
+# 2^-16 of the bound per element) and the bf16 output rounding (2^-9 relative), so it is held to a
+# tighter bound than the bf16 parity bar, on heavy-tailed activations (1% of the columns x50); two to
+# four tokens (tensor-core kernel) keep the bf16 bar. (300, 28672) puts 56 activation tiles in
+# shared memory next to the code ring.
+TOL_DP = 4e-3
+
+
+@pytest.mark.parametrize("N", [1, 2, 3, 4])
+@pytest.mark.parametrize("m,n,d", [(1000, 4096, 8), (300, 8192, 4), (300, 28672, 8), (16, 64, 8), (4000, 512, 4)])
+def test_gemm_packed2b_few_tokens_heavy_tailed(N, m, n, d):
+    rng = np.random.default_rng(7 * N + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n))
+    X[:, rng.random(n) < 0.01] *= 50.0
+    Xb = wl.bf16_bits(X.astype(np.float32))
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+    lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    tol = TOL_DP if N == 1 else TOL_BF16
+    assert max_rel(host_bf16(Y), ref) <= tol
+
+
+def test_gemm_packed2b_one_token_zero_activations():
+    # a half-zero token, and an all-zero token (scale 0)
+    rng = np.random.default_rng(5)
+    m, n, d, N = 256, 2048, 8, 1
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    for zero in ("half", "all"):
+        X = rng.normal(0, 1, (N, n))
+        X[0, :1024] = 0.0
+        if zero == "all":
+            X[0, :] = 0.0
+        Xb = wl.bf16_bits(X.astype(np.float32))
+        ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+        Y = empty_bf16(N, m)
+        ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+        lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+        got = host_bf16(Y)
+        if zero == "all":
+            assert np.all(got == 0.0)
+        else:
+            assert max_rel(got, ref) <= TOL_DP
 
 
 # ----------------------------------------------------------------------------- failure detection
