@@ -739,34 +739,107 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
 
 // ------------------------------------------------------------------ block Walsh-Hadamard rotation
 //
-// out[r, blk*B + j] = (1/sqrt(B)) sum_i in[r, blk*B + i] * H_B[i][j] (Sylvester H, symmetric):
-// one CTA per (row, block) transforms the block in shared memory (log2 B butterfly stages).
-// in may equal out (each block is read whole before it is written).
+// out[r, blk*B + j] = (1/sqrt(B)) sum_i in[r, blk*B + i] * H_B[i][j] (Sylvester H, symmetric). The
+// transform factors over the bits of the index: one stage per bit combines each pair of elements whose
+// indices differ in that bit only, (u, v) -> (u + v, u - v). in may equal out (each block is read whole
+// before it is written).
+//
+// Blocks of B >= 64: one CTA of T = B / E threads per (row, block); element idx = t + T i sits in
+// register i of thread t. Index bits [log2 T, log2 B) are combined in registers, bits [0, 5) (the lane)
+// with warp shuffles, and bits [5, log2 T) (the warp) after one exchange through shared memory, where
+// each thread takes elements that differ only in those bits and then writes its results.
+// Blocks of B <= 32: one thread per block, all stages in registers.
+
+template <int E>
+__device__ __forceinline__ void wht_registers(float (&x)[E]) {
+#pragma unroll
+    for (int h = 1; h < E; h <<= 1)
+#pragma unroll
+        for (int i = 0; i < E; ++i)
+            if ((i & h) == 0) {
+                const float u = x[i], v = x[i + h];
+                x[i] = u + v;
+                x[i + h] = u - v;
+            }
+}
 
 template <typename InT>
-__global__ void __launch_bounds__(1024)
-hadamard_kernel(const InT *__restrict__ in, int64_t n, int bsz, float *out) {
+__device__ __forceinline__ float load_act(const InT *p, int64_t i) {
+    if constexpr (sizeof(InT) == 2)
+        return __uint_as_float(static_cast<uint32_t>(p[i]) << 16);
+    else
+        return p[i];
+}
+
+template <int LB>
+struct WhtShape {
+    static constexpr int B = 1 << LB;
+    static constexpr int E = LB >= 14 ? 32 : (LB >= 9 ? 16 : B / 32);   // elements per thread
+    static constexpr int T = B / E;                                        // threads, 32 .. 1024
+    static constexpr int LT = LB >= 14 ? LB - 5 : (LB >= 9 ? LB - 4 : 5);
+    static constexpr int W = LT - 5;                                       // warp index bits
+};
+
+template <int LB, typename InT>
+__global__ void __launch_bounds__(WhtShape<LB>::T)
+hadamard_block_kernel(const InT *__restrict__ in, int64_t n, float *out) {
+    using S = WhtShape<LB>;
+    constexpr int E = S::E, T = S::T, W = S::W;
+    static_assert(S::B == E * T && (1 << S::LT) == T && (1 << W) <= E, "bad shape");
     extern __shared__ float hbuf[];
-    const int64_t row = blockIdx.x;
-    const int64_t base = row * n + static_cast<int64_t>(blockIdx.y) * bsz;
-    for (int i = threadIdx.x; i < bsz; i += blockDim.x) {
-        if constexpr (sizeof(InT) == 2)
-            hbuf[i] = __uint_as_float(static_cast<uint32_t>(in[base + i]) << 16);
-        else
-            hbuf[i] = in[base + i];
-    }
-    __syncthreads();
-    for (int h = 1; h < bsz; h <<= 1) {
-        for (int p = threadIdx.x; p < bsz / 2; p += blockDim.x) {
-            const int i = (p / h) * 2 * h + (p % h);
-            const float u = hbuf[i], v = hbuf[i + h];
-            hbuf[i] = u + v;
-            hbuf[i + h] = u - v;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * n + static_cast<int64_t>(blockIdx.y) * S::B;
+    const float scale = rsqrtf(static_cast<float>(S::B));
+    float x[E];
+#pragma unroll
+    for (int i = 0; i < E; ++i) x[i] = load_act(in, base + t + T * i);
+    wht_registers<E>(x);                                   // bits [LT, LB)
+#pragma unroll
+    for (int h = 1; h < 32; h <<= 1) {                     // bits [0, 5)
+        const bool hi = (lane & h) != 0;
+#pragma unroll
+        for (int i = 0; i < E; ++i) {
+            const float o = __shfl_xor_sync(0xffffffffu, x[i], h);
+            x[i] = hi ? o - x[i] : x[i] + o;
         }
-        __syncthreads();
     }
-    const float scale = rsqrtf(static_cast<float>(bsz));
-    for (int i = threadIdx.x; i < bsz; i += blockDim.x) out[base + i] = hbuf[i] * scale;
+    if constexpr (W == 0) {
+#pragma unroll
+        for (int i = 0; i < E; ++i) out[base + t + T * i] = x[i] * scale;
+    } else {
+        // bits [5, LT): element lane | k << 5 | (warp | g << W) << LT, k < 2^W, g < E / 2^W
+#pragma unroll
+        for (int i = 0; i < E; ++i) hbuf[t + T * i] = x[i];
+        __syncthreads();
+        constexpr int K = 1 << W, G = E / K;
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            float y[K];
+            const int hi_part = (warp | (g << W)) << S::LT;
+#pragma unroll
+            for (int k = 0; k < K; ++k) y[k] = hbuf[lane | (k << 5) | hi_part];
+            wht_registers<K>(y);
+#pragma unroll
+            for (int k = 0; k < K; ++k) out[base + (lane | (k << 5) | hi_part)] = y[k] * scale;
+        }
+    }
+}
+
+template <int LB, typename InT>
+__global__ void __launch_bounds__(256)
+hadamard_small_kernel(const InT *__restrict__ in, int64_t rows, int64_t n, float *out) {
+    constexpr int B = 1 << LB;
+    const int64_t nb = n >> LB;
+    const int64_t blk = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+    if (blk >= rows * nb) return;
+    const int64_t base = (blk / nb) * n + (blk % nb) * B;
+    float x[B];
+#pragma unroll
+    for (int i = 0; i < B; ++i) x[i] = load_act(in, base + i);
+    wht_registers<B>(x);
+    const float scale = rsqrtf(static_cast<float>(B));
+#pragma unroll
+    for (int i = 0; i < B; ++i) out[base + i] = x[i] * scale;
 }
 
 int hadamard_block_size(int64_t n) {
@@ -775,23 +848,52 @@ int hadamard_block_size(int64_t n) {
     return bsz;
 }
 
-cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t n, float *out, cudaStream_t st) {
-    const int bsz = hadamard_block_size(n);
-    const int threads = bsz / 2 < 1024 ? (bsz / 2 < 32 ? 32 : bsz / 2) : 1024;
-    const size_t smem = static_cast<size_t>(bsz) * 4;
-    dim3 grid(static_cast<unsigned>(rows), static_cast<unsigned>(n / bsz));
-    cudaError_t e;
-    if (in_bf16) {
-        e = ensure_dynamic_smem(reinterpret_cast<const void *>(hadamard_kernel<uint16_t>), static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        hadamard_kernel<uint16_t><<<grid, threads, smem, st>>>(static_cast<const uint16_t *>(in), n, bsz, out);
+template <int LB, typename InT>
+static cudaError_t launch_wht(const InT *in, int64_t rows, int64_t n, float *out, cudaStream_t st) {
+    if constexpr (LB <= 5) {
+        const int64_t blocks = rows * (n >> LB);
+        hadamard_small_kernel<LB, InT><<<static_cast<unsigned>((blocks + 255) / 256), 256, 0, st>>>(in, rows, n, out);
     } else {
-        e = ensure_dynamic_smem(reinterpret_cast<const void *>(hadamard_kernel<float>), static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        hadamard_kernel<float><<<grid, threads, smem, st>>>(static_cast<const float *>(in), n, bsz, out);
+        using S = WhtShape<LB>;
+        const size_t smem = S::W > 0 ? static_cast<size_t>(S::B) * 4 : 0;
+        if (smem) {
+            const cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(hadamard_block_kernel<LB, InT>),
+                                                      static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+        }
+        dim3 grid(static_cast<unsigned>(rows), static_cast<unsigned>(n >> LB));
+        hadamard_block_kernel<LB, InT><<<grid, S::T, smem, st>>>(in, n, out);
     }
-    count_launch();
     return cudaGetLastError();
+}
+
+template <typename InT>
+static cudaError_t launch_wht_any(const InT *in, int64_t rows, int64_t n, float *out, cudaStream_t st) {
+    switch (hadamard_block_size(n)) {
+        case 1: return launch_wht<0>(in, rows, n, out, st);
+        case 2: return launch_wht<1>(in, rows, n, out, st);
+        case 4: return launch_wht<2>(in, rows, n, out, st);
+        case 8: return launch_wht<3>(in, rows, n, out, st);
+        case 16: return launch_wht<4>(in, rows, n, out, st);
+        case 32: return launch_wht<5>(in, rows, n, out, st);
+        case 64: return launch_wht<6>(in, rows, n, out, st);
+        case 128: return launch_wht<7>(in, rows, n, out, st);
+        case 256: return launch_wht<8>(in, rows, n, out, st);
+        case 512: return launch_wht<9>(in, rows, n, out, st);
+        case 1024: return launch_wht<10>(in, rows, n, out, st);
+        case 2048: return launch_wht<11>(in, rows, n, out, st);
+        case 4096: return launch_wht<12>(in, rows, n, out, st);
+        case 8192: return launch_wht<13>(in, rows, n, out, st);
+        case 16384: return launch_wht<14>(in, rows, n, out, st);
+        default: return launch_wht<15>(in, rows, n, out, st);
+    }
+}
+
+cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t n, float *out, cudaStream_t st) {
+    const cudaError_t e = in_bf16 ? launch_wht_any(static_cast<const uint16_t *>(in), rows, n, out, st)
+                                  : launch_wht_any(static_cast<const float *>(in), rows, n, out, st);
+    count_launch();
+    return e;
 }
 
 size_t packed_gemv_workspace(int64_t N, int64_t n) {

@@ -367,7 +367,8 @@ def test_init_latent_matches_oracle_and_requantizes_to_the_same_codes(m, n):
 
 # ----------------------------------------------------------------------------- Hadamard rotation
 
-@pytest.mark.parametrize("rows,n", [(3, 8), (5, 96), (2, 8192), (4, 14336)])
+@pytest.mark.parametrize("rows,n", [(3, 8), (5, 96), (3, 64), (2, 1024), (2, 8192), (4, 14336), (3, 6144), (1, 16384),
+                                    (2, 65536)])
 def test_hadamard_rotation_matches_oracle(rows, n):
     torch = T()
     X = np.random.default_rng(rows + n).normal(size=(rows, n)).astype(np.float32)
