@@ -291,28 +291,42 @@ packed_gemv_kernel(const uint8_t *__restrict__ packed, int64_t m, int64_t n, int
 }
 
 // ------------------------------------------------------------------ TMA-streamed variant
+//
+// Persistent CTAs: one producer thread streams (R rows x 512 columns) code tiles through a ring of 2-D
+// TMA copies (128-byte swizzle, bank-conflict-free fragment reads). CW consumer warps: warp w owns the
+// 64-column slice w % 8 of every tile and the RBW consecutive 16-row blocks of row group w / 8, so a
+// unit has R = (CW / 8) * 16 * RBW rows. mma.sync is latency-bound per warp here, so the warp count
+// is what hides the conversion and MMA latencies; the eight slices of a row are summed through
+// shared memory in a fixed order at the end of each unit.
 
 constexpr int kTmaStages = 8;
-constexpr int kTmaMaxRows = 128;      // rows of W per unit (multiple of 16)
 constexpr int kColGroups = 8;         // 64-column slices of a 512-column tile
 constexpr int kTileCols = 512;        // 128 bytes of codes per row per stage
-
-struct GemvSmem {
-    uint8_t ring[kTmaStages][kTmaMaxRows * 128];
-    float red[kColGroups][kTmaMaxRows][17];
-    uint64_t full[kTmaStages];
-    uint64_t empty[kTmaStages];
-    float corr[16];
-};
+constexpr size_t kGemvSmemLimit = 227 * 1024;
 
 struct GemvTmaParams {
     int64_t m, N, npad, nprep;
-    int R, units, nkc;
+    int R, units, nkc, stages;
     const uint16_t *Xp;       // [N][npad] (token 0 of this launch)
     const float *corrpart;    // [N][nprep]
     uint16_t *Y;              // [N][m]
     int32_t *status;
 };
+
+// Shared-memory layout (offsets from the 1024-byte aligned base): ring, slice partial sums
+// [8][R][8 NT + 1], barriers, per-token constants.
+struct GemvTmaLayout {
+    size_t red, bars, corr, total;
+};
+__host__ __device__ inline GemvTmaLayout gemv_tma_layout(int R, int stages, int nt) {
+    GemvTmaLayout L;
+    L.red = static_cast<size_t>(stages) * static_cast<size_t>(R) * 128;
+    L.bars = L.red + static_cast<size_t>(kColGroups) * static_cast<size_t>(R) * (8 * nt + 1) * 4;
+    L.bars = (L.bars + 15) / 16 * 16;
+    L.corr = L.bars + 2 * kTmaStages * 8;
+    L.total = L.corr + 16 * 4;
+    return L;
+}
 
 __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
     uint32_t v;
@@ -320,20 +334,28 @@ __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
     return v;
 }
 
-// NT: 8-token MMA tiles (1: N <= 8, 2: N <= 16). CW: consumer warps; with 16 the two warps of a
-// 64-column slice split its rows, doubling the warps available to hide latency.
-template <int NT, int CW>
+// NT: 8-token MMA tiles (1: N <= 8, 2: N <= 16). CW: consumer warps (a multiple of 8). RBW: 16-row
+// blocks per warp per tile.
+template <int NT, int CW, int RBW>
 __global__ void __launch_bounds__(32 * (CW + 1), 1)
 packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaParams p) {
-    constexpr int kRbPerWarp = (kTmaMaxRows / 16) / (CW / kColGroups);
+    static_assert(CW % kColGroups == 0, "consumer warps must cover the 8 slices");
+    constexpr int R = (CW / kColGroups) * 16 * RBW;
+    constexpr int LD = 8 * NT + 1;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    GemvSmem &s = *reinterpret_cast<GemvSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const GemvTmaLayout L = gemv_tma_layout(R, p.stages, NT);
+    float *red = reinterpret_cast<float *>(base + L.red);          // [8][R][LD]
+    uint64_t *full = reinterpret_cast<uint64_t *>(base + L.bars);
+    uint64_t *empty = full + kTmaStages;
+    float *corr_s = reinterpret_cast<float *>(base + L.corr);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr uint32_t kStageBytes = static_cast<uint32_t>(R) * 128u;
     if (threadIdx.x == 0) {
         prefetch_tensormap(&tmC);
-        for (int i = 0; i < kTmaStages; ++i) {
-            mbar_init(&s.full[i], 1);
-            mbar_init(&s.empty[i], CW);
+        for (int i = 0; i < p.stages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], CW);
         }
         fence_barrier_init();
     }
@@ -342,14 +364,14 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
     if (warp == 0) {
         // ---------------------------------------------------------------- producer: code tiles -> ring
         if (lane == 0) {
-            const uint32_t bytes = static_cast<uint32_t>(p.R) * 128u;
-            int it = 0;
+            int st = 0;
+            uint32_t ph = 0;
             for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
-                for (int kc = 0; kc < p.nkc; ++kc, ++it) {
-                    const int st = it % kTmaStages;
-                    if (!mbar_wait(&s.empty[st], ((it / kTmaStages) & 1) ^ 1, p.status)) return;
-                    mbar_arrive_expect_tx(&s.full[st], bytes);
-                    tma_load_2d(s.ring[st], &tmC, kc * 128, u * p.R, &s.full[st]);
+                for (int kc = 0; kc < p.nkc; ++kc) {
+                    if (!mbar_wait(&empty[st], ph ^ 1, p.status)) return;
+                    mbar_arrive_expect_tx(&full[st], kStageBytes);
+                    tma_load_2d(base + static_cast<size_t>(st) * kStageBytes, &tmC, kc * 128, u * R, &full[st]);
+                    if (++st == p.stages) { st = 0; ph ^= 1; }
                 }
             }
         }
@@ -359,16 +381,17 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
     // -------------------------------------------------------------------- consumers
     asm volatile("griddepcontrol.wait;" ::: "memory");   // X' and corr partials of the prep kernel
     const int cw = (warp - 1) % kColGroups;              // 64-column slice
-    const int rb0 = ((warp - 1) / kColGroups) * kRbPerWarp;
+    const int rb0 = ((warp - 1) / kColGroups) * RBW;
     const int g = lane >> 2, tid = lane & 3;
     const int ct = threadIdx.x - 32;
-    if (ct < p.N) s.corr[ct] = token_corr(p.corrpart, ct, p.nprep);
+    if (ct < p.N) corr_s[ct] = token_corr(p.corrpart, ct, p.nprep);
     asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
     const bool has0 = g < p.N, has1 = (g + 8) < p.N;
     const uint32_t *xp0 = reinterpret_cast<const uint32_t *>(p.Xp + (has0 ? g : 0) * p.npad);
     const uint32_t *xp1 = reinterpret_cast<const uint32_t *>(p.Xp + (has1 ? g + 8 : 0) * p.npad);
-    const int nrb = p.R / 16;
-    const uint32_t swz = static_cast<uint32_t>((cw ^ g) << 4) + 4u * tid;   // this lane's word in a swizzled row
+    // this lane's word in its rows (row % 8 == g): 16-byte chunk cw ^ g, word tid
+    const uint32_t swz = static_cast<uint32_t>((cw ^ g) << 4) + 4u * tid + static_cast<uint32_t>((rb0 * 16 + g) * 128);
+    const uint32_t ring0 = smem_u32(base);
 
     // activation fragments of this warp's 64 columns of tile kc (16-column block of this lane's word);
     // the next tile's fragments are fetched while the current tile is multiplied.
@@ -384,58 +407,58 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
     uint2 bcur[4][NT], bnext[4][NT];
     load_frags(0, bcur);
 
-    int it = 0;
+    int st = 0;
+    uint32_t ph = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-        float acc[kRbPerWarp][NT][4];
+        float acc[RBW][NT][4];
 #pragma unroll
-        for (int i = 0; i < kRbPerWarp; ++i)
+        for (int i = 0; i < RBW; ++i)
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) acc[i][nt][e] = 0.0f;
 
-        for (int kc = 0; kc < p.nkc; ++kc, ++it) {
-            const int st = it % kTmaStages;
+        for (int kc = 0; kc < p.nkc; ++kc) {
             load_frags(kc + 1 < p.nkc ? kc + 1 : 0, bnext);
-            if (!mbar_wait(&s.full[st], (it / kTmaStages) & 1, p.status)) { ok = false; break; }
-            const uint32_t base = smem_u32(s.ring[st]) + swz;
+            if (!mbar_wait(&full[st], ph, p.status)) { ok = false; break; }
+            const uint32_t tbase = ring0 + static_cast<uint32_t>(st) * kStageBytes + swz;
             // row blocks in pairs: two blocks' fragments converted, then their MMAs interleaved (h outer)
 #pragma unroll
-            for (int rp = 0; rp < kRbPerWarp / 2; ++rp) {
-                const int rb = rb0 + 2 * rp;
-                if (rb < nrb) {
-                    const bool second = rb + 1 < nrb;
-                    uint32_t w[2][2];
+            for (int rp = 0; rp < (RBW + 1) / 2; ++rp) {
+                constexpr int kLast = RBW - 1;
+                const bool second = 2 * rp + 1 <= kLast;
+                uint32_t w[2][2];
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        const uint32_t rbase = static_cast<uint32_t>((rb + j) * 16 + g) * 128u;
-                        w[j][0] = (j == 0 || second) ? lds32(base + rbase) : 0u;
-                        w[j][1] = (j == 0 || second) ? lds32(base + rbase + 8u * 128u) : 0u;
-                    }
-                    uint32_t f[2][2][8];
+                for (int j = 0; j < 2; ++j) {
+                    const uint32_t rbase = static_cast<uint32_t>((2 * rp + j) * 16 * 128);
+                    w[j][0] = (j == 0 || second) ? lds32(tbase + rbase) : 0u;
+                    w[j][1] = (j == 0 || second) ? lds32(tbase + rbase + 8u * 128u) : 0u;
+                }
+                uint32_t f[2][2][8];
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
+                for (int j = 0; j < 2; ++j) {
+                    if (j == 0 || second) {
                         codes_to_frags(w[j][0], f[j][0]);
                         codes_to_frags(w[j][1], f[j][1]);
                     }
+                }
 #pragma unroll
-                    for (int h = 0; h < 4; ++h) {
+                for (int h = 0; h < 4; ++h) {
 #pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            if (j == 0 || second) {
+                    for (int j = 0; j < 2; ++j) {
+                        if (j == 0 || second) {
 #pragma unroll
-                                for (int nt = 0; nt < NT; ++nt)
-                                    mma_bf16_16816(acc[2 * rp + j][nt], f[j][0][2 * h], f[j][1][2 * h],
-                                                   f[j][0][2 * h + 1], f[j][1][2 * h + 1], bcur[h][nt].x,
-                                                   bcur[h][nt].y);
-                            }
+                            for (int nt = 0; nt < NT; ++nt)
+                                mma_bf16_16816(acc[2 * rp + j][nt], f[j][0][2 * h], f[j][1][2 * h], f[j][0][2 * h + 1],
+                                               f[j][1][2 * h + 1], bcur[h][nt].x, bcur[h][nt].y);
                         }
                     }
                 }
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(&s.empty[st]);
+            if (lane == 0) mbar_arrive(&empty[st]);
+            if (++st == p.stages) { st = 0; ph ^= 1; }
 #pragma unroll
             for (int h = 0; h < 4; ++h)
 #pragma unroll
@@ -444,28 +467,28 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
         if (!ok) break;
         // cross-slice reduction (fixed order), + corr, bf16 store
 #pragma unroll
-        for (int i = 0; i < kRbPerWarp; ++i) {
-            const int rb = rb0 + i;
-            if (rb < nrb) {
+        for (int i = 0; i < RBW; ++i) {
+            const int r = 16 * (rb0 + i) + g;
 #pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                    s.red[cw][16 * rb + g][nt * 8 + 2 * tid] = acc[i][nt][0];
-                    s.red[cw][16 * rb + g][nt * 8 + 2 * tid + 1] = acc[i][nt][1];
-                    s.red[cw][16 * rb + g + 8][nt * 8 + 2 * tid] = acc[i][nt][2];
-                    s.red[cw][16 * rb + g + 8][nt * 8 + 2 * tid + 1] = acc[i][nt][3];
-                }
+            for (int nt = 0; nt < NT; ++nt) {
+                float *r0 = red + (static_cast<size_t>(cw) * R + r) * LD + nt * 8 + 2 * tid;
+                float *r8 = r0 + 8 * LD;
+                r0[0] = acc[i][nt][0];
+                r0[1] = acc[i][nt][1];
+                r8[0] = acc[i][nt][2];
+                r8[1] = acc[i][nt][3];
             }
         }
         asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
-        const int64_t row0 = static_cast<int64_t>(u) * p.R;
-        for (int o = ct; o < p.R * p.N; o += 32 * CW) {
-            const int rl = o % p.R, tl = o / p.R;
+        const int64_t row0 = static_cast<int64_t>(u) * R;
+        for (int o = ct; o < R * p.N; o += 32 * CW) {
+            const int rl = o % R, tl = o / R;
             const int64_t row = row0 + rl;
             if (row >= p.m) continue;
             float v = 0.0f;
 #pragma unroll
-            for (int w = 0; w < kColGroups; ++w) v += s.red[w][rl][tl];
-            v += s.corr[tl];
+            for (int w = 0; w < kColGroups; ++w) v += red[(static_cast<size_t>(w) * R + rl) * LD + tl];
+            v += corr_s[tl];
             const __nv_bfloat16 h = __float2bfloat16_rn(v);
             p.Y[static_cast<int64_t>(tl) * p.m + row] = *reinterpret_cast<const uint16_t *>(&h);
         }
@@ -907,17 +930,36 @@ size_t packed_gemv_corr_offset(int64_t N, int64_t n) {
     return ((xp + 255) / 256) * 256;
 }
 
-// Rows per unit for the TMA variants: balance the units over the persistent CTAs (R a multiple of step).
-static int choose_rows(int64_t m, int ctas, int step = 16) {
-    int best = 64;
+// Tensor-core variant configurations: (token groups, consumer warps, row blocks per warp). The unit
+// has (CW / 8) * 16 * RBW rows; the launcher picks the configuration whose units balance best over
+// the CTAs.
+struct GemvTmaConfig {
+    int nt, cw, rbw;
+    void (*kernel)(const CUtensorMap, const GemvTmaParams);
+};
+// In order of preference (measured on the 70B gate: 24 x 2 at 1-8 tokens, 8 x 4 at 9-16 tokens);
+// a later entry wins only if its units balance at least half a percent better.
+static const GemvTmaConfig kGemvTmaConfigs[] = {
+    {1, 24, 2, packed_gemv_tma_kernel<1, 24, 2>}, {1, 16, 4, packed_gemv_tma_kernel<1, 16, 4>},
+    {1, 24, 4, packed_gemv_tma_kernel<1, 24, 4>}, {1, 16, 2, packed_gemv_tma_kernel<1, 16, 2>},
+    {1, 24, 1, packed_gemv_tma_kernel<1, 24, 1>}, {1, 16, 1, packed_gemv_tma_kernel<1, 16, 1>},
+    {2, 8, 4, packed_gemv_tma_kernel<2, 8, 4>},   {2, 8, 2, packed_gemv_tma_kernel<2, 8, 2>},
+    {2, 16, 2, packed_gemv_tma_kernel<2, 16, 2>}, {2, 16, 1, packed_gemv_tma_kernel<2, 16, 1>},
+};
+
+static const GemvTmaConfig *choose_tma_config(int64_t m, int ctas, int nt) {
+    const GemvTmaConfig *best = nullptr;
     double best_eff = -1.0;
-    for (int R = kTmaMaxRows; R >= 64; R -= step) {
+    for (const GemvTmaConfig &c : kGemvTmaConfigs) {
+        if (c.nt != nt) continue;
+        const int R = (c.cw / kColGroups) * 16 * c.rbw;
         const int64_t units = (m + R - 1) / R;
         const int64_t rounds = (units + ctas - 1) / ctas;
         const double eff = static_cast<double>(units) / static_cast<double>(rounds * (units < ctas ? units : ctas));
         const double rows_eff = static_cast<double>(m) / static_cast<double>(units * R);
-        const double e = eff * rows_eff;
-        if (e > best_eff + 1e-9) { best_eff = e; best = R; }
+        const double busy = static_cast<double>(units < ctas ? units : ctas) / static_cast<double>(ctas);
+        const double e = eff * rows_eff * busy;
+        if (e > best_eff + 0.005) { best_eff = e; best = &c; }
     }
     return best;
 }
@@ -1045,31 +1087,32 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (a.n % 64 == 0 && a.m >= 16) {
-        const int R = choose_rows(a.m, num_sms);
-        CUtensorMap map;
-        if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
-        const int units = static_cast<int>((a.m + R - 1) / R);
-        const int grid = units < num_sms ? units : num_sms;
-        const size_t smem = sizeof(GemvSmem) + 1024;
         for (int64_t t0 = 0; t0 < a.N; t0 += 16) {
+            const int64_t ntok = (a.N - t0) < 16 ? (a.N - t0) : 16;
+            const GemvTmaConfig *c = choose_tma_config(a.m, num_sms, ntok > 8 ? 2 : 1);
+            const int R = (c->cw / kColGroups) * 16 * c->rbw;
+            CUtensorMap map;
+            if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
+            int stages = kTmaStages;
+            while (stages > 2 && gemv_tma_layout(R, stages, c->nt).total + 1024 > kGemvSmemLimit) --stages;
             GemvTmaParams p;
             p.m = a.m;
-            p.N = (a.N - t0) < 16 ? (a.N - t0) : 16;
+            p.N = ntok;
             p.npad = npad;
             p.nprep = nprep;
             p.R = R;
-            p.units = units;
+            p.units = static_cast<int>((a.m + R - 1) / R);
             p.nkc = static_cast<int>(npad / kTileCols);
+            p.stages = stages;
             p.Xp = a.Xp + t0 * npad;
             p.corrpart = a.corr + t0 * nprep;
             p.Y = a.Y + t0 * a.m;
             p.status = a.status;
-            const bool two = p.N > 8;
-            auto k = two ? packed_gemv_tma_kernel<2, 8> : packed_gemv_tma_kernel<1, 16>;
-            const int threads = two ? 32 * 9 : 32 * 17;
-            e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
+            const int grid = p.units < num_sms ? p.units : num_sms;
+            const size_t smem = gemv_tma_layout(R, stages, c->nt).total + 1024;
+            e = ensure_dynamic_smem(reinterpret_cast<const void *>(c->kernel), static_cast<int>(smem));
             if (e != cudaSuccess) return e;
-            e = launch_pdl(k, dim3(grid), dim3(threads), smem, st, map, p);
+            e = launch_pdl(c->kernel, dim3(grid), dim3(32 * (c->cw + 1)), smem, st, map, p);
             count_launch();
             if (e != cudaSuccess) return e;
         }
