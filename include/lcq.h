@@ -24,8 +24,11 @@
  *     lcq_workspace_size(op, ...) bytes (LCQ_ERR_WORKSPACE otherwise). The
  *     first 256 bytes of a workspace hold a device status word that kernels
  *     set on device-detected errors (LCQ_ERR_SINGULAR, LCQ_ERR_TIMEOUT);
- *     read it with lcq_device_status(). A workspace must not be shared by
- *     calls that may run concurrently.
+ *     read it with lcq_device_status(). The header must be zero before a
+ *     workspace is first used (lcq_encode also keeps a counter there that
+ *     returns to zero at the end of every call); after a device-detected
+ *     error, zero it again. A workspace must not be shared by calls that may
+ *     run concurrently.
  *   - Packed codes: 4 per byte; column c of a row sits in bits
  *     2*(c mod 4) .. 2*(c mod 4)+1 of byte c/4 of that row (LSB first);
  *     a packed matrix is m x (n/4) bytes.
@@ -106,9 +109,10 @@ size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d);
  * latent  [m][n] fp32 output u, or NULL.
  * mse     device double, receives mean((W - (A z + b))^2) over all m*n
  *         weights (0 when m*n == 0), or NULL.
- * A^{-1} is formed on the device (fp64 Gauss-Jordan, rounded to fp32); if A
- * is singular the device status word becomes LCQ_ERR_SINGULAR and every code
- * is 0. Needs lcq_workspace_size(LCQ_OP_ENCODE, 0, m, n, d) bytes of ws.
+ * A^{-1} is formed on the device to fp32 accuracy (fp32 Gauss-Jordan refined
+ * by Newton steps with a double-float residual; fp64 Gauss-Jordan when A is
+ * badly conditioned); if A is singular the device status word becomes
+ * LCQ_ERR_SINGULAR and every code is 0. Needs lcq_workspace_size(LCQ_OP_ENCODE, 0, m, n, d) bytes of ws.
  */
 lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b,
                       uint8_t *packed, uint8_t *codes, float *latent, double *mse,

@@ -24,7 +24,7 @@ struct EncodeArgs {
     float *latent;
     double *mse;
     double *partials;     // [grid] per-CTA sums of squared residuals
-    unsigned *counter;    // zeroed before launch
+    unsigned *counter;    // zero between calls: the last CTA wraps it back (atomicInc)
     int32_t *status;
 };
 

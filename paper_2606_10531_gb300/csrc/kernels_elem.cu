@@ -6,9 +6,10 @@
 //   reduce_partials  fixed-order sum of per-CTA dA/db partials
 //
 // encode and quant_decode stream their fp32 input through a shared-memory ring
-// filled by the bulk-copy (TMA) engine: one producer thread issues 16 KB
-// cp.async.bulk copies, eight compute warps consume them. Each compute thread
-// owns 16 consecutive weights of a chunk, i.e. whole groups for d = 4 and 8.
+// filled by the bulk-copy (TMA) engine: one producer thread issues 22 KB
+// cp.async.bulk copies, eleven compute warps consume them. In encode, thread t takes
+// the groups t, t + T, ... of a chunk (conflict-free shared-memory reads); in quant_decode
+// each compute thread owns 16 consecutive weights, i.e. whole groups for d = 4 and 8.
 #include "common.cuh"
 #include "internal.h"
 
@@ -29,7 +30,8 @@ struct StreamSmem {
     float A[64];
     float M[64];        // A^T A (encode MSE)
     float b[8];
-    double gj[8][16];
+    double gj[8][16];   // fp64 elimination (fallback)
+    float gjf[8][16];   // Newton iterate X (columns 0..d-1) and residual R (columns d..2d-1)
     double dred[kComputeWarps];
     int singular;
 };
@@ -54,10 +56,11 @@ __device__ void stream_producer(StreamSmem &s, const float *src, int64_t total, 
     }
 }
 
-// One warp: A^{-1} by Gauss-Jordan elimination with partial pivoting in fp64, rounded to fp32,
-// and M = A^T A. Sets s.singular if a pivot is (relatively) zero.
-template <int D>
-__device__ void invert_warp(StreamSmem &s) {
+// One warp: A^{-1} by Gauss-Jordan elimination with partial pivoting in fp64, rounded to fp32.
+// Sets s.singular if a pivot is (relatively) zero. Slow on this part (fp64 latency), so it is the
+// fallback of invert_warp.
+template <int D, typename Smem>
+__device__ void invert_fp64_warp(Smem &s) {
     const int lane = threadIdx.x & 31;
     double amax = 0.0;
     for (int e = lane; e < D * 2 * D; e += 32) {
@@ -65,12 +68,6 @@ __device__ void invert_warp(StreamSmem &s) {
         const double v = c < D ? static_cast<double>(s.A[r * D + c]) : (c - D == r ? 1.0 : 0.0);
         s.gj[r][c] = v;
         if (c < D) amax = fmax(amax, fabs(v));
-    }
-    for (int e = lane; e < D * D; e += 32) {
-        const int i = e / D, j = e % D;
-        double acc = 0.0;
-        for (int r = 0; r < D; ++r) acc += static_cast<double>(s.A[r * D + i]) * static_cast<double>(s.A[r * D + j]);
-        s.M[e] = static_cast<float>(acc);
     }
     for (int o = 16; o; o >>= 1) amax = fmax(amax, __shfl_xor_sync(0xffffffffu, amax, o));
     __syncwarp();
@@ -109,6 +106,164 @@ __device__ void invert_warp(StreamSmem &s) {
         s.Ainv[e] = singular ? 0.0f : static_cast<float>(s.gj[r][D + c]);
     }
     if (lane == 0) s.singular = singular;
+    __syncwarp();
+}
+
+// Error-free transformations in fp32: a*b = p + e exactly (FMA), and a + b = s + err exactly (TwoSum).
+__device__ __forceinline__ void two_prod(float a, float b, float &p, float &e) {
+    p = a * b;
+    e = fmaf(a, b, -p);
+}
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) {
+    s = a + b;
+    const float bb = s - a;
+    err = (a - (s - bb)) + (b - bb);
+}
+
+// One warp: A^{-1} and M = A^T A (fp32).
+//  1. Gauss-Jordan elimination with partial pivoting in fp32, in registers: lane r + D h (r < D,
+//     h < 2D/8) holds columns 8h .. 8h+7 of row r of [A | I]; pivots, row swaps and the pivot row
+//     are exchanged with warp shuffles.
+//  2. Newton steps X <- X + X R with the residual R = I - A X accumulated in double-float (fp32 pairs:
+//     FMA-exact products, TwoSum accumulation): each step squares the residual (I - A X' = R^2) without
+//     fp64 arithmetic, which is slow on this part. One step suffices for well-conditioned A.
+//  3. If the residual does not reach the acceptance bound within four steps (A badly conditioned, or
+//     non-finite), the fp64 elimination runs instead.
+// Sets s.singular if a pivot is (relatively) zero.
+template <int D, typename Smem>
+__device__ void invert_warp(Smem &s) {
+    constexpr int H = 2 * D / 8;                 // 8-column blocks of [A | I]
+    const int lane = threadIdx.x & 31;
+    const int r = lane % D, h = lane / D;
+    const bool act = lane < D * H;
+    float row[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int c = 8 * h + j;
+        row[j] = !act ? 0.0f : (c < D ? s.A[r * D + c] : (c - D == r ? 1.0f : 0.0f));
+    }
+    for (int e = lane; e < D * D; e += 32) {
+        const int i = e / D, j = e % D;
+        float acc = 0.0f;
+        for (int k = 0; k < D; ++k) acc = fmaf(s.A[k * D + i], s.A[k * D + j], acc);
+        s.M[e] = acc;
+    }
+    float amax = 0.0f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+        if (8 * h + j < D) amax = fmaxf(amax, fabsf(row[j]));
+    for (int o = 16; o; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+    int singular = !(amax > 0.0f) || !isfinite(amax);
+#pragma unroll
+    for (int c = 0; c < D; ++c) {
+        if (singular) break;
+        // pivot: largest |a[r][c]| over rows r >= c (column c sits in block 0, lane r)
+        float v = (act && h == 0 && r >= c) ? fabsf(row[c]) : -1.0f;
+        int idx = r;
+        for (int o = 16; o; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+            if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
+        }
+        if (!(static_cast<double>(v) > 1e-12 * static_cast<double>(amax)) || !isfinite(v)) { singular = 1; break; }
+        const int prow = idx;
+        // swap rows c and prow, within each column block
+        const int src = (r == c) ? prow : (r == prow ? c : r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src + D * h);
+        const float piv = __shfl_sync(0xffffffffu, row[c], c);     // a[c][c], block 0
+        const float rinv = 1.0f / piv;
+        if (r == c) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) row[j] *= rinv;
+        }
+        const float f = __shfl_sync(0xffffffffu, row[c], r);       // a[r][c] of this lane's row
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const float pc = __shfl_sync(0xffffffffu, row[j], c + D * h);   // pivot row, same block
+            if (r != c) row[j] = fmaf(-f, pc, row[j]);
+        }
+    }
+    if (singular) {
+        for (int e = lane; e < D * D; e += 32) s.Ainv[e] = 0.0f;
+        if (lane == 0) s.singular = 1;
+        __syncwarp();
+        return;
+    }
+    // X = right half of [I | A^{-1}]
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int c = 8 * h + j;
+        if (act && c >= D) s.gjf[r][c - D] = row[j];
+    }
+    __syncwarp();
+    // Acceptance: the residual of any fp32-stored inverse has a rounding floor of about
+    // cond(A) 2^-24; stop after the update whose residual was within 8x that floor (capped at 1e-4,
+    // beyond which the fp64 elimination is used), cond(A) estimated as ||A||_inf ||X||_inf.
+    float arow = 0.0f, xrow = 0.0f;
+    if (lane < D) {
+        for (int k = 0; k < D; ++k) {
+            arow += fabsf(s.A[lane * D + k]);
+            xrow += fabsf(s.gjf[lane][k]);
+        }
+    }
+    for (int o = 16; o; o >>= 1) {
+        arow = fmaxf(arow, __shfl_xor_sync(0xffffffffu, arow, o));
+        xrow = fmaxf(xrow, __shfl_xor_sync(0xffffffffu, xrow, o));
+    }
+    const float accept = fmaxf(1e-6f, fminf(8.0f * arow * xrow * 5.9604645e-8f, 1e-4f));
+    bool ok = false;
+    for (int pass = 0; pass < 4; ++pass) {
+        float res = 0.0f;
+        float Rv[2] = {0.0f, 0.0f};
+        for (int q = 0; q < 2; ++q) {
+            const int e = lane + 32 * q;
+            if (e < D * D) {
+                const int i = e / D, j = e % D;
+                float hi = (i == j) ? 1.0f : 0.0f, lo = 0.0f;
+                for (int k = 0; k < D; ++k) {
+                    float pp, pe, t, te;
+                    two_prod(s.A[i * D + k], s.gjf[k][j], pp, pe);
+                    two_sum(hi, -pp, t, te);
+                    hi = t;
+                    lo += te - pe;
+                }
+                Rv[q] = hi + lo;
+                res = fmaxf(res, fabsf(Rv[q]));
+            }
+        }
+        for (int o = 16; o; o >>= 1) res = fmaxf(res, __shfl_xor_sync(0xffffffffu, res, o));
+        if (!(res <= 0.5f)) break;                              // not converging (or non-finite): fall back
+        for (int q = 0; q < 2; ++q) {
+            const int e = lane + 32 * q;
+            if (e < D * D) s.gjf[e / D][D + e % D] = Rv[q];      // R beside X
+        }
+        __syncwarp();
+        float Xn[2] = {0.0f, 0.0f};
+        for (int q = 0; q < 2; ++q) {
+            const int e = lane + 32 * q;
+            if (e < D * D) {
+                const int i = e / D, j = e % D;
+                float corr = 0.0f;
+                for (int k = 0; k < D; ++k) corr = fmaf(s.gjf[i][k], s.gjf[k][D + j], corr);
+                Xn[q] = s.gjf[i][j] + corr;
+            }
+        }
+        __syncwarp();
+        for (int q = 0; q < 2; ++q) {
+            const int e = lane + 32 * q;
+            if (e < D * D) s.gjf[e / D][e % D] = Xn[q];
+        }
+        __syncwarp();
+        if (res <= accept) { ok = true; break; }
+    }
+    if (!ok) {
+        invert_fp64_warp<D>(s);
+        return;
+    }
+    for (int e = lane; e < D * D; e += 32) s.Ainv[e] = s.gjf[e / D][e % D];
+    if (lane == 0) s.singular = 0;
+    __syncwarp();
 }
 
 // ------------------------------------------------------------------ encode
@@ -213,12 +368,21 @@ encode_kernel(EncodeArgs a) {
     compute_bar();
     if (s.singular && blockIdx.x == 0 && threadIdx.x == 32) set_status(a.status, LCQ_ERR_SINGULAR);
 
+    // Thread t encodes the groups t, t + T, ... of each chunk (T compute threads), so consecutive threads
+    // read consecutive groups. For d = 8 a group is two 16-byte units; threads with bit 2 of t set read
+    // the second unit first, which puts the eight 16-byte reads of a quarter warp in distinct banks.
+    // Their weights arrive with the halves swapped, so their copy of A^{-1} has its columns swapped too.
+    const int t = threadIdx.x - 32;
+    const int hswap = (D == 8) ? ((t >> 2) & 1) : 0;
     float2 Ai2[D / 2][D], c2[D / 2];
     QuadCoef<D> qc;
 #pragma unroll
     for (int kp = 0; kp < D / 2; ++kp)
 #pragma unroll
-        for (int j = 0; j < D; ++j) Ai2[kp][j] = make_float2(s.Ainv[(2 * kp) * D + j], s.Ainv[(2 * kp + 1) * D + j]);
+        for (int j = 0; j < D; ++j) {
+            const int jc = j ^ (4 * hswap);
+            Ai2[kp][j] = make_float2(s.Ainv[(2 * kp) * D + jc], s.Ainv[(2 * kp + 1) * D + jc]);
+        }
 #pragma unroll
     for (int kp = 0; kp < D / 2; ++kp) {
         float c0 = 0.0f, c1 = 0.0f;
@@ -241,8 +405,9 @@ encode_kernel(EncodeArgs a) {
         }
     }
 
-    const int t = threadIdx.x - 32;
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
+    constexpr int kGroupsPerThread = kPerThread / D;
+    constexpr int kThreads = 32 * kComputeWarps;
     float sq = 0.0f;
     int i = 0;
     for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++i) {
@@ -250,56 +415,45 @@ encode_kernel(EncodeArgs a) {
         if (!mbar_wait(&s.full[st], (i / kStages) & 1, a.status)) break;
         const int64_t base = c * kChunk;
         const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
-        const int64_t off = static_cast<int64_t>(t) * kPerThread;
-        if (off < cnt) {
-            const int valid = static_cast<int>((cnt - off) < kPerThread ? (cnt - off) : kPerThread);
-            const float *src = s.buf[st] + off;
-            const int64_t gidx = base + off;   // flat weight index, multiple of 16
-            uint32_t p = 0;
-            // every group of the slice is computed (a ragged tail reads stale shared memory that is
-            // neither stored nor summed): valid is a multiple of d
+        const int ngroups = static_cast<int>(cnt / D);   // n % 8 == 0: whole groups
 #pragma unroll
-            for (int g = 0; g < kPerThread / D; ++g) {
+        for (int k = 0; k < kGroupsPerThread; ++k) {
+            const int g = t + k * kThreads;
+            if (g < ngroups) {
+                const float4 *src = reinterpret_cast<const float4 *>(s.buf[st] + g * D);
                 float w[D];
-#pragma unroll
-                for (int q = 0; q < D / 4; ++q) {
-                    const float4 f = reinterpret_cast<const float4 *>(src + g * D)[q];
-                    w[4 * q] = f.x; w[4 * q + 1] = f.y; w[4 * q + 2] = f.z; w[4 * q + 3] = f.w;
+                if (D == 8) {
+                    const float4 f0 = src[hswap], f1 = src[1 - hswap];
+                    w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
+                    w[4] = f1.x; w[5] = f1.y; w[6] = f1.z; w[7] = f1.w;
+                } else {
+                    const float4 f0 = src[0];
+                    w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
                 }
                 float u[D];
                 float gsq = 0.0f;
-                encode_group<D, kMse>(w, Ai2, qc, c2, p, 2 * g * D, u, gsq);
-                if (g * D < valid) {
-                    sq += gsq;
-                    if (kLatent) {
-                        float4 *dst = reinterpret_cast<float4 *>(a.latent + gidx + g * D);
-#pragma unroll
-                        for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
-                    }
+                uint32_t p = 0;
+                encode_group<D, kMse>(w, Ai2, qc, c2, p, 0, u, gsq);
+                sq += gsq;
+                const int64_t gidx = base + static_cast<int64_t>(g) * D;   // flat index of the group's first weight
+                if (a.packed) {
+                    if (D == 8) *reinterpret_cast<uint16_t *>(a.packed + gidx / 4) = static_cast<uint16_t>(p);
+                    else a.packed[gidx / 4] = static_cast<uint8_t>(p);
                 }
-            }
-
-            if (valid == kPerThread) {
-                if (a.packed) *reinterpret_cast<uint32_t *>(a.packed + gidx / 4) = p;
                 if (a.codes) {
-                    // spread 2-bit fields to bytes: byte k of word q = code 4q + k
-                    uint32_t ww[4];
+                    uint32_t ww[D / 4];
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
+                    for (int q = 0; q < D / 4; ++q) {
                         const uint32_t f = (p >> (8 * q)) & 0xFFu;
                         ww[q] = (f & 3u) | (((f >> 2) & 3u) << 8) | (((f >> 4) & 3u) << 16) | (((f >> 6) & 3u) << 24);
                     }
-                    *reinterpret_cast<uint4 *>(a.codes + gidx) = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+                    if (D == 8) *reinterpret_cast<uint2 *>(a.codes + gidx) = make_uint2(ww[0], ww[D / 4 - 1]);
+                    else *reinterpret_cast<uint32_t *>(a.codes + gidx) = ww[0];
                 }
-            } else {
+                if (kLatent) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.latent + gidx);
 #pragma unroll
-                for (int k = 0; k < kPerThread; k += 4) {
-                    if (k < valid) {
-                        if (a.packed) a.packed[(gidx + k) / 4] = static_cast<uint8_t>((p >> (2 * k)) & 0xFFu);
-#pragma unroll
-                        for (int e = 0; e < 4; ++e)
-                            if (a.codes) a.codes[gidx + k + e] = static_cast<uint8_t>((p >> (2 * (k + e))) & 3u);
-                    }
+                    for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
                 }
             }
         }
@@ -311,17 +465,25 @@ encode_kernel(EncodeArgs a) {
         for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
         if (lane == 0) s.dred[warp - 1] = static_cast<double>(sq);
         compute_bar();
-        if (t == 0) {
-            double acc = 0.0;
-            for (int w = 0; w < kComputeWarps; ++w) acc += s.dred[w];
-            a.partials[blockIdx.x] = acc;
-            __threadfence();
-            const unsigned prev = atomicAdd(a.counter, 1u);
+        if (warp == 1) {
+            // per-CTA partial; the counter wraps to zero when the last CTA arrives (atomicInc), so it
+            // is back at zero for the next call without a reset
+            unsigned prev = 0;
+            if (lane == 0) {
+                double acc = 0.0;
+                for (int w = 0; w < kComputeWarps; ++w) acc += s.dred[w];
+                a.partials[blockIdx.x] = acc;
+                __threadfence();
+                prev = atomicInc(a.counter, gridDim.x - 1);
+            }
+            prev = __shfl_sync(0xffffffffu, prev, 0);
             if (prev == gridDim.x - 1) {
+                // last CTA: the partials summed by the warp in a fixed order
                 __threadfence();
                 double tot = 0.0;
-                for (unsigned p = 0; p < gridDim.x; ++p) tot += __ldcg(a.partials + p);
-                *a.mse = total > 0 ? tot / static_cast<double>(total) : 0.0;
+                for (unsigned q = lane; q < gridDim.x; q += 32) tot += __ldcg(a.partials + q);
+                for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+                if (lane == 0) *a.mse = total > 0 ? tot / static_cast<double>(total) : 0.0;
             }
         }
     }

@@ -338,7 +338,6 @@ lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *
     a.partials = reinterpret_cast<double *>(static_cast<uint8_t *>(ws) + kHeader);
     a.counter = &h->counter;
     a.status = &h->status;
-    if (mse) LCQ_TRY(cuda_status(cudaMemsetAsync(&h->counter, 0, sizeof(uint32_t), st)));
     return cuda_status(launch_encode(a, d, num_sms_current(), st));
 }
 

@@ -76,6 +76,34 @@ def test_encode_matches_oracle(m, n, d):
     print(f"near-boundary codes excluded: {int(np.sum(ref['near']))} of {m * n}")
 
 
+@pytest.mark.parametrize("d", [4, 8])
+@pytest.mark.parametrize("cond", [1e3, 1e6, 3e7])
+def test_encode_inverse_accuracy_ill_conditioned(d, cond):
+    # With b = 0 and a one-hot group w = e_g, the latent is u = A^{-1} e_g exactly (every other product
+    # is an exact zero), so the latent output exposes the device's A^{-1} column by column. It must be
+    # the fp64 inverse rounded to fp32, whatever the conditioning (the widest case takes the fp64
+    # elimination path).
+    torch = T()
+    rng = np.random.default_rng(int(cond) + d)
+    Q1, _ = np.linalg.qr(rng.normal(size=(d, d)))
+    Q2, _ = np.linalg.qr(rng.normal(size=(d, d)))
+    A = (0.02 * Q1 @ np.diag(np.logspace(0, -np.log10(cond), d)) @ Q2.T).astype(np.float32)
+    b = np.zeros(d, dtype=np.float32)
+    m = 4
+    W = np.tile(np.eye(d, dtype=np.float32).reshape(1, d * d), (m, 1))      # groups e_0 .. e_{d-1}
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, d * d, d)
+    latent = torch.empty((m, d * d), dtype=torch.float32, device="cuda")
+    mse = torch.empty(1, dtype=torch.float64, device="cuda")
+    lcq.lcq_encode(dev(W), dev(A), dev(b), d, ws, latent=latent, mse=mse)
+    assert lcq.lcq_device_status(ws) == 0
+    inv = oracle.inverse(A)                                  # fp64
+    got = latent.cpu().numpy().astype(np.float64).reshape(m, d, d)   # [row][group g][k] = A^{-1}[k][g]
+    for r in range(m):
+        # fp32 rounding of each entry, plus the forward error of any fp64 inverse (~cond * 1e-16 of its norm)
+        tol = 2.5e-7 * np.abs(inv) + 2e-8 * np.max(np.abs(inv))
+        assert np.all(np.abs(got[r].T - inv) <= tol), f"max err/tol {np.max(np.abs(got[r].T - inv) / tol)}"
+
+
 def test_encode_nonfinite_inputs():
     torch = T()
     d, m, n = 8, 4, 32
