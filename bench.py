@@ -178,7 +178,8 @@ def traffic_from_profile(kernel_src: str):
 # ----------------------------------------------------------------------------- extras
 
 def time_encode_70b(torch, lcq, wl, seed, device, pk):
-    """Bulk encode of all linears of a Llama-3-70B layer (d=8): packed codes + MSE."""
+    """Bulk encode of all linears of a Llama-3-70B layer (d=8): packed codes + MSE, as one batched call
+    (lcq_encode_batch); the same pass as seven lcq_encode calls is reported beside it."""
     mats = wl.llama3_70b_layer_encode()
     bufs = []
     for i, mx in enumerate(mats):
@@ -188,14 +189,19 @@ def time_encode_70b(torch, lcq, wl, seed, device, pk):
         bufs.append((mx, W, A, b, torch.empty((mx.m, mx.n // 4), dtype=torch.uint8, device=device),
                      torch.empty(1, dtype=torch.float64, device=device),
                      lcq.workspace(lcq.LCQ_OP_ENCODE, 0, mx.m, mx.n, mx.d, device)))
+    items = [{"W": W, "A": A, "b": b, "packed": pk_, "mse": mse} for mx, W, A, b, pk_, mse, _ in bufs]
+    items_codes = [{"W": W, "A": A, "b": b, "packed": pk_} for mx, W, A, b, pk_, mse, _ in bufs]
+    ws_batch = lcq.workspace(lcq.LCQ_OP_ENCODE_BATCH, len(items), 0, 0, mats[0].d, device)
 
     def run():
-        for mx, W, A, b, pk_, mse, ws in bufs:
-            lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
+        lcq.lcq_encode_batch(items, mats[0].d, ws_batch)
 
     def run_codes_only():
+        lcq.lcq_encode_batch(items_codes, mats[0].d, ws_batch)
+
+    def run_single_calls():
         for mx, W, A, b, pk_, mse, ws in bufs:
-            lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_)
+            lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
 
     def timed(fn, iters=10):
         for _ in range(3):
@@ -209,21 +215,25 @@ def time_encode_70b(torch, lcq, wl, seed, device, pk):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / 1e3 / iters
 
+    t_single = timed(run_single_calls)
     t_codes = timed(run_codes_only)
     t = timed(run)
     weights = sum(mx.m * mx.n for mx in mats)
     gbs = weights * 4.25 / t / 1e9
+    assert lcq.lcq_device_status(ws_batch) == 0
     for *_, ws in bufs:
         assert lcq.lcq_device_status(ws) == 0
     mses = [float(x[5].item()) for x in bufs]
-    del bufs
+    del bufs, items, items_codes
     return {"workload": "llama3-70b-layer bulk encode: q,o 8192x8192, k,v 1024x8192, gate,up 28672x8192, "
-                        "down 8192x28672; d=8; W ~N(0,0.015) + 0.1% Student-t(4); packed codes + MSE",
+                        "down 8192x28672; d=8; W ~N(0,0.015) + 0.1% Student-t(4); packed codes + MSE; "
+                        "one lcq_encode_batch call",
             "weights": weights, "ms": t * 1e3, "GB/s": gbs, "bytes_per_weight": 4.25,
             "frac_hbm": gbs / pk["hbm"], "mse": mses, "l2": "inputs larger than L2 (3.4 GB per pass)",
             "codes_only": {"ms": t_codes * 1e3, "GB/s": weights * 4.25 / t_codes / 1e9,
                            "frac_hbm": weights * 4.25 / t_codes / 1e9 / pk["hbm"],
-                           "note": "same pass without the reconstruction MSE"}}
+                           "note": "same batched pass without the reconstruction MSE"},
+            "seven_lcq_encode_calls": {"ms": t_single * 1e3, "frac_hbm": weights * 4.25 / t_single / 1e9 / pk["hbm"]}}
 
 
 def time_gemv_70b(torch, lcq, wl, seed, device, pk):

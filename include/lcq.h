@@ -63,7 +63,8 @@ typedef enum lcq_op {
     LCQ_OP_LINEAR_FWD = 2,
     LCQ_OP_LINEAR_BWD = 3,
     LCQ_OP_GEMM_PACKED2B = 4,
-    LCQ_OP_GEMM_PACKED2B_HADAMARD = 5
+    LCQ_OP_GEMM_PACKED2B_HADAMARD = 5,
+    LCQ_OP_ENCODE_BATCH = 6          /* N = number of matrices; m, n unused */
 } lcq_op;
 
 /* Gradient estimators for dP through the rounding (Sec. 3.3). */
@@ -117,6 +118,36 @@ size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d);
 lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b,
                       uint8_t *packed, uint8_t *codes, float *latent, double *mse,
                       void *ws, size_t ws_bytes, void *stream);
+
+/* One matrix of lcq_encode_batch: the arguments of lcq_encode for it. */
+typedef struct lcq_encode_item {
+    const float *W;        /* [m][n] fp32 input                              */
+    int64_t m, n;          /* n a multiple of 8                              */
+    const float *A, *b;    /* its affine map (d x d row-major, d)            */
+    uint8_t *packed;       /* [m][n/4] uint8 output, or NULL                 */
+    uint8_t *codes;        /* [m][n] uint8 output, or NULL                   */
+    float *latent;         /* [m][n] fp32 output, or NULL                    */
+    double *mse;           /* device double output, or NULL                  */
+} lcq_encode_item;
+
+#define LCQ_ENCODE_BATCH_MAX 16
+
+/*
+ * lcq_encode_batch - lcq_encode of several matrices (the bulk encode of all linears of a layer: PTQ
+ * initialisation, per-step requantisation). Every output is exactly the one lcq_encode gives for the
+ * same matrix. The matrices share the group size d. When no item asks for the MSE they stream through
+ * one persistent launch, so the per-call costs (launch, forming A^{-1}, filling the ring) are paid
+ * once for the batch; when any item asks for it, each matrix gets its own launch (measured faster).
+ *
+ * items  host array of `count` matrices, 1 <= count <= LCQ_ENCODE_BATCH_MAX; each item is
+ *        validated as lcq_encode validates its arguments.
+ * Needs lcq_workspace_size(LCQ_OP_ENCODE_BATCH, count, 0, 0, d) bytes of ws. The workspace header
+ * holds one counter per matrix, which returns to zero at the end of every call (the header must be
+ * zero before first use). If any A is singular the status word becomes LCQ_ERR_SINGULAR and that
+ * matrix's codes are 0.
+ */
+lcq_status lcq_encode_batch(const lcq_encode_item *items, int count, int d, void *ws, size_t ws_bytes,
+                            void *stream);
 
 /*
  * lcq_decode - affine decode of packed codes (Sec. 3.2 Eq. def:forward):

@@ -19,13 +19,15 @@ STATUS_NAMES = {0: "LCQ_OK", 1: "LCQ_ERR_NULL", 2: "LCQ_ERR_SHAPE", 3: "LCQ_ERR_
                 5: "LCQ_ERR_WORKSPACE", 6: "LCQ_ERR_CUDA", 7: "LCQ_ERR_SINGULAR", 8: "LCQ_ERR_TIMEOUT",
                 9: "LCQ_ERR_ARG", 10: "LCQ_ERR_LIMIT"}
 LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B, LCQ_OP_GEMM_PACKED2B_HADAMARD = 1, 2, 3, 4, 5
+LCQ_OP_ENCODE_BATCH = 6
+LCQ_ENCODE_BATCH_MAX = 16
 LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 
 # Every symbol include/lcq.h declares.
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
            "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout",
-           "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard")
+           "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard", "lcq_encode_batch")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
                 "gemv_prep", "gemv")
 
@@ -50,9 +52,16 @@ class lcq_opts(ctypes.Structure):
 
 _P = ctypes.c_void_p
 _I64 = ctypes.c_int64
+
+
+class lcq_encode_item(ctypes.Structure):
+    _fields_ = [("W", _P), ("m", _I64), ("n", _I64), ("A", _P), ("b", _P), ("packed", _P), ("codes", _P),
+                ("latent", _P), ("mse", _P)]
 _SIG = {
     "lcq_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I64, _I64, _I64, ctypes.c_int]),
     "lcq_encode": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "lcq_encode_batch": (ctypes.c_int, [ctypes.POINTER(lcq_encode_item), ctypes.c_int, ctypes.c_int, _P,
+                                        ctypes.c_size_t, _P]),
     "lcq_decode": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
     "lcq_pack2b": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
     "lcq_linear_fwd": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P,
@@ -143,6 +152,17 @@ def lcq_encode(W, A, b, d: int, ws, packed=None, codes=None, latent=None, mse=No
     m, n = W.shape
     _check(lib().lcq_encode(_ptr(W), m, n, d, _ptr(A), _ptr(b), _ptr(packed), _ptr(codes), _ptr(latent), _ptr(mse),
                             _ptr(ws), ws.numel(), _stream(stream)), "lcq_encode")
+
+
+def lcq_encode_batch(items, d: int, ws, stream=None):
+    """items: sequence of dicts with W, A, b and optional packed, codes, latent, mse tensors (as lcq_encode)."""
+    arr = (lcq_encode_item * len(items))()
+    for k, it in enumerate(items):
+        m, n = it["W"].shape
+        addr = lambda t: None if t is None else t.data_ptr()  # noqa: E731
+        arr[k] = lcq_encode_item(addr(it["W"]), m, n, addr(it["A"]), addr(it["b"]), addr(it.get("packed")),
+                                 addr(it.get("codes")), addr(it.get("latent")), addr(it.get("mse")))
+    _check(lib().lcq_encode_batch(arr, len(items), d, _ptr(ws), ws.numel(), _stream(stream)), "lcq_encode_batch")
 
 
 def lcq_decode(packed, n: int, d: int, A, b, W_hat_f32=None, W_hat_bf16=None, stream=None):

@@ -28,6 +28,32 @@ struct EncodeArgs {
     int32_t *status;
 };
 
+constexpr int kEncodeBatchMax = 16;   // = LCQ_ENCODE_BATCH_MAX
+constexpr int kEncodeBatchPartials = 2048;   // per-matrix partials slots in a batch workspace (>= grid)
+
+struct EncodeBatchItem {
+    const float *W;
+    int64_t m, n;
+    const float *A, *b;
+    uint8_t *packed, *codes;
+    float *latent;
+    double *mse;
+    int64_t chunk0;       // first chunk of this matrix in the batch's chunk list
+    int64_t nchunks;
+};
+
+struct EncodeBatchArgs {
+    EncodeBatchItem item[kEncodeBatchMax];
+    int count;
+    int64_t total_chunks;
+    double *partials;     // [count][grid] per-CTA sums of squared residuals
+    unsigned *counters;   // [count], zero between calls (atomicInc wraps them back)
+    int32_t *status;
+};
+
+// Chunk size (fp32 weights) of the encode pipeline.
+int64_t encode_chunk_size();
+
 struct QuantDecodeArgs {
     const float *P;
     int64_t m, n;
@@ -48,6 +74,7 @@ struct DecodeArgs {
 
 int encode_max_blocks(int num_sms);
 cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t st);
+cudaError_t launch_encode_batch(const EncodeBatchArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, int num_sms, cudaStream_t st);

@@ -340,6 +340,128 @@ __device__ __forceinline__ void encode_group(const float *w, const float2 (&Ai2)
     if (kMse) sq += quad_form<D>(qc, e);
 }
 
+// The per-thread copy of a matrix's encode constants: A^{-1} as row pairs (columns swapped for the
+// threads that read the halves of their groups swapped), c = -A^{-1} b, and the quadratic-form
+// coefficients of A^T A.
+template <int D>
+__device__ __forceinline__ void load_encode_constants(const float *Ainv, const float *M, const float *b, int hswap,
+                                                      float2 (&Ai2)[D / 2][D], float2 (&c2)[D / 2], QuadCoef<D> &qc) {
+#pragma unroll
+    for (int kp = 0; kp < D / 2; ++kp)
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            const int jc = j ^ (4 * hswap);
+            Ai2[kp][j] = make_float2(Ainv[(2 * kp) * D + jc], Ainv[(2 * kp + 1) * D + jc]);
+        }
+#pragma unroll
+    for (int kp = 0; kp < D / 2; ++kp) {
+        float c0 = 0.0f, c1 = 0.0f;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            c0 = fmaf(-Ainv[(2 * kp) * D + j], b[j], c0);
+            c1 = fmaf(-Ainv[(2 * kp + 1) * D + j], b[j], c1);
+        }
+        c2[kp] = make_float2(c0, c1);
+    }
+    int idx = 0;
+#pragma unroll
+    for (int i = 0; i < D; i += 2) {
+        qc.diag[i / 2] = M[i * D + i];
+        // row i gets 2*M[i][j] for j > i; row i+1 gets M[i+1][i+1] at j = i+1, 2*M[i+1][j] beyond
+#pragma unroll
+        for (int j = i + 1; j < D; ++j)
+            qc.pair[idx++] = make_float2(2.0f * M[i * D + j], (j == i + 1 ? 1.0f : 2.0f) * M[(i + 1) * D + j]);
+    }
+}
+
+// Encode one chunk held in shared memory (cnt weights starting at flat index base of a matrix).
+// Thread t encodes the groups t, t + T, ... of the chunk (T compute threads), so consecutive threads
+// read consecutive groups. For d = 8 a group is two 16-byte units; threads with bit 2 of t set read
+// the second unit first, which puts the eight 16-byte reads of a quarter warp in distinct banks (their
+// constants were loaded with the columns swapped to match).
+template <int D, bool kMse>
+__device__ __forceinline__ void encode_chunk(const float *buf, int64_t base, int64_t cnt, int t, int hswap,
+                                             const float2 (&Ai2)[D / 2][D], const QuadCoef<D> &qc,
+                                             const float2 (&c2)[D / 2], uint8_t *packed, uint8_t *codes, float *latent,
+                                             float &sq) {
+    constexpr int kGroupsPerThread = kPerThread / D;
+    constexpr int kThreads = 32 * kComputeWarps;
+    const int ngroups = static_cast<int>(cnt / D);   // n % 8 == 0: whole groups
+#pragma unroll
+    for (int k = 0; k < kGroupsPerThread; ++k) {
+        const int g = t + k * kThreads;
+        if (g < ngroups) {
+            const float4 *src = reinterpret_cast<const float4 *>(buf + g * D);
+            float w[D];
+            if (D == 8) {
+                const float4 f0 = src[hswap], f1 = src[1 - hswap];
+                w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
+                w[4] = f1.x; w[5] = f1.y; w[6] = f1.z; w[7] = f1.w;
+            } else {
+                const float4 f0 = src[0];
+                w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
+            }
+            float u[D];
+            float gsq = 0.0f;
+            uint32_t p = 0;
+            encode_group<D, kMse>(w, Ai2, qc, c2, p, 0, u, gsq);
+            sq += gsq;
+            const int64_t gidx = base + static_cast<int64_t>(g) * D;   // flat index of the group's first weight
+            if (packed) {
+                if (D == 8) *reinterpret_cast<uint16_t *>(packed + gidx / 4) = static_cast<uint16_t>(p);
+                else packed[gidx / 4] = static_cast<uint8_t>(p);
+            }
+            if (codes) {
+                uint32_t ww[D / 4];
+#pragma unroll
+                for (int q = 0; q < D / 4; ++q) {
+                    const uint32_t f = (p >> (8 * q)) & 0xFFu;
+                    ww[q] = (f & 3u) | (((f >> 2) & 3u) << 8) | (((f >> 4) & 3u) << 16) | (((f >> 6) & 3u) << 24);
+                }
+                if (D == 8) *reinterpret_cast<uint2 *>(codes + gidx) = make_uint2(ww[0], ww[D / 4 - 1]);
+                else *reinterpret_cast<uint32_t *>(codes + gidx) = ww[0];
+            }
+            if (latent) {
+                float4 *dst = reinterpret_cast<float4 *>(latent + gidx);
+#pragma unroll
+                for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+            }
+        }
+    }
+}
+
+
+// End of a matrix's share of a CTA: the compute threads' sums of squared residuals become one
+// per-CTA partial (fixed order); the CTA that arrives last (counter wraps back to zero, atomicInc)
+// sums the partials in a fixed order and writes the mean. All compute warps call it together; dred
+// must not be reused until every compute warp has passed the next compute_bar.
+__device__ __forceinline__ void mse_flush(float &sq, double *dred, double *partials, unsigned *counter, double *mse,
+                                          int64_t total) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    if (lane == 0) dred[warp - 1] = static_cast<double>(sq);
+    sq = 0.0f;
+    compute_bar();
+    if (warp == 1) {
+        unsigned prev = 0;
+        if (lane == 0) {
+            double acc = 0.0;
+            for (int w = 0; w < kComputeWarps; ++w) acc += dred[w];
+            partials[blockIdx.x] = acc;
+            __threadfence();
+            prev = atomicInc(counter, gridDim.x - 1);
+        }
+        prev = __shfl_sync(0xffffffffu, prev, 0);
+        if (prev == gridDim.x - 1) {
+            __threadfence();
+            double tot = 0.0;
+            for (unsigned q = lane; q < gridDim.x; q += 32) tot += __ldcg(partials + q);
+            for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+            if (lane == 0 && mse) *mse = total > 0 ? tot / static_cast<double>(total) : 0.0;
+        }
+    }
+}
+
 template <int D, bool kMse, bool kLatent>
 __global__ void __launch_bounds__(kStreamThreads, 1)
 encode_kernel(EncodeArgs a) {
@@ -368,46 +490,13 @@ encode_kernel(EncodeArgs a) {
     compute_bar();
     if (s.singular && blockIdx.x == 0 && threadIdx.x == 32) set_status(a.status, LCQ_ERR_SINGULAR);
 
-    // Thread t encodes the groups t, t + T, ... of each chunk (T compute threads), so consecutive threads
-    // read consecutive groups. For d = 8 a group is two 16-byte units; threads with bit 2 of t set read
-    // the second unit first, which puts the eight 16-byte reads of a quarter warp in distinct banks.
-    // Their weights arrive with the halves swapped, so their copy of A^{-1} has its columns swapped too.
     const int t = threadIdx.x - 32;
     const int hswap = (D == 8) ? ((t >> 2) & 1) : 0;
     float2 Ai2[D / 2][D], c2[D / 2];
     QuadCoef<D> qc;
-#pragma unroll
-    for (int kp = 0; kp < D / 2; ++kp)
-#pragma unroll
-        for (int j = 0; j < D; ++j) {
-            const int jc = j ^ (4 * hswap);
-            Ai2[kp][j] = make_float2(s.Ainv[(2 * kp) * D + jc], s.Ainv[(2 * kp + 1) * D + jc]);
-        }
-#pragma unroll
-    for (int kp = 0; kp < D / 2; ++kp) {
-        float c0 = 0.0f, c1 = 0.0f;
-#pragma unroll
-        for (int j = 0; j < D; ++j) {
-            c0 = fmaf(-s.Ainv[(2 * kp) * D + j], s.b[j], c0);
-            c1 = fmaf(-s.Ainv[(2 * kp + 1) * D + j], s.b[j], c1);
-        }
-        c2[kp] = make_float2(c0, c1);
-    }
-    {
-        int idx = 0;
-#pragma unroll
-        for (int i = 0; i < D; i += 2) {
-            qc.diag[i / 2] = s.M[i * D + i];
-            // row i gets 2*M[i][j] for j > i; row i+1 gets M[i+1][i+1] at j = i+1, 2*M[i+1][j] beyond
-#pragma unroll
-            for (int j = i + 1; j < D; ++j)
-                qc.pair[idx++] = make_float2(2.0f * s.M[i * D + j], (j == i + 1 ? 1.0f : 2.0f) * s.M[(i + 1) * D + j]);
-        }
-    }
+    load_encode_constants<D>(s.Ainv, s.M, s.b, hswap, Ai2, c2, qc);
 
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
-    constexpr int kGroupsPerThread = kPerThread / D;
-    constexpr int kThreads = 32 * kComputeWarps;
     float sq = 0.0f;
     int i = 0;
     for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++i) {
@@ -415,78 +504,132 @@ encode_kernel(EncodeArgs a) {
         if (!mbar_wait(&s.full[st], (i / kStages) & 1, a.status)) break;
         const int64_t base = c * kChunk;
         const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
-        const int ngroups = static_cast<int>(cnt / D);   // n % 8 == 0: whole groups
-#pragma unroll
-        for (int k = 0; k < kGroupsPerThread; ++k) {
-            const int g = t + k * kThreads;
-            if (g < ngroups) {
-                const float4 *src = reinterpret_cast<const float4 *>(s.buf[st] + g * D);
-                float w[D];
-                if (D == 8) {
-                    const float4 f0 = src[hswap], f1 = src[1 - hswap];
-                    w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
-                    w[4] = f1.x; w[5] = f1.y; w[6] = f1.z; w[7] = f1.w;
-                } else {
-                    const float4 f0 = src[0];
-                    w[0] = f0.x; w[1] = f0.y; w[2] = f0.z; w[3] = f0.w;
-                }
-                float u[D];
-                float gsq = 0.0f;
-                uint32_t p = 0;
-                encode_group<D, kMse>(w, Ai2, qc, c2, p, 0, u, gsq);
-                sq += gsq;
-                const int64_t gidx = base + static_cast<int64_t>(g) * D;   // flat index of the group's first weight
-                if (a.packed) {
-                    if (D == 8) *reinterpret_cast<uint16_t *>(a.packed + gidx / 4) = static_cast<uint16_t>(p);
-                    else a.packed[gidx / 4] = static_cast<uint8_t>(p);
-                }
-                if (a.codes) {
-                    uint32_t ww[D / 4];
-#pragma unroll
-                    for (int q = 0; q < D / 4; ++q) {
-                        const uint32_t f = (p >> (8 * q)) & 0xFFu;
-                        ww[q] = (f & 3u) | (((f >> 2) & 3u) << 8) | (((f >> 4) & 3u) << 16) | (((f >> 6) & 3u) << 24);
-                    }
-                    if (D == 8) *reinterpret_cast<uint2 *>(a.codes + gidx) = make_uint2(ww[0], ww[D / 4 - 1]);
-                    else *reinterpret_cast<uint32_t *>(a.codes + gidx) = ww[0];
-                }
-                if (kLatent) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.latent + gidx);
-#pragma unroll
-                    for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
-                }
-            }
-        }
+        encode_chunk<D, kMse>(s.buf[st], base, cnt, t, hswap, Ai2, qc, c2, a.packed, a.codes,
+                              kLatent ? a.latent : nullptr, sq);
         __syncwarp();
         if (lane == 0) mbar_arrive(&s.empty[st]);
     }
+    if (kMse) mse_flush(sq, s.dred, a.partials, a.counter, a.mse, total);
+}
 
-    if (kMse) {
-        for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-        if (lane == 0) s.dred[warp - 1] = static_cast<double>(sq);
-        compute_bar();
-        if (warp == 1) {
-            // per-CTA partial; the counter wraps to zero when the last CTA arrives (atomicInc), so it
-            // is back at zero for the next call without a reset
-            unsigned prev = 0;
-            if (lane == 0) {
-                double acc = 0.0;
-                for (int w = 0; w < kComputeWarps; ++w) acc += s.dred[w];
-                a.partials[blockIdx.x] = acc;
-                __threadfence();
-                prev = atomicInc(a.counter, gridDim.x - 1);
-            }
-            prev = __shfl_sync(0xffffffffu, prev, 0);
-            if (prev == gridDim.x - 1) {
-                // last CTA: the partials summed by the warp in a fixed order
-                __threadfence();
-                double tot = 0.0;
-                for (unsigned q = lane; q < gridDim.x; q += 32) tot += __ldcg(a.partials + q);
-                for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
-                if (lane == 0) *a.mse = total > 0 ? tot / static_cast<double>(total) : 0.0;
-            }
+// ------------------------------------------------------------------ batched encode (codes, latents)
+//
+// Several matrices (same d) in one persistent launch: their chunks form one list, streamed through
+// the ring in order; CTA b takes chunks b, b + G, ... of the list (G CTAs), so it visits the matrices in
+// order. Compute warp w forms A^{-1} of matrices w - 1, w - 1 + kComputeWarps, ... in parallel. Used
+// when no matrix asks for the MSE (see launch_encode_batch).
+
+struct InvSlot {
+    float A[64];
+    float Ainv[64];
+    float M[64];
+    float b[8];
+    float gjf[8][16];
+    double gj[8][16];
+    int singular;
+};
+
+struct EncBatchSmem {
+    float buf[kStages][kChunk];
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    InvSlot inv[kEncodeBatchMax];
+};
+
+__device__ __forceinline__ int batch_item_of(const EncodeBatchArgs &a, int64_t c, int from) {
+    int j = from;
+    while (j + 1 < a.count && c >= a.item[j + 1].chunk0) ++j;
+    return j;
+}
+
+// One matrix of a batched encode, for one CTA: its constants and its chunks (the sequence the
+// producer streams). Kept out of line so that its loop is compiled on its own (measured faster).
+template <int D, bool kLatent>
+__device__ __noinline__ void encode_batch_matrix(EncBatchSmem &s, const EncodeBatchArgs &a, int j, int &it, bool &ok) {
+    const int lane = threadIdx.x & 31;
+    const int t = threadIdx.x - 32;
+    const int hswap = (D == 8) ? ((t >> 2) & 1) : 0;
+    float2 Ai2[D / 2][D], c2[D / 2];
+    QuadCoef<D> qc;
+    float sq = 0.0f;
+    const int64_t chunk0 = a.item[j].chunk0, chunk1 = chunk0 + a.item[j].nchunks;
+    const int64_t total = a.item[j].m * a.item[j].n;
+    // this CTA's first chunk of matrix j: the first c >= chunk0 with c = blockIdx.x (mod gridDim.x)
+    const int64_t G = gridDim.x;
+    const int64_t first = chunk0 + ((static_cast<int64_t>(blockIdx.x) - chunk0) % G + G) % G;
+    if (first < chunk1) {
+        load_encode_constants<D>(s.inv[j].Ainv, s.inv[j].M, s.inv[j].b, hswap, Ai2, c2, qc);
+        uint8_t *const packed = a.item[j].packed;
+        uint8_t *const codes = a.item[j].codes;
+        float *const latent = kLatent ? a.item[j].latent : nullptr;
+        for (int64_t c = first; c < chunk1 && ok; c += G, ++it) {
+            const int st = it % kStages;
+            if (!mbar_wait(&s.full[st], (it / kStages) & 1, a.status)) { ok = false; break; }
+            const int64_t base = (c - chunk0) * kChunk;
+            const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
+            encode_chunk<D, false>(s.buf[st], base, cnt, t, hswap, Ai2, qc, c2, packed, codes, latent, sq);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.empty[st]);
         }
     }
+}
+
+template <int D, bool kLatent>
+__global__ void __launch_bounds__(kStreamThreads, 1)
+encode_batch_kernel(const __grid_constant__ EncodeBatchArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    EncBatchSmem &s = *reinterpret_cast<EncBatchSmem *>(smem_raw);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], kComputeWarps);
+        }
+        fence_barrier_init();
+    }
+    for (int e = threadIdx.x; e < a.count * (D * D + D); e += blockDim.x) {
+        const int j = e / (D * D + D), r = e % (D * D + D);
+        if (r < D * D) s.inv[j].A[r] = a.item[j].A[r];
+        else s.inv[j].b[r - D * D] = a.item[j].b[r - D * D];
+    }
+    __syncthreads();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int it = 0, j = -1;
+            int64_t next0 = 0, chunk0 = 0, total = 0;
+            const float *W = nullptr;
+            for (int64_t c = blockIdx.x; c < a.total_chunks; c += gridDim.x, ++it) {
+                if (c >= next0) {   // this chunk belongs to a later matrix: cache its fields
+                    j = batch_item_of(a, c, j < 0 ? 0 : j);
+                    chunk0 = a.item[j].chunk0;
+                    total = a.item[j].m * a.item[j].n;
+                    W = a.item[j].W;
+                    next0 = j + 1 < a.count ? a.item[j + 1].chunk0 : a.total_chunks;
+                }
+                const int st = it % kStages;
+                if (!mbar_wait(&s.empty[st], ((it / kStages) & 1) ^ 1, a.status)) return;
+                const int64_t base = (c - chunk0) * kChunk;
+                const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
+                const uint32_t bytes = static_cast<uint32_t>(cnt * 4);
+                mbar_arrive_expect_tx(&s.full[st], bytes);
+                bulk_g2s(s.buf[st], W + base, bytes, &s.full[st]);
+            }
+        }
+        return;
+    }
+    // compute warps: every matrix's A^{-1}, one matrix per warp at a time
+    for (int j = warp - 1; j < a.count; j += kComputeWarps) invert_warp<D>(s.inv[j]);
+    compute_bar();
+    if (blockIdx.x == 0 && threadIdx.x == 32) {
+        for (int j = 0; j < a.count; ++j)
+            if (s.inv[j].singular) set_status(a.status, LCQ_ERR_SINGULAR);
+    }
+
+    int it = 0;   // position in this CTA's chunk sequence (ring stage and phase), continued across matrices
+    bool ok = true;
+    for (int j = 0; j < a.count; ++j) encode_batch_matrix<D, kLatent>(s, a, j, it, ok);
 }
 
 // ------------------------------------------------------------------ quantize + decode (forward prologue)
@@ -789,6 +932,51 @@ cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t 
         k = mse ? (lat ? encode_kernel<8, true, true> : encode_kernel<8, true, false>)
                 : (lat ? encode_kernel<8, false, true> : encode_kernel<8, false, false>);
     }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    trace_begin(LCQ_K_ENCODE, st);
+    k<<<grid, kStreamThreads, smem, st>>>(a);
+    trace_end(LCQ_K_ENCODE, st);
+    count_launch();
+    return cudaGetLastError();
+}
+
+int64_t encode_chunk_size() { return kChunk; }
+
+cudaError_t launch_encode_batch(const EncodeBatchArgs &a, int d, int num_sms, cudaStream_t st) {
+    bool mse = false, lat = false;
+    for (int i = 0; i < a.count; ++i) {
+        mse = mse || a.item[i].mse != nullptr;
+        lat = lat || a.item[i].latent != nullptr;
+    }
+    if (mse) {
+        // With the reconstruction MSE, the single-matrix kernel measured faster per matrix than the
+        // fused batch kernel (whose MSE variant compiles to ~25% more instructions per group), so each
+        // matrix gets its own launch, with its own partials and counter in the batch workspace.
+        for (int i = 0; i < a.count; ++i) {
+            const EncodeBatchItem &it = a.item[i];
+            if (it.m * it.n == 0) {
+                if (it.mse) {
+                    const cudaError_t e = cudaMemsetAsync(it.mse, 0, sizeof(double), st);
+                    if (e != cudaSuccess) return e;
+                }
+                continue;
+            }
+            EncodeArgs e;
+            e.W = it.W; e.m = it.m; e.n = it.n; e.A = it.A; e.b = it.b;
+            e.packed = it.packed; e.codes = it.codes; e.latent = it.latent; e.mse = it.mse;
+            e.partials = a.partials + static_cast<int64_t>(i) * kEncodeBatchPartials;
+            e.counter = a.counters + i;
+            e.status = a.status;
+            const cudaError_t r = launch_encode(e, d, num_sms, st);
+            if (r != cudaSuccess) return r;
+        }
+        return cudaSuccess;
+    }
+    const int grid = static_cast<int>(a.total_chunks < num_sms ? (a.total_chunks > 0 ? a.total_chunks : 1) : num_sms);
+    const size_t smem = sizeof(EncBatchSmem);
+    void (*k)(const EncodeBatchArgs) = d == 4 ? (lat ? encode_batch_kernel<4, true> : encode_batch_kernel<4, false>)
+                                              : (lat ? encode_batch_kernel<8, true> : encode_batch_kernel<8, false>);
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     trace_begin(LCQ_K_ENCODE, st);

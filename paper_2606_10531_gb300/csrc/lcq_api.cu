@@ -98,7 +98,10 @@ constexpr int kMaxGemmCtas = 1024;        // upper bound on the persistent GEMM 
 struct Header {
     int32_t status;
     uint32_t counter;
+    uint32_t pad[14];
+    uint32_t batch_counters[kEncodeBatchMax];   // lcq_encode_batch, one per matrix
 };
+static_assert(sizeof(Header) <= kHeader, "workspace header");
 
 static lcq_status check_common(int64_t m, int64_t n, int d) {
     if (d != 4 && d != 8) return LCQ_ERR_UNSUPPORTED;
@@ -170,6 +173,9 @@ size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d) {
     switch (op) {
         case LCQ_OP_ENCODE:
             return kHeader + align256(sizeof(double) * 2 * 1024);
+        case LCQ_OP_ENCODE_BATCH:
+            if (N < 1 || N > kEncodeBatchMax) return 0;
+            return kHeader + align256(sizeof(double) * kEncodeBatchPartials * static_cast<size_t>(N));
         case LCQ_OP_LINEAR_FWD:
             return kHeader + align256(mn * 2);
         case LCQ_OP_LINEAR_BWD:
@@ -339,6 +345,48 @@ lcq_status lcq_encode(const float *W, int64_t m, int64_t n, int d, const float *
     a.counter = &h->counter;
     a.status = &h->status;
     return cuda_status(launch_encode(a, d, num_sms_current(), st));
+}
+
+lcq_status lcq_encode_batch(const lcq_encode_item *items, int count, int d, void *ws, size_t ws_bytes, void *stream) {
+    if (!items) return LCQ_ERR_NULL;
+    if (count < 1 || count > kEncodeBatchMax) return LCQ_ERR_SHAPE;
+    if (d != 4 && d != 8) return LCQ_ERR_UNSUPPORTED;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_ENCODE_BATCH, count, 0, 0, d)));
+    EncodeBatchArgs a;
+    std::memset(&a, 0, sizeof(a));
+    const int64_t chunk = encode_chunk_size();
+    int64_t c0 = 0;
+    for (int i = 0; i < count; ++i) {
+        const lcq_encode_item &it = items[i];
+        LCQ_TRY(check_common(it.m, it.n, d));
+        const int64_t mn = it.m * it.n;
+        LCQ_TRY(check_tensor(it.W, mn));
+        if (!it.A || !it.b) return LCQ_ERR_NULL;
+        LCQ_TRY(check_tensor(it.packed, mn, false));
+        LCQ_TRY(check_tensor(it.codes, mn, false));
+        LCQ_TRY(check_tensor(it.latent, mn, false));
+        if (it.mse && (reinterpret_cast<uintptr_t>(it.mse) & 7u)) return LCQ_ERR_ALIGN;
+        EncodeBatchItem &e = a.item[i];
+        e.W = it.W; e.m = it.m; e.n = it.n; e.A = it.A; e.b = it.b;
+        e.packed = it.packed; e.codes = it.codes; e.latent = it.latent; e.mse = it.mse;
+        e.chunk0 = c0;
+        e.nchunks = (mn + chunk - 1) / chunk;
+        c0 += e.nchunks;
+    }
+    a.count = count;
+    a.total_chunks = c0;
+    cudaStream_t st = as_stream(stream);
+    if (c0 == 0) {
+        // every matrix is empty: the MSE of an empty matrix is 0
+        for (int i = 0; i < count; ++i)
+            if (items[i].mse) LCQ_TRY(cuda_status(cudaMemsetAsync(items[i].mse, 0, sizeof(double), st)));
+        return LCQ_OK;
+    }
+    Header *h = static_cast<Header *>(ws);
+    a.partials = reinterpret_cast<double *>(static_cast<uint8_t *>(ws) + kHeader);
+    a.counters = h->batch_counters;
+    a.status = &h->status;
+    return cuda_status(launch_encode_batch(a, d, num_sms_current(), st));
 }
 
 lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const float *A, const float *b,

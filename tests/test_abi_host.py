@@ -112,3 +112,28 @@ def test_empty_problems_need_no_device(L):
     # nothing to do: returns before touching CUDA
     assert L.lcq_decode(None, 0, 16, 8, FAKE, FAKE, None, None, None) == OK
     assert L.lcq_pack2b(None, 0, 16, None, None) == OK
+
+
+def test_encode_batch_validation(L):
+    ws_ok = FAKE
+    big = 1 << 30
+    items = (lcq.lcq_encode_item * 2)()
+    for k in range(2):
+        items[k] = lcq.lcq_encode_item(FAKE, 8, 16, FAKE, FAKE, FAKE, None, None, None)
+    eb = lambda arr=items, count=2, d=4, ws=ws_ok, ws_bytes=big: L.lcq_encode_batch(arr, count, d, ws, ws_bytes, None)  # noqa: E731
+    assert eb(arr=None) == NULL
+    assert eb(count=0) == SHAPE
+    assert eb(count=17) == SHAPE
+    assert eb(d=5) == UNSUP
+    assert eb(ws_bytes=16) == WS
+    bad = (lcq.lcq_encode_item * 2)()
+    bad[0] = lcq.lcq_encode_item(FAKE, 8, 16, FAKE, FAKE, FAKE, None, None, None)
+    bad[1] = lcq.lcq_encode_item(FAKE, 8, 12, FAKE, FAKE, FAKE, None, None, None)     # n % 8 != 0
+    assert eb(arr=bad) == SHAPE
+    bad[1] = lcq.lcq_encode_item(FAKE, 8, 16, None, FAKE, FAKE, None, None, None)     # A missing
+    assert eb(arr=bad) == NULL
+    bad[1] = lcq.lcq_encode_item(FAKE + 4, 8, 16, FAKE, FAKE, FAKE, None, None, None)  # W misaligned
+    assert eb(arr=bad) == ALIGN
+    assert L.lcq_workspace_size(6, 0, 0, 0, 8) == 0
+    assert L.lcq_workspace_size(6, 17, 0, 0, 8) == 0
+    assert 0 < L.lcq_workspace_size(6, 1, 0, 0, 8) < L.lcq_workspace_size(6, 7, 0, 0, 8)

@@ -104,6 +104,53 @@ def test_encode_inverse_accuracy_ill_conditioned(d, cond):
         assert np.all(np.abs(got[r].T - inv) <= tol), f"max err/tol {np.max(np.abs(got[r].T - inv) / tol)}"
 
 
+@pytest.mark.parametrize("d", [4, 8])
+def test_encode_batch_matches_single_calls_and_oracle(d):
+    # the batch gives, matrix by matrix, exactly what lcq_encode gives; and both match the oracle
+    torch = T()
+    rng = np.random.default_rng(77 + d)
+    shapes = [(512, 512), (37, 24), (129, 4104), (0, 64), (300, 1000), (64, 8), (700, 2048), (5, 40),
+              (1024, 512), (33, 96), (16, 16), (250, 1024)]      # 12 matrices: some warps invert two
+    items, singles, refs = [], [], []
+    for k, (m, n) in enumerate(shapes):
+        W = rng.normal(0, 0.02, (m, n)).astype(np.float32)
+        A, b = config_A(d, rng), config_b(d, rng)
+        it = {"W": dev(W), "A": dev(A), "b": dev(b),
+              "packed": torch.empty((m, n // 4), dtype=torch.uint8, device="cuda"),
+              "codes": torch.empty((m, n), dtype=torch.uint8, device="cuda") if k % 2 == 0 else None,
+              "latent": torch.empty((m, n), dtype=torch.float32, device="cuda") if k % 3 == 0 else None,
+              "mse": torch.full((1,), -1.0, dtype=torch.float64, device="cuda") if k != 5 else None}
+        items.append(it)
+        one = {kk: (torch.empty_like(v) if kk in ("packed", "codes", "latent", "mse") and v is not None else v)
+               for kk, v in it.items()}
+        singles.append(one)
+        refs.append((W, A, b))
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE_BATCH, len(items), 0, 0, d)
+    for _ in range(2):                    # twice: the per-matrix counters must come back to zero
+        lcq.lcq_encode_batch(items, d, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    for it, one, (W, A, b) in zip(items, singles, refs):
+        m, n = W.shape
+        ws1 = lcq.workspace(lcq.LCQ_OP_ENCODE, 0, m, n, d)
+        lcq.lcq_encode(one["W"], one["A"], one["b"], d, ws1, packed=one["packed"], codes=one["codes"],
+                       latent=one["latent"], mse=one["mse"])
+        for key in ("packed", "codes", "latent"):
+            if it[key] is not None:
+                assert torch.equal(it[key], one[key]), key
+        if it["mse"] is not None:
+            assert it["mse"].item() == one["mse"].item()
+        if m * n == 0:
+            if it["mse"] is not None:
+                assert it["mse"].item() == 0.0
+            continue
+        ref = oracle.encode(W, A, b, d)
+        z = oracle.unpack2b(it["packed"].cpu().numpy(), n)
+        keep = ~ref["near"]
+        assert int(np.sum((z != ref["codes"]) & keep)) == 0
+        if it["mse"] is not None:
+            assert abs(it["mse"].item() - ref["mse"]) <= 1e-4 * ref["mse"] + 1e-12
+
+
 def test_encode_nonfinite_inputs():
     torch = T()
     d, m, n = 8, 4, 32
