@@ -10,6 +10,6 @@ finite differences, hand-worked fixtures in tests/golden/).
 """
 from .lcvq import (BITS, DGE_GRAD_MAX, DGE_K, ZMAX, SingularMatrix, brute_nearest, decode, dge_f,  # noqa: F401
                    dge_fprime, dge_grad, encode, gemm_packed2b, gemm_packed2b_hadamard, hadamard_block,
-                   hadamard_rotate, init_latent,
+                   hadamard_rotate, init_latent, ldl_block, ldlq, ldlq_latent_given_codes, proxy_loss,
                    init_codebook, inverse, latent, linear_bwd, linear_fwd, mse, near_boundary,
                    pack2b, quantize, round_clamp, unpack2b)

@@ -18,6 +18,9 @@ inverse) with no blocking, fusion or reordering:
   * forward             Y = X W_hat^T (nn.Linear orientation)   (Sec. 3.2, Eq. def:forward_x)
   * backward            exact gradients of the linear map, with the
                         straight-through estimator dW_z/dW_p = 1 (Sec. 3.3)
+  * LDLQ initialisation column groups quantized in order, each target
+                        corrected by the earlier groups' errors through the
+                        block U D U^T factor of the proxy Hessian (Sec. 2.2)
 
 Readings where the paper is silent or inconsistent (listed in the design doc):
   * encode maps a real weight group to latent coordinates u = A^{-1}(w - B)
@@ -30,6 +33,9 @@ Readings where the paper is silent or inconsistent (listed in the design doc):
     which the integer decision is taken on both sides): fl(fl(P*fl(1/s)) + t);
   * packed storage: 4 codes per byte, column c in bits 2(c mod 4)..+1 of
     byte floor(c/4), least significant first.
+  * LDLQ (Sec. 2.2 names the algorithm, QuIP, and gives no formula): the
+    block form with d x d blocks, the LC-VQ rounding encoder as the group
+    quantizer, and errors W - W_hat measured against the original weights.
 """
 from __future__ import annotations
 
@@ -292,3 +298,92 @@ def brute_nearest(W, A, b, d: int):
     """
     from . import _native
     return _native.brute_nearest(W, A, b, d)
+
+
+# ----------------------------------------------------------------------------- LDLQ initialisation
+#
+# Sec. 2.2 initialises the codes with LDLQ (QuIP, Chee et al. 2023): the column groups of W are
+# quantized one after another, and each group's target is its own weights plus the accumulated
+# reconstruction error of the groups before it, fed forward through the factor of the proxy
+# Hessian H. With groups of d columns (the block form used for vector quantizers, QuIP#):
+#
+#     H = (U + I) D (U + I)^T      U strictly upper block-triangular (d x d blocks), D block diagonal
+#     T_k = W_k + sum_{j<k} (W_j - W_hat_j) U_{j,k}            (target of column group k)
+#     z_k = clip(round(A^{-1}(T_k - B)), 0, 3),  W_hat_k = A z_k + B   (the LC-VQ rounding encoder)
+#
+# With U = 0 (H block diagonal) this is the plain encoder. The reconstruction error of the result
+# satisfies (W_hat - W)(U + I) = eta, eta_k = W_hat_k - T_k, so the proxy loss
+# tr((W_hat - W) H (W_hat - W)^T) equals sum_k sum_r eta_{r,k} D_k eta_{r,k}^T.
+
+def ldl_block(H, d: int):
+    """Block U D U^T factorisation H = (U + I) D (U + I)^T of a symmetric positive definite matrix
+    (the factorisation LDLQ feeds its errors through; Sec. 2.2, LDLQ).
+
+    Eliminates the d x d blocks from the last to the first: D_k is the current Schur-complement
+    block, the column block above it is U_{<k,k} = S_{<k,k} D_k^{-1}, and the leading blocks are
+    replaced by their Schur complement S_{<k,<k} - S_{<k,k} D_k^{-1} S_{k,<k}.
+    Returns U (n x n fp64, zero on and below the block diagonal) and D (G x d x d fp64).
+    """
+    S = _f64(H).copy()
+    n = S.shape[0]
+    if S.shape != (n, n) or n % d:
+        raise ValueError("H must be n x n with n a multiple of d")
+    G = n // d
+    U = np.zeros((n, n))
+    D = np.zeros((G, d, d))
+    for k in reversed(range(G)):
+        blk = slice(k * d, (k + 1) * d)
+        D[k] = S[blk, blk]
+        if k == 0:
+            break
+        lead = slice(0, k * d)
+        Uk = S[lead, blk] @ np.linalg.inv(D[k])
+        U[lead, blk] = Uk
+        S[lead, lead] -= Uk @ S[blk, lead]
+    return U, D
+
+
+def ldlq(W, U, A, b, d: int) -> dict:
+    """LDLQ sweep with the LC-VQ rounding encoder as the group quantizer (Sec. 2.2, LDLQ):
+    column groups k = 0 .. G-1 in order, target T_k = W_k + sum_{j<k} (W_j - W_hat_j) U_{j,k}.
+
+    U is the strictly upper block factor of ldl_block. Returns the codes (uint8 m x n), the latent
+    coordinates of the targets u = A^{-1}(T - B) (fp64, for the near-boundary mask), the targets T,
+    the reconstruction MSE mean((W - W_hat)^2) and W_hat.
+    """
+    W64, U64, A64, b64 = _f64(W), _f64(U), _f64(A), _f64(b)
+    m, n = W64.shape
+    if n % d:
+        raise ValueError(f"n={n} is not a multiple of the group size d={d}")
+    Ainv = inverse(A)
+    What = np.zeros((m, n))
+    T = np.zeros((m, n))
+    Ulat = np.zeros((m, n))
+    Z = np.zeros((m, n), dtype=np.uint8)
+    for k in range(n // d):
+        blk = slice(k * d, (k + 1) * d)
+        Tk = W64[:, blk] + (W64[:, :k * d] - What[:, :k * d]) @ U64[:k * d, blk]
+        uk = (Tk - b64) @ Ainv.T                  # row-vector form of A^{-1} (T_k - B)
+        zk = round_clamp(uk)
+        Z[:, blk] = zk
+        What[:, blk] = zk.astype(np.float64) @ A64.T + b64
+        T[:, blk] = Tk
+        Ulat[:, blk] = uk
+    return {"codes": Z, "latent": Ulat, "near": near_boundary(Ulat), "target": T, "W_hat": What,
+            "mse": float(np.mean((W64 - What) ** 2)) if W64.size else 0.0}
+
+
+def ldlq_latent_given_codes(W, Z, U, A, b, d: int) -> np.ndarray:
+    """Latent coordinates A^{-1}(T_k - B) of every LDLQ target when the earlier groups were decided
+    as Z (Sec. 2.2, LDLQ): T = W + (W - decode(Z)) U with U strictly upper block-triangular, so
+    T_k only sees groups j < k. A valid LDLQ result satisfies round_clamp(latent) == Z."""
+    W64 = _f64(W)
+    m, n = W64.shape
+    T = W64 + (W64 - decode(Z, A, b, d)) @ _f64(U)
+    return ((_grouped(T, d) - _f64(b)) @ inverse(A).T).reshape(m, n)
+
+
+def proxy_loss(W, W_hat, H) -> float:
+    """tr((W_hat - W) H (W_hat - W)^T), the layer-output error LDLQ minimises for E[x x^T] = H."""
+    E = _f64(W_hat) - _f64(W)
+    return float(np.einsum("ri,ij,rj->", E, _f64(H), E))

@@ -16,7 +16,13 @@ Distributions (std, not variance, in every N(0, s)):
   * A = 0.01 I + N(0, 1e-3) (d x d), b ~ N(0, 1e-3) (d);
   * X, dY ~ N(0, 1) rounded to bf16; the 7B-projection workload scales
     round(0.01 n) seeded input channels of X by 20 (activation outliers);
-  * packed deployment codes: uniform random bytes (4 uniform codes each).
+  * packed deployment codes: uniform random bytes (4 uniform codes each);
+  * proxy Hessian for LDLQ (stands in for the calibration statistics E[x x^T] of
+    1,024 RedPajama samples, which are absent): H0 = S (K/2 + V V^T/(2r)) S with
+    K_ij = 0.9^|i-j| (neighbouring-channel correlation), V ~ N(0,1) of rank r = 8
+    (a few dominant activation directions) and S = diag(1, with round(0.01 n)
+    seeded outlier channels scaled by 20); H = H0 + 0.01 mean(diag H0) I (1%
+    dampening), rounded to fp32.
 """
 from __future__ import annotations
 
@@ -24,7 +30,7 @@ import dataclasses
 
 import numpy as np
 
-PARTS = {"W": 0, "A": 1, "b": 2, "X": 3, "dY": 4, "codes": 5, "outliers": 6}
+PARTS = {"W": 0, "A": 1, "b": 2, "X": 3, "dY": 4, "codes": 5, "outliers": 6, "hessian": 7}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -69,6 +75,19 @@ def llama3_70b_layer_encode(d: int = 8):
     h, kv, f = 8192, 1024, 28672
     shapes = [("q", h, h), ("k", kv, h), ("v", kv, h), ("o", h, h), ("gate", f, h), ("up", f, h), ("down", h, f)]
     return [Matrix(nm, m, n, d, 0, w_std=0.015, heavy_tail=True) for nm, m, n in shapes]
+
+
+def llama3_70b_gate_ldlq(d: int = 8):
+    """LDLQ initialisation of the Llama-3-70B gate projection 28672x8192 (heavy-tailed fp32 weights)."""
+    return [Matrix("gate70b", 28672, 8192, d, 0, w_std=0.015, heavy_tail=True)]
+
+
+def llama3_8b_gate_ldlq(d: int = 8):
+    """LDLQ initialisation of the Llama-3-8B gate projection 14336x4096 (heavy-tailed fp32 weights)."""
+    return [Matrix("gate8b", 14336, 4096, d, 0, w_std=0.015, heavy_tail=True)]
+
+
+HESSIAN_RHO, HESSIAN_RANK, HESSIAN_DAMP = 0.9, 8, 0.01
 
 
 # ----------------------------------------------------------------------------- NumPy draws
@@ -133,6 +152,19 @@ def draw_packed_codes(mx: Matrix, seed: int, index: int) -> np.ndarray:
     return rng.integers(0, 256, size=(mx.m, mx.n // 4), dtype=np.uint8)
 
 
+def draw_hessian(n: int, seed: int, index: int) -> np.ndarray:
+    """Synthetic symmetric positive definite proxy Hessian [n][n] fp32 (recipe in the module doc)."""
+    rng = _rng(seed, index, "hessian")
+    V = rng.standard_normal((n, HESSIAN_RANK))
+    s = np.ones(n)
+    s[rng.choice(n, size=int(round(0.01 * n)), replace=False)] = 20.0
+    i = np.arange(n)
+    K = HESSIAN_RHO ** np.abs(i[:, None] - i[None, :]).astype(np.float64)
+    H0 = s[:, None] * (0.5 * K + (0.5 / HESSIAN_RANK) * (V @ V.T)) * s[None, :]
+    H = H0 + HESSIAN_DAMP * np.mean(np.diag(H0)) * np.eye(n)
+    return H.astype(np.float32)
+
+
 # ----------------------------------------------------------------------------- device draws
 
 def _torch_gen(torch, device, seed: int, index: int, part: str):
@@ -184,3 +216,17 @@ def torch_dY(torch, mx: Matrix, seed: int, index: int, device, tokens: int | Non
 def torch_packed_codes(torch, mx: Matrix, seed: int, index: int, device):
     g = _torch_gen(torch, device, seed, index, "codes")
     return torch.randint(0, 256, (mx.m, mx.n // 4), generator=g, device=device, dtype=torch.int32).to(torch.uint8)
+
+
+def torch_hessian(torch, n: int, seed: int, index: int, device):
+    """Device draw of the synthetic proxy Hessian (same recipe as draw_hessian, torch generator)."""
+    g = _torch_gen(torch, device, seed, index, "hessian")
+    V = torch.randn((n, HESSIAN_RANK), generator=g, device=device, dtype=torch.float32)
+    s = torch.ones(n, device=device, dtype=torch.float32)
+    s[torch.randperm(n, generator=g, device=device)[:int(round(0.01 * n))]] = 20.0
+    i = torch.arange(n, device=device, dtype=torch.float32)
+    H = torch.pow(torch.tensor(HESSIAN_RHO, device=device), (i[:, None] - i[None, :]).abs())
+    H.mul_(0.5).addmm_(V, V.t(), alpha=0.5 / HESSIAN_RANK)
+    H.mul_(s[:, None]).mul_(s[None, :])
+    H.diagonal().add_(HESSIAN_DAMP * H.diagonal().mean())
+    return H

@@ -386,3 +386,156 @@ def test_rotation_cancels_through_the_product():
     X = RNG.normal(size=(2, n))
     np.testing.assert_allclose(oracle.gemm_packed2b_hadamard(oracle.hadamard_rotate(X, n), oracle.pack2b(Z), A, b, d, n),
                                oracle.gemm_packed2b(X, oracle.pack2b(Z), A, b, d, n), rtol=1e-12, atol=1e-14)
+
+
+# ----------------------------------------------------------------------------- LDLQ initialisation
+
+def _ar1(n, rho):
+    i = np.arange(n)
+    return rho ** np.abs(i[:, None] - i[None, :]).astype(np.float64)
+
+
+def test_ldl_block_of_ar1_correlation_is_its_closed_form():
+    """H_ij = rho^|i-j| (a stationary AR(1) covariance). Running the process backwards,
+    x_i = rho x_{i+1} + sqrt(1 - rho^2) e_i, gives the scalar factor M_ij = rho^(j-i) (j >= i),
+    D = diag(1 - rho^2, ..., 1 - rho^2, 1). The d-block factor is M B^-1, B D B^T with
+    B = blockdiag(M_kk); by the Markov property only the first column of each off-diagonal
+    block of U is non-zero: U[r, kd] = rho^(kd - r)."""
+    rho, n = 0.7, 24
+    H = _ar1(n, rho)
+    U1, D1 = oracle.ldl_block(H, 1)
+    i = np.arange(n)
+    want_U1 = np.where(i[None, :] > i[:, None], rho ** (i[None, :] - i[:, None]).astype(float), 0.0)
+    assert np.allclose(U1, want_U1, rtol=0, atol=1e-13)
+    want_D1 = np.full(n, 1 - rho * rho)
+    want_D1[-1] = 1.0
+    assert np.allclose(D1[:, 0, 0], want_D1, rtol=0, atol=1e-13)
+    for d in (4, 8):
+        U, D = oracle.ldl_block(H, d)
+        want_U = np.zeros((n, n))
+        for k in range(1, n // d):
+            want_U[:k * d, k * d] = rho ** (k * d - np.arange(k * d)).astype(float)
+        assert np.allclose(U, want_U, rtol=0, atol=1e-13)
+        for k in range(n // d):
+            Mkk = np.triu(rho ** np.abs(np.subtract.outer(np.arange(d), np.arange(d))).astype(float))
+            Dk = np.diag(want_D1[k * d:(k + 1) * d])
+            assert np.allclose(D[k], Mkk @ Dk @ Mkk.T, rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_ldl_block_reconstructs_spd_matrices(d):
+    from paper_2606_10531_gb300 import workloads as wl
+    rng = np.random.default_rng(7)
+    Q = rng.normal(size=(64, 64))
+    for H in (Q @ Q.T + 0.5 * np.eye(64), wl.draw_hessian(64, 0, 3).astype(np.float64)):
+        U, D = oracle.ldl_block(H, d)
+        n = H.shape[0]
+        blk = np.arange(n) // d
+        assert np.all(U[blk[:, None] >= blk[None, :]] == 0.0)       # strictly upper block-triangular
+        Dfull = np.zeros((n, n))
+        for k in range(n // d):
+            assert np.allclose(D[k], D[k].T, rtol=0, atol=1e-12 * np.abs(D[k]).max())
+            assert np.linalg.eigvalsh(D[k]).min() > 0
+            Dfull[k * d:(k + 1) * d, k * d:(k + 1) * d] = D[k]
+        M = U + np.eye(n)
+        assert np.allclose(M @ Dfull @ M.T, H, rtol=0, atol=1e-11 * np.abs(H).max())
+
+
+def _ldlq_case(m, n, d, seed, H=None):
+    from paper_2606_10531_gb300 import workloads as wl
+    rng = np.random.default_rng(seed)
+    W = rng.normal(0.0, 0.015, (m, n))
+    A = config_like_A(d, rng)
+    b = rng.normal(0.0, 1e-3, d)
+    if H is None:
+        H = wl.draw_hessian(n, seed, 0).astype(np.float64)
+    return W, A, b, H
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_ldlq_with_block_diagonal_hessian_is_the_rounding_encoder(d):
+    """No correlation between column groups: U = 0, no feedback, LDLQ = plain rounding."""
+    rng = np.random.default_rng(11)
+    n = 8 * d
+    H = np.zeros((n, n))
+    for k in range(n // d):
+        Q = rng.normal(size=(d, d))
+        H[k * d:(k + 1) * d, k * d:(k + 1) * d] = Q @ Q.T + np.eye(d)
+    W, A, b, _ = _ldlq_case(16, n, d, 5, H)
+    U, _ = oracle.ldl_block(H, d)
+    assert np.all(U == 0.0)
+    r = oracle.ldlq(W, U, A, b, d)
+    e = oracle.encode(W, A, b, d)
+    assert np.array_equal(r["codes"], e["codes"])
+    assert r["mse"] == pytest.approx(e["mse"], rel=1e-12)
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_ldlq_equals_the_optq_schur_complement_form(d):
+    """QuIP shows LDLQ equals OPTQ: after the groups before k are fixed, the remaining columns are
+    completed optimally, W_R - (W_hat_Q - W_Q) H_QR H_RR^-1, and group k is rounded from that.
+    Computed here from H by linear solves, independently of the factorisation."""
+    W, A, b, H = _ldlq_case(12, 8 * d, d, 21)
+    m, n = W.shape
+    Ainv = np.linalg.inv(A)
+    What = np.zeros((m, n))
+    Z = np.zeros((m, n), dtype=np.uint8)
+    T = np.zeros((m, n))
+    for k in range(n // d):
+        q, r = slice(0, k * d), slice(k * d, n)
+        TR = W[:, r] - (What[:, q] - W[:, q]) @ np.linalg.solve(H[r, r], H[q, r].T).T
+        Tk = TR[:, :d]
+        z = np.clip(np.rint((Tk - b) @ Ainv.T), 0, 3)
+        Z[:, k * d:(k + 1) * d] = z
+        What[:, k * d:(k + 1) * d] = z @ A.T + b
+        T[:, k * d:(k + 1) * d] = Tk
+    U, _ = oracle.ldl_block(H, d)
+    res = oracle.ldlq(W, U, A, b, d)
+    assert np.abs(res["target"] - T).max() < 1e-12
+    assert np.array_equal(res["codes"], Z)
+    assert not res["near"].any()
+
+
+@pytest.mark.parametrize("d", [4, 8])
+def test_ldlq_proxy_loss_is_the_d_weighted_sum_of_rounding_errors(d):
+    """(W_hat - W)(U + I) = eta with eta_k = W_hat_k - T_k, so
+    tr((W_hat - W) H (W_hat - W)^T) = sum_{r,k} eta_{r,k} D_k eta_{r,k}^T."""
+    W, A, b, H = _ldlq_case(20, 16 * d, d, 31)
+    U, D = oracle.ldl_block(H, d)
+    res = oracle.ldlq(W, U, A, b, d)
+    eta = (res["W_hat"] - res["target"]).reshape(W.shape[0], -1, d)
+    rhs = float(np.einsum("rkj,kji,rki->", eta, D, eta))
+    assert oracle.proxy_loss(W, res["W_hat"], H) == pytest.approx(rhs, rel=1e-9)
+
+
+def test_ldlq_given_codes_reproduces_the_sweep_targets():
+    W, A, b, H = _ldlq_case(24, 64, 8, 41)
+    U, _ = oracle.ldl_block(H, 8)
+    res = oracle.ldlq(W, U, A, b, 8)
+    lat = oracle.ldlq_latent_given_codes(W, res["codes"], U, A, b, 8)
+    assert np.abs(lat - res["latent"]).max() < 1e-10
+    assert np.array_equal(oracle.round_clamp(lat), res["codes"])
+
+
+def test_ldlq_keeps_codewords_fixed():
+    """A matrix that is itself decoded codewords has zero error at every step: LDLQ returns its codes."""
+    rng = np.random.default_rng(3)
+    d = 8
+    A = config_like_A(d, rng)
+    b = rng.normal(0.0, 1e-3, d)
+    Z0 = rng.integers(0, 4, (10, 64)).astype(np.uint8)
+    W = oracle.decode(Z0, A, b, d)
+    _, _, _, H = _ldlq_case(1, 64, d, 2)
+    U, _ = oracle.ldl_block(H, d)
+    assert np.array_equal(oracle.ldlq(W, U, A, b, d)["codes"], Z0)
+
+
+def test_ldlq_lowers_the_proxy_loss_against_plain_rounding():
+    """The feedback is what LDLQ adds: on a correlated Hessian its proxy loss is below that of
+    rounding every group on its own (seeded instance)."""
+    d = 8
+    W, A, b, H = _ldlq_case(64, 256, d, 51)
+    U, _ = oracle.ldl_block(H, d)
+    res = oracle.ldlq(W, U, A, b, d)
+    plain = oracle.decode(oracle.encode(W, A, b, d)["codes"], A, b, d)
+    assert oracle.proxy_loss(W, res["W_hat"], H) < 0.9 * oracle.proxy_loss(W, plain, H)
