@@ -51,7 +51,7 @@ typedef enum lcq_status {
     LCQ_ERR_UNSUPPORTED = 4, /* d not in {4, 8}, unknown STE mode                       */
     LCQ_ERR_WORKSPACE = 5,   /* workspace NULL or smaller than lcq_workspace_size()     */
     LCQ_ERR_CUDA = 6,        /* a CUDA runtime call or kernel launch failed             */
-    LCQ_ERR_SINGULAR = 7,    /* device-detected: A is not invertible (encode)           */
+    LCQ_ERR_SINGULAR = 7,    /* device-detected: A (or a block of D, LDLQ) not invertible */
     LCQ_ERR_TIMEOUT = 8,     /* device-detected: a bounded pipeline wait gave up        */
     LCQ_ERR_ARG = 9,         /* any other invalid argument (e.g. latent_scale == 0)     */
     LCQ_ERR_LIMIT = 10       /* problem larger than the static scratch of a _noalloc call */
@@ -64,7 +64,9 @@ typedef enum lcq_op {
     LCQ_OP_LINEAR_BWD = 3,
     LCQ_OP_GEMM_PACKED2B = 4,
     LCQ_OP_GEMM_PACKED2B_HADAMARD = 5,
-    LCQ_OP_ENCODE_BATCH = 6          /* N = number of matrices; m, n unused */
+    LCQ_OP_ENCODE_BATCH = 6,         /* N = number of matrices; m, n unused */
+    LCQ_OP_LDL_FACTOR = 7,           /* n, d; N, m unused */
+    LCQ_OP_LDLQ = 8                  /* m, n, d; N unused */
 } lcq_op;
 
 /* Gradient estimators for dP through the rounding (Sec. 3.3). */
@@ -148,6 +150,45 @@ typedef struct lcq_encode_item {
  */
 lcq_status lcq_encode_batch(const lcq_encode_item *items, int count, int d, void *ws, size_t ws_bytes,
                             void *stream);
+
+/*
+ * lcq_ldl_factor - block U D U^T factorisation of a proxy Hessian, the factor LDLQ feeds its errors
+ * through (Sec. 2.2 initialises the codes with LDLQ):
+ *
+ *     H = (U + I) D (U + I)^T
+ *
+ * U is strictly upper block-triangular in d x d blocks (zero on and below the block diagonal), D is
+ * block diagonal. The blocks are eliminated from the last to the first in 128-column panels, in fp32.
+ *
+ * H  [n][n] fp32, symmetric positive definite; only its upper triangle (i <= j) is read.
+ * U  [n][n] fp32 output; every element is written.
+ * D  [n/d][d][d] fp32 output (block k is D_k), or NULL.
+ * If a block D_k is singular (H not positive definite) the status word becomes LCQ_ERR_SINGULAR.
+ * Needs lcq_workspace_size(LCQ_OP_LDL_FACTOR, 0, 0, n, d) bytes of ws (a copy of H, about 4 n^2 bytes).
+ */
+lcq_status lcq_ldl_factor(const float *H, int64_t n, int d, float *U, float *D, void *ws, size_t ws_bytes,
+                          void *stream);
+
+/*
+ * lcq_ldlq - LDLQ initialisation of the codes (Sec. 2.2): the column groups k = 0, 1, ... of W are
+ * rounded in order by the LC-VQ encoder, each from a target that carries the earlier groups' errors
+ * forward through the factor U of lcq_ldl_factor (rows are independent):
+ *
+ *     T_k = W_k + sum_{j<k} (W_j - W_hat_j) U_{j,k},    z_k = clip(round_half_even(A^{-1}(T_k - b)), 0, 3),
+ *     W_hat_k = A z_k + b                               (W_k: the d columns of group k)
+ *
+ * W       [m][n] fp32 input.
+ * U       [n][n] fp32; only the entries above the block diagonal are read.
+ * packed  [m][n/4] uint8 output, or NULL.
+ * codes   [m][n] uint8 output (one code per byte), or NULL.
+ * mse     device double, receives mean((W - W_hat)^2) (0 when m*n == 0), or NULL.
+ * Arithmetic is fp32 (the targets' feedback sums run in another order than a sequential
+ * evaluation). If A is singular the status word becomes LCQ_ERR_SINGULAR and every code is 0.
+ * Needs lcq_workspace_size(LCQ_OP_LDLQ, 0, m, n, d) bytes of ws (the error history, 4 n bytes per
+ * row of m rounded up to 64 rows).
+ */
+lcq_status lcq_ldlq(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, const float *U,
+                    uint8_t *packed, uint8_t *codes, double *mse, void *ws, size_t ws_bytes, void *stream);
 
 /*
  * lcq_decode - affine decode of packed codes (Sec. 3.2 Eq. def:forward):
@@ -321,7 +362,9 @@ typedef enum lcq_kernel_kind {
     LCQ_K_REDUCE = 7,        /* fixed-order dA/db reduction                  */
     LCQ_K_GEMV_PREP = 8,     /* reserved (the transform is timed inside GEMV) */
     LCQ_K_GEMV = 9,          /* packed product: activation transform + main  */
-    LCQ_K_NUM_KINDS = 10
+    LCQ_K_LDL_FACTOR = 10,   /* LDLQ: block U D U^T factorisation (all its launches) */
+    LCQ_K_LDLQ = 11,         /* LDLQ: error-feedback sweep                   */
+    LCQ_K_NUM_KINDS = 12
 } lcq_kernel_kind;
 lcq_status lcq_trace_enable(int on);
 /*

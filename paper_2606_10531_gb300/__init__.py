@@ -20,6 +20,7 @@ STATUS_NAMES = {0: "LCQ_OK", 1: "LCQ_ERR_NULL", 2: "LCQ_ERR_SHAPE", 3: "LCQ_ERR_
                 9: "LCQ_ERR_ARG", 10: "LCQ_ERR_LIMIT"}
 LCQ_OP_ENCODE, LCQ_OP_LINEAR_FWD, LCQ_OP_LINEAR_BWD, LCQ_OP_GEMM_PACKED2B, LCQ_OP_GEMM_PACKED2B_HADAMARD = 1, 2, 3, 4, 5
 LCQ_OP_ENCODE_BATCH = 6
+LCQ_OP_LDL_FACTOR, LCQ_OP_LDLQ = 7, 8
 LCQ_ENCODE_BATCH_MAX = 16
 LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 
@@ -27,9 +28,10 @@ LCQ_STE_IDENTITY, LCQ_STE_CLIPPED, LCQ_STE_DGE = 0, 1, 2
 EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_linear_fwd", "lcq_linear_bwd",
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
            "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout",
-           "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard", "lcq_encode_batch")
+           "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard", "lcq_encode_batch",
+           "lcq_ldl_factor", "lcq_ldlq")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
-                "gemv_prep", "gemv")
+                "gemv_prep", "gemv", "ldl_factor", "ldlq")
 
 
 class LCQError(RuntimeError):
@@ -63,6 +65,8 @@ _SIG = {
     "lcq_encode_batch": (ctypes.c_int, [ctypes.POINTER(lcq_encode_item), ctypes.c_int, ctypes.c_int, _P,
                                         ctypes.c_size_t, _P]),
     "lcq_decode": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
+    "lcq_ldl_factor": (ctypes.c_int, [_P, _I64, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
+    "lcq_ldlq": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "lcq_pack2b": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
     "lcq_linear_fwd": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P,
                                       ctypes.c_size_t, _P]),
@@ -163,6 +167,18 @@ def lcq_encode_batch(items, d: int, ws, stream=None):
         arr[k] = lcq_encode_item(addr(it["W"]), m, n, addr(it["A"]), addr(it["b"]), addr(it.get("packed")),
                                  addr(it.get("codes")), addr(it.get("latent")), addr(it.get("mse")))
     _check(lib().lcq_encode_batch(arr, len(items), d, _ptr(ws), ws.numel(), _stream(stream)), "lcq_encode_batch")
+
+
+def lcq_ldl_factor(H, d: int, U, ws, D=None, stream=None):
+    n = H.shape[0]
+    _check(lib().lcq_ldl_factor(_ptr(H), n, d, _ptr(U), _ptr(D), _ptr(ws), ws.numel(), _stream(stream)),
+           "lcq_ldl_factor")
+
+
+def lcq_ldlq(W, A, b, U, d: int, ws, packed=None, codes=None, mse=None, stream=None):
+    m, n = W.shape
+    _check(lib().lcq_ldlq(_ptr(W), m, n, d, _ptr(A), _ptr(b), _ptr(U), _ptr(packed), _ptr(codes), _ptr(mse),
+                          _ptr(ws), ws.numel(), _stream(stream)), "lcq_ldlq")
 
 
 def lcq_decode(packed, n: int, d: int, A, b, W_hat_f32=None, W_hat_bf16=None, stream=None):

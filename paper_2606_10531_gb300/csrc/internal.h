@@ -51,6 +51,34 @@ struct EncodeBatchArgs {
     int32_t *status;
 };
 
+// LDLQ (Sec. 2.2): block U D U^T factorisation of the proxy Hessian, and the error-feedback sweep.
+struct LdlFactorArgs {
+    const float *H;           // [n][n] symmetric positive definite (upper triangle read)
+    int64_t n;
+    int d;
+    float *U;                 // [n][n] output, zero on and below the block diagonal
+    float *D;                 // [n/d][d][d] output, or null
+    float *scratch;           // ldl_factor_scratch_bytes(n)
+    int32_t *status;
+};
+size_t ldl_factor_scratch_bytes(int64_t n);
+cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st);
+
+struct LdlqArgs {
+    const float *W;
+    int64_t m, n;
+    int d;
+    const float *A, *b, *U;
+    uint8_t *packed, *codes;
+    double *mse;
+    float *E;                 // error history, ldlq_history_bytes(m, n)
+    double *partials;         // [ldlq_tiles(m)]
+    int32_t *status;
+};
+int64_t ldlq_tiles(int64_t m);
+size_t ldlq_history_bytes(int64_t m, int64_t n);
+cudaError_t launch_ldlq(const LdlqArgs &a, cudaStream_t st);
+
 // Chunk size (fp32 weights) of the encode pipeline.
 int64_t encode_chunk_size();
 

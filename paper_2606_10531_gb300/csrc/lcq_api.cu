@@ -184,6 +184,10 @@ size_t lcq_workspace_size(int op, int64_t N, int64_t m, int64_t n, int d) {
             return kHeader + packed_gemv_workspace(N, n);
         case LCQ_OP_GEMM_PACKED2B_HADAMARD:
             return kHeader + align256(static_cast<size_t>(N) * static_cast<size_t>(n) * 4) + packed_gemv_workspace(N, n);
+        case LCQ_OP_LDL_FACTOR:
+            return kHeader + ldl_factor_scratch_bytes(n);
+        case LCQ_OP_LDLQ:
+            return kHeader + align256(ldlq_history_bytes(m, n)) + align256(sizeof(double) * ldlq_tiles(m));
         default:
             return 0;
     }
@@ -290,6 +294,47 @@ lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_
     a.corr = reinterpret_cast<float *>(base + packed_gemv_corr_offset(N, n));
     a.status = &h->status;
     return cuda_status(launch_packed_gemv(a, d, num_sms_current(), st));
+}
+
+lcq_status lcq_ldl_factor(const float *H, int64_t n, int d, float *U, float *D, void *ws, size_t ws_bytes,
+                          void *stream) {
+    LCQ_TRY(check_common(0, n, d));
+    if (n == 0) return LCQ_OK;
+    if (n > 65536) return LCQ_ERR_SHAPE;
+    LCQ_TRY(check_tensor(H, n * n));
+    LCQ_TRY(check_tensor(U, n * n));
+    LCQ_TRY(check_tensor(D, n * d, false));
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_LDL_FACTOR, 0, 0, n, d)));
+    cudaStream_t st = as_stream(stream);
+    Header *h = static_cast<Header *>(ws);
+    LdlFactorArgs a{H, n, d, U, D, reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kHeader), &h->status};
+    trace_begin(LCQ_K_LDL_FACTOR, st);
+    const cudaError_t e = launch_ldl_factor(a, st);
+    trace_end(LCQ_K_LDL_FACTOR, st);
+    return cuda_status(e);
+}
+
+lcq_status lcq_ldlq(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, const float *U,
+                    uint8_t *packed, uint8_t *codes, double *mse, void *ws, size_t ws_bytes, void *stream) {
+    LCQ_TRY(check_common(m, n, d));
+    const int64_t mn = m * n;
+    LCQ_TRY(check_tensor(W, mn));
+    LCQ_TRY(check_tensor(U, n * n));
+    LCQ_TRY(check_tensor(packed, mn, false));
+    LCQ_TRY(check_tensor(codes, mn, false));
+    if (!A || !b) return LCQ_ERR_NULL;
+    if (ldlq_tiles(m) * n >= (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_LDLQ, 0, m, n, d)));
+    cudaStream_t st = as_stream(stream);
+    if (mn == 0) return mse ? cuda_status(cudaMemsetAsync(mse, 0, sizeof(double), st)) : LCQ_OK;
+    Header *h = static_cast<Header *>(ws);
+    uint8_t *base = static_cast<uint8_t *>(ws) + kHeader;
+    LdlqArgs a{W, m, n, d, A, b, U, packed, codes, mse, reinterpret_cast<float *>(base),
+               reinterpret_cast<double *>(base + align256(ldlq_history_bytes(m, n))), &h->status};
+    trace_begin(LCQ_K_LDLQ, st);
+    const cudaError_t e = launch_ldlq(a, st);
+    trace_end(LCQ_K_LDLQ, st);
+    return cuda_status(e);
 }
 
 lcq_status lcq_init_codebook(const float *G, int d, float *A, float *b, void *stream) {

@@ -1,0 +1,547 @@
+// LDLQ initialisation of the codes (Sec. 2.2 adopts LDLQ, QuIP): the column groups of W are
+// quantized in order, each group's target being its weights plus the earlier groups' errors fed
+// through the block U D U^T factor of the proxy Hessian H:
+//
+//     H = (U + I) D (U + I)^T,   T_k = W_k + sum_{j<k} (W_j - W_hat_j) U_{j,k},
+//     z_k = clip(round(A^{-1}(T_k - b)), 0, 3),   W_hat_k = A z_k + b.
+//
+// Factorisation (ldl_panel_kernel, ldl_gemm_nt_kernel): right-looking over 128-column panels from
+// the last to the first. A panel's diagonal block is factored by one CTA in shared memory; the
+// column block above it and the Schur-complement update of the leading matrix are fp32 SIMT GEMMs
+// (Y = S_QP M^-T, U_QP = S_QP M^-T D^-1, S_QQ -= Y U_QP^T; upper triangle only, the panel kernel
+// mirrors it).
+//
+// Sweep (ldlq_sweep_kernel): rows are independent, so one CTA takes 64 rows through every column
+// chunk of 128 columns. For chunk c it first forms the feedback of all earlier columns as a GEMM,
+// F = E_{<c} U_{<c,c} (E = W - W_hat, this CTA's own error history, written by it in earlier chunks),
+// then rounds the chunk's groups in order, adding the in-chunk feedback as it goes. One producer
+// thread streams 32-row slices of U (and of the error history) through a TMA ring; the error history
+// of the previous chunk is loaded only after the compute threads have published it (an mbarrier
+// phase per chunk, after a generic-to-async proxy fence).
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "internal.h"
+#include "invert.cuh"
+
+namespace lcq {
+
+// ================================================================== factorisation
+
+constexpr int kLdlPanel = 128;        // panel width (columns), a multiple of 8
+constexpr int kLdlThreads = 256;
+constexpr int kLdlLd = kLdlPanel + 1;
+
+struct LdlPanelSmem {
+    float S[kLdlPanel][kLdlLd];       // Schur block of the panel (symmetrised); later M^-1
+    float Up[kLdlPanel][kLdlLd];      // U of the panel (strictly upper d x d blocks)
+    float Dinv[kLdlPanel / 4][64];    // D_k^{-1} per group
+    InvScratch inv;
+};
+
+// Factor the diagonal block S[c0:c0+P, c0:c0+P] (upper triangle read, mirrored) of the current
+// Schur complement: U and D of the panel's groups, eliminated from the last group to the first; then
+// M^-1 = (I + U_PP)^-1 by block back substitution, and D^-1 M^-1. Writes U's panel block, D (if
+// requested), Minv and Binv (P x P, leading dimension kLdlPanel).
+template <int D>
+__global__ void __launch_bounds__(kLdlThreads)
+ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, float *__restrict__ U,
+                 float *__restrict__ Dout, float *__restrict__ Minv, float *__restrict__ Binv, int32_t *status) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    LdlPanelSmem &s = *reinterpret_cast<LdlPanelSmem *>(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int G = P / D;
+    for (int e = tid; e < P * P; e += kLdlThreads) {
+        const int i = e / P, j = e % P;
+        const int64_t lo = i <= j ? i : j, hi = i <= j ? j : i;
+        s.S[i][j] = S[(c0 + lo) * n + c0 + hi];
+        s.Up[i][j] = 0.0f;
+    }
+    __syncthreads();
+    for (int k = G - 1; k >= 0; --k) {
+        const int kd = k * D;
+        if (warp == 0) {
+            for (int e = tid; e < D * D; e += 32) s.inv.A[e] = s.S[kd + e / D][kd + e % D];
+            __syncwarp();
+            invert_warp<D>(s.inv);
+            for (int e = tid; e < D * D; e += 32) {
+                s.Dinv[k][e] = s.inv.Ainv[e];
+                if (Dout) Dout[(c0 / D + k) * D * D + e] = s.inv.A[e];
+            }
+            if (tid == 0 && s.inv.singular) set_status(status, LCQ_ERR_SINGULAR);
+        }
+        __syncthreads();
+        if (k == 0) break;
+        // U_{<k,k} = S_{<k,k} D_k^{-1}
+        for (int e = tid; e < kd * D; e += kLdlThreads) {
+            const int i = e / D, j = e % D;
+            float acc = 0.0f;
+#pragma unroll
+            for (int q = 0; q < D; ++q) acc = fmaf(s.S[i][kd + q], s.Dinv[k][q * D + j], acc);
+            s.Up[i][kd + j] = acc;
+        }
+        __syncthreads();
+        // S_{<k,<k} -= U_{<k,k} S_{k,<k}
+        for (int e = tid; e < kd * kd; e += kLdlThreads) {
+            const int i = e / kd, j = e % kd;
+            float acc = s.S[i][j];
+#pragma unroll
+            for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[kd + q][j], acc);
+            s.S[i][j] = acc;
+        }
+        __syncthreads();
+    }
+    // U's panel block (the zero blocks stay as the caller cleared them)
+    for (int e = tid; e < P * P; e += kLdlThreads) {
+        const int i = e / P, j = e % P;
+        if (i / D < j / D) U[(c0 + i) * n + c0 + j] = s.Up[i][j];
+    }
+    // X = M^-1, M = I + Up unit upper: X_k = E_k - sum_{j>k} Up_{k,j} X_j, block rows from the last
+    for (int k = G - 1; k >= 0; --k) {
+        const int kd = k * D;
+        for (int e = tid; e < D * P; e += kLdlThreads) {
+            const int r = kd + e / P, col = e % P;
+            float acc = (r == col) ? 1.0f : 0.0f;
+            for (int c = kd + D; c < P; ++c) acc = fmaf(-s.Up[r][c], s.S[c][col], acc);
+            s.S[r][col] = acc;
+        }
+        __syncthreads();
+    }
+    for (int e = tid; e < P * P; e += kLdlThreads) {
+        const int i = e / P, j = e % P;
+        Minv[i * kLdlPanel + j] = s.S[i][j];
+        const int k = i / D, r = i % D;
+        float acc = 0.0f;
+#pragma unroll
+        for (int q = 0; q < D; ++q) acc = fmaf(s.Dinv[k][r * D + q], s.S[k * D + q][j], acc);
+        Binv[i * kLdlPanel + j] = acc;
+    }
+}
+
+// C[i][j] = beta C[i][j] + alpha sum_k A[i][k] B[j][k] for i < M, j < N (K a multiple of 16; rows
+// of A and B 16-byte aligned). upper: skip the 64 x 64 tiles that lie wholly below the diagonal.
+constexpr int kGemmTile = 64, kGemmK = 16, kGemmPad = 68;
+
+__global__ void __launch_bounds__(256)
+ldl_gemm_nt_kernel(const float *__restrict__ Am, int64_t lda, const float *__restrict__ Bm, int64_t ldb,
+                   float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int K, float alpha, float beta,
+                   int upper) {
+    const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kGemmTile, j0 = static_cast<int64_t>(blockIdx.x) * kGemmTile;
+    if (upper && i0 > j0 + kGemmTile - 1) return;
+    __shared__ __align__(16) float As[kGemmK][kGemmPad];
+    __shared__ __align__(16) float Bs[kGemmK][kGemmPad];
+    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+    const int lr = tid >> 2, lk = (tid & 3) * 4;
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < K; k0 += kGemmK) {
+        float4 va = make_float4(0.f, 0.f, 0.f, 0.f), vb = va;
+        if (i0 + lr < M) va = *reinterpret_cast<const float4 *>(Am + (i0 + lr) * lda + k0 + lk);
+        if (j0 + lr < N) vb = *reinterpret_cast<const float4 *>(Bm + (j0 + lr) * ldb + k0 + lk);
+        As[lk + 0][lr] = va.x; As[lk + 1][lr] = va.y; As[lk + 2][lr] = va.z; As[lk + 3][lr] = va.w;
+        Bs[lk + 0][lr] = vb.x; Bs[lk + 1][lr] = vb.y; Bs[lk + 2][lr] = vb.z; Bs[lk + 3][lr] = vb.w;
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < kGemmK; ++kk) {
+            const float4 a = *reinterpret_cast<const float4 *>(&As[kk][ty * 4]);
+            const float4 b = *reinterpret_cast<const float4 *>(&Bs[kk][tx * 4]);
+            const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int64_t r = i0 + ty * 4 + i;
+        if (r >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int64_t c = j0 + tx * 4 + j;
+            if (c >= N) continue;
+            float *p = C + r * ldc + c;
+            *p = beta == 0.0f ? alpha * acc[i][j] : fmaf(alpha, acc[i][j], beta * *p);
+        }
+    }
+}
+
+size_t ldl_factor_scratch_bytes(int64_t n) {
+    const auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+    const size_t nn = static_cast<size_t>(n);
+    return al(nn * nn * 4) + al(nn * kLdlPanel * 4) + 2 * al(size_t(kLdlPanel) * kLdlPanel * 4);
+}
+
+static cudaError_t gemm_nt(const float *A, int64_t lda, const float *B, int64_t ldb, float *C, int64_t ldc, int64_t M,
+                           int64_t N, int K, float alpha, float beta, bool upper, cudaStream_t st) {
+    if (M <= 0 || N <= 0) return cudaSuccess;
+    dim3 grid(static_cast<unsigned>((N + kGemmTile - 1) / kGemmTile), static_cast<unsigned>((M + kGemmTile - 1) / kGemmTile));
+    ldl_gemm_nt_kernel<<<grid, 256, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, alpha, beta, upper ? 1 : 0);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
+    const int64_t n = a.n;
+    const size_t nn = static_cast<size_t>(n);
+    const auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+    float *S = a.scratch;
+    float *Y = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(S) + al(nn * nn * 4));
+    float *Minv = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(Y) + al(nn * kLdlPanel * 4));
+    float *Binv = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(Minv) + al(size_t(kLdlPanel) * kLdlPanel * 4));
+    void (*panel)(const float *, int64_t, int64_t, int, float *, float *, float *, float *, int32_t *) =
+        a.d == 4 ? ldl_panel_kernel<4> : ldl_panel_kernel<8>;
+    const int smem = static_cast<int>(sizeof(LdlPanelSmem));
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(panel), smem);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaMemcpyAsync(S, a.H, nn * nn * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(a.U, 0, nn * nn * 4, st)) != cudaSuccess) return e;
+    for (int64_t c1 = n; c1 > 0; c1 -= kLdlPanel) {
+        const int64_t c0 = c1 > kLdlPanel ? c1 - kLdlPanel : 0;
+        const int P = static_cast<int>(c1 - c0);
+        panel<<<1, kLdlThreads, smem, st>>>(S, n, c0, P, a.U, a.D, Minv, Binv, a.status);
+        count_launch();
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if (c0 == 0) break;
+        // Y = S_QP M^-T, U_QP = S_QP (D^-1 M^-1)^T, S_QQ -= Y U_QP^T (P = kLdlPanel here)
+        if ((e = gemm_nt(S + c0, n, Minv, kLdlPanel, Y, kLdlPanel, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
+        if ((e = gemm_nt(S + c0, n, Binv, kLdlPanel, a.U + c0, n, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
+        if ((e = gemm_nt(Y, kLdlPanel, a.U + c0, n, S, n, c0, c0, P, -1.0f, 1.0f, true, st)) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+// ================================================================== sweep
+
+constexpr int kSwR = 64;              // rows per CTA
+constexpr int kSwC = 128;             // columns per chunk (4 slices of 32)
+constexpr int kSwBK = 32;             // rows of U / of the error history per ring stage
+constexpr int kSwStages = 4;
+constexpr int kSwWarps = 8;           // compute warps; + 1 producer warp
+constexpr int kSwThreads = 32 * (kSwWarps + 1);
+constexpr int kSwExLd = 33;           // padded row of the per-slice error exchange (conflict-free scalar access)
+
+struct SweepSmem {
+    float ring_u[kSwStages][kSwBK][kSwC];    // U[k0 .. k0+31][c0 .. c0+127]
+    float ring_e[kSwStages][kSwBK][kSwR];    // E[k0 .. k0+31][64 rows] (history, k-major)
+    float T[kSwR][kSwC + 4];                 // feedback of the earlier chunks, then the chunk's weights
+    float ex[kSwC / 32][kSwR][kSwExLd];      // errors of one slice, for the later slices
+    float A[64], Ainv[64], b[8];
+    InvScratch inv;
+    double red[kSwWarps];
+    uint64_t full[kSwStages], empty[kSwStages], edone;
+};
+
+__device__ __forceinline__ void sweep_bar() {
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * kSwWarps) : "memory");
+}
+// the warps taking part in the errors of slice s: warps 2s .. 7
+__device__ __forceinline__ void slice_bar(int s) {
+    asm volatile("bar.sync %0, %1;" ::"r"(2 + s), "r"(32 * (kSwWarps - 2 * s)) : "memory");
+}
+// shared-memory load the compiler must not hoist (keeps the d x d constants out of registers)
+__device__ __forceinline__ float lds_nohoist(const float *p) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(smem_u32(p)));
+    return v;
+}
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+struct SweepParams {
+    const float *W;
+    int64_t m, n;
+    const float *A, *b;
+    uint8_t *packed, *codes;
+    float *E;                  // [tiles][n][kSwR] error history
+    double *partials;          // [tiles] per-CTA sum of squared errors, or null
+    int32_t *status;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kSwThreads, 1)
+ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmE, const SweepParams p) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    SweepSmem &s = *reinterpret_cast<SweepSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int64_t n = p.n, tile = blockIdx.x;
+    const int nchunks = static_cast<int>((n + kSwC - 1) / kSwC);
+    if (tid == 0) {
+        for (int i = 0; i < kSwStages; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], kSwWarps);
+        }
+        mbar_init(&s.edone, 32 * kSwWarps);
+        fence_barrier_init();
+    }
+    if (tid < D * D) s.A[tid] = s.inv.A[tid] = p.A[tid];
+    if (tid < D) s.b[tid] = p.b[tid];
+    __syncthreads();
+
+    if (warp == kSwWarps) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            prefetch_tensormap(&tmU);
+            prefetch_tensormap(&tmE);
+            int st = 0;
+            uint32_t ph = 0;
+            for (int c = 0; c < nchunks; ++c) {
+                const int c0 = c * kSwC;
+                const int cend = static_cast<int>(n < c0 + kSwC ? n : c0 + kSwC);
+                for (int k0 = 0; k0 < cend; k0 += kSwBK) {
+                    const bool gemm = k0 < c0;
+                    if (gemm && k0 == c0 - kSwC && !mbar_wait(&s.edone, (c - 1) & 1, p.status)) return;
+                    if (!mbar_wait(&s.empty[st], ph ^ 1, p.status)) return;
+                    mbar_arrive_expect_tx(&s.full[st], gemm ? sizeof(s.ring_u[0]) + sizeof(s.ring_e[0]) : sizeof(s.ring_u[0]));
+                    tma_load_2d(&s.ring_u[st][0][0], &tmU, c0, k0, &s.full[st]);
+                    if (gemm) tma_load_2d(&s.ring_e[st][0][0], &tmE, 0, static_cast<int32_t>(tile * n + k0), &s.full[st]);
+                    if (++st == kSwStages) { st = 0; ph ^= 1; }
+                }
+            }
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- compute
+    if (warp == 0) invert_warp<D>(s.inv);
+    sweep_bar();
+    if (tid < D * D) s.Ainv[tid] = s.inv.Ainv[tid];
+    if (tid == 0 && s.inv.singular && blockIdx.x == 0) set_status(p.status, LCQ_ERR_SINGULAR);
+    sweep_bar();
+
+    const int ty = tid >> 4, tx = tid & 15;           // feedback GEMM: rows 4ty.., cols 4tx.. and 64+4tx..
+    const int q = warp >> 1, r = (warp & 1) * 32 + lane;   // rounding: row r, slice q (columns 32q .. 32q+31)
+    const int64_t grow = tile * kSwR + r;
+    const bool row_ok = grow < p.m;
+    int st = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    double sq = 0.0;
+
+    for (int c = 0; c < nchunks; ++c) {
+        const int c0 = c * kSwC;
+        const int cw = static_cast<int>(n - c0 < kSwC ? n - c0 : kSwC);
+        const int col0 = c0 + 32 * q;                  // this thread's first column
+        float w[32];
+#pragma unroll
+        for (int i = 0; i < 32; i += 4) {
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (row_ok && col0 + i < n) v = *reinterpret_cast<const float4 *>(p.W + grow * n + col0 + i);
+            w[i] = v.x; w[i + 1] = v.y; w[i + 2] = v.z; w[i + 3] = v.w;
+        }
+        // feedback of the earlier chunks: F = E_{<c0} U_{<c0, chunk}
+        float acc[4][8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+        for (int k0 = 0; k0 < c0; k0 += kSwBK) {
+            if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
+            if (ok) {
+#pragma unroll 8
+                for (int kk = 0; kk < kSwBK; ++kk) {
+                    const float4 a = *reinterpret_cast<const float4 *>(&s.ring_e[st][kk][4 * ty]);
+                    const float4 b0 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][4 * tx]);
+                    const float4 b1 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][64 + 4 * tx]);
+                    const float av[4] = {a.x, a.y, a.z, a.w};
+                    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.empty[st]);
+            if (++st == kSwStages) { st = 0; ph ^= 1; }
+        }
+        sweep_bar();                                   // the previous chunk's readers of T are done
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][4 * tx]) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][64 + 4 * tx]) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+        }
+        sweep_bar();
+        float t[32];
+#pragma unroll
+        for (int i = 0; i < 32; i += 4) {
+            float4 *tp = reinterpret_cast<float4 *>(&s.T[r][32 * q + i]);
+            const float4 v = *tp;
+            t[i] = w[i] + v.x; t[i + 1] = w[i + 1] + v.y; t[i + 2] = w[i + 2] + v.z; t[i + 3] = w[i + 3] + v.w;
+            *tp = make_float4(w[i], w[i + 1], w[i + 2], w[i + 3]);   // own region: the weights, for the errors
+        }
+        uint32_t bits0 = 0, bits1 = 0;
+        float csq = 0.0f;
+        // the chunk's slices in order: slice s is rounded by warps 2s, 2s+1 (its columns are theirs);
+        // its errors then reach the later slices through U's diagonal block
+        for (int sl = 0; sl * 32 < cw; ++sl) {
+            if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
+            const float(*Us)[kSwC] = s.ring_u[st];
+            if (q == sl) {
+#pragma unroll 1
+                for (int j = 0; j < 32 / D; ++j) {
+                    float u[D], e[D];
+#pragma unroll
+                    for (int i = 0; i < D; ++i) {
+                        float v = 0.0f;
+#pragma unroll
+                        for (int jj = 0; jj < D; ++jj) v = fmaf(lds_nohoist(&s.Ainv[i * D + jj]), t[j * D + jj] - lds_nohoist(&s.b[jj]), v);
+                        u[i] = v;
+                    }
+                    uint32_t z[D];
+#pragma unroll
+                    for (int i = 0; i < D; ++i) z[i] = round_clamp3(u[i]);
+#pragma unroll
+                    for (int i = 0; i < D; ++i) {
+                        float wh = lds_nohoist(&s.b[i]);
+#pragma unroll
+                        for (int jj = 0; jj < D; ++jj) wh = fmaf(lds_nohoist(&s.A[i * D + jj]), static_cast<float>(z[jj]), wh);
+                        e[i] = lds_nohoist(&s.T[r][32 * sl + j * D + i]) - wh;
+                    }
+#pragma unroll
+                    for (int i = 0; i < D; ++i) {
+                        const int cc = j * D + i;
+                        if (cc < 16) bits0 |= z[i] << (2 * cc);
+                        else bits1 |= z[i] << (2 * (cc - 16));
+                        if (col0 + cc < n) csq = fmaf(e[i], e[i], csq);
+                    }
+                    // later groups of this slice, one row of U at a time (the empty asm keeps the
+                    // compiler from hoisting every row's loads at once)
+#pragma unroll
+                    for (int i = 0; i < D; ++i) {
+                        const float4 *urow = reinterpret_cast<const float4 *>(&Us[j * D + i][32 * sl]);
+#pragma unroll
+                        for (int c4 = (j + 1) * D / 4; c4 < 8; ++c4) {
+                            const float4 uv = urow[c4];
+                            t[4 * c4] = fmaf(e[i], uv.x, t[4 * c4]);
+                            t[4 * c4 + 1] = fmaf(e[i], uv.y, t[4 * c4 + 1]);
+                            t[4 * c4 + 2] = fmaf(e[i], uv.z, t[4 * c4 + 2]);
+                            t[4 * c4 + 3] = fmaf(e[i], uv.w, t[4 * c4 + 3]);
+                        }
+                        asm volatile("" ::: "memory");
+                    }
+#pragma unroll
+                    for (int i = 0; i < D; ++i) t[j * D + i] = e[i];
+                }
+                if (sl < kSwC / 32 - 1) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) s.ex[sl][r][i] = t[i];
+                }
+            }
+            if (sl < kSwC / 32 - 1 && q >= sl) slice_bar(sl);
+            if (q > sl) {
+                // t += e_slice U[slice rows][this thread's columns]
+#pragma unroll 2
+                for (int i = 0; i < 32; ++i) {
+                    const float ei = s.ex[sl][r][i];
+                    const float4 *urow = reinterpret_cast<const float4 *>(&Us[i][32 * q]);
+#pragma unroll
+                    for (int c4 = 0; c4 < 8; ++c4) {
+                        const float4 uv = urow[c4];
+                        t[4 * c4] = fmaf(ei, uv.x, t[4 * c4]);
+                        t[4 * c4 + 1] = fmaf(ei, uv.y, t[4 * c4 + 1]);
+                        t[4 * c4 + 2] = fmaf(ei, uv.z, t[4 * c4 + 2]);
+                        t[4 * c4 + 3] = fmaf(ei, uv.w, t[4 * c4 + 3]);
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.empty[st]);
+            if (++st == kSwStages) { st = 0; ph ^= 1; }
+        }
+        // this thread's columns: error history (k-major), codes
+        if (col0 < n) {
+            float *Eh = p.E + (tile * n + col0) * kSwR + r;
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                if (col0 + i < n) Eh[static_cast<int64_t>(i) * kSwR] = t[i];
+            if (row_ok && p.packed) {
+                uint8_t *pk = p.packed + grow * (n / 4) + col0 / 4;
+                if (col0 + 32 <= n && (reinterpret_cast<uintptr_t>(pk) & 7u) == 0) {
+                    *reinterpret_cast<uint2 *>(pk) = make_uint2(bits0, bits1);
+                } else {
+                    for (int i = 0; i < 32 && col0 + i < n; i += 4)
+                        pk[i / 4] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 0xFFu);
+                }
+            }
+            if (row_ok) {
+                if (p.codes) {
+                    uint8_t *cd = p.codes + grow * n + col0;
+                    for (int i = 0; i < 32 && col0 + i < n; ++i)
+                        cd[i] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 3u);
+                }
+            }
+        }
+        if (row_ok) sq += static_cast<double>(csq);
+        fence_proxy_async_global();
+        mbar_arrive(&s.edone);
+    }
+    if (p.partials) {
+        for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+        if (lane == 0) s.red[warp] = sq;
+        sweep_bar();
+        if (tid == 0) {
+            double tot = 0.0;
+            for (int i = 0; i < kSwWarps; ++i) tot += s.red[i];
+            p.partials[blockIdx.x] = tot;
+        }
+    }
+}
+
+// mse = sum of the per-CTA partials (fixed order) / count
+__global__ void ldlq_mse_kernel(const double *partials, int nparts, double count, double *mse) {
+    __shared__ double red[256];
+    double v = 0.0;
+    for (int i = threadIdx.x; i < nparts; i += 256) v += partials[i];
+    red[threadIdx.x] = v;
+    __syncthreads();
+    for (int o = 128; o; o >>= 1) {
+        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *mse = count > 0.0 ? red[0] / count : 0.0;
+}
+
+int64_t ldlq_tiles(int64_t m) { return (m + kSwR - 1) / kSwR; }
+size_t ldlq_history_bytes(int64_t m, int64_t n) {
+    return static_cast<size_t>(ldlq_tiles(m)) * kSwR * static_cast<size_t>(n) * 4;
+}
+
+static bool make_map_f32(CUtensorMap *map, const float *base, uint64_t inner, uint64_t outer, uint64_t ld_elems,
+                         uint32_t box_inner, uint32_t box_outer) {
+    auto enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
+    if (!enc) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {ld_elems * 4};
+    cuuint32_t box[2] = {box_inner, box_outer}, estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+cudaError_t launch_ldlq(const LdlqArgs &a, cudaStream_t st) {
+    const int64_t tiles = ldlq_tiles(a.m);
+    CUtensorMap tmU, tmE;
+    if (!make_map_f32(&tmU, a.U, a.n, a.n, a.n, kSwC, kSwBK) ||
+        !make_map_f32(&tmE, a.E, kSwR, static_cast<uint64_t>(tiles * a.n), kSwR, kSwR, kSwBK))
+        return cudaErrorInvalidValue;
+    SweepParams p{a.W, a.m, a.n, a.A, a.b, a.packed, a.codes, a.E, a.mse ? a.partials : nullptr, a.status};
+    void (*k)(const CUtensorMap, const CUtensorMap, const SweepParams) =
+        a.d == 4 ? ldlq_sweep_kernel<4> : ldlq_sweep_kernel<8>;
+    const int smem = static_cast<int>(sizeof(SweepSmem)) + 1024;
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), smem);
+    if (e != cudaSuccess) return e;
+    k<<<static_cast<unsigned>(tiles), kSwThreads, smem, st>>>(tmU, tmE, p);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.mse) {
+        ldlq_mse_kernel<<<1, 256, 0, st>>>(a.partials, static_cast<int>(tiles),
+                                           static_cast<double>(a.m) * static_cast<double>(a.n), a.mse);
+        count_launch();
+        e = cudaGetLastError();
+    }
+    return e;
+}
+
+}  // namespace lcq
