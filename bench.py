@@ -46,10 +46,11 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the separate encode / packed-product timings")
-    ap.add_argument("--case", choices=["linear", "encode", "gemv"], default=None,
+    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq"], default=None,
                     help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
                          "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
-                         "28672 x 8192, gemv = 70B gate at --tokens tokens")
+                         "28672 x 8192, gemv = 70B gate at --tokens tokens, ldlq = LDLQ sweep of a "
+                         "9728 x 4096 slice of the 8B gate (one wave, small case)")
     ap.add_argument("--tokens", type=int, default=None, help="tokens of the gemv profiling case (default 16)")
     return ap.parse_args()
 
@@ -360,6 +361,60 @@ def time_training_sets(torch, lcq, wl, seed, device, pk):
     return out
 
 
+# fp32 FMA peak of the CUDA cores (the LDLQ sweep is bound by it): 152 SMs x 128 FP32 lanes x 2 flops
+# per FMA x 2.07 GHz maximum SM clock
+FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def time_ldlq_70b(torch, lcq, wl, seed, device, pk):
+    """LDLQ initialisation of the Llama-3-70B gate (28672 x 8192, d = 8) with the synthetic proxy Hessian:
+    the block U D U^T factorisation (lcq_ldl_factor) and the error-feedback sweep (lcq_ldlq), each timed
+    with CUDA events over 3 calls after one warm-up call."""
+    mx = wl.llama3_70b_gate_ldlq()[0]
+    m, n, d = mx.m, mx.n, mx.d
+    H = wl.torch_hessian(torch, n, seed + 4000, 0, device)
+    W = wl.torch_W(torch, mx, seed + 4000, 0, device)
+    A = wl.torch_A(torch, mx, seed + 4000, 0, device).contiguous()
+    b = wl.torch_b(torch, mx, seed + 4000, 0, device).contiguous()
+    U = torch.empty((n, n), dtype=torch.float32, device=device)
+    wsf = lcq.workspace(lcq.LCQ_OP_LDL_FACTOR, 0, 0, n, d, device)
+    wss = lcq.workspace(lcq.LCQ_OP_LDLQ, 0, m, n, d, device)
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device=device)
+    mse = torch.empty(1, dtype=torch.float64, device=device)
+
+    def timed(fn, reps=3):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e-3 / reps
+
+    t_f = timed(lambda: lcq.lcq_ldl_factor(H, d, U, wsf))
+    lcq.lcq_trace_enable(True)
+    t_s = timed(lambda: lcq.lcq_ldlq(W, A, b, U, d, wss, packed=packed, mse=mse))
+    lcq.lcq_trace_enable(False)
+    sweep_calls, sweep_ms = lcq.lcq_trace_read().get("ldlq", (0, 0.0))
+    assert lcq.lcq_device_status(wsf) == 0 and lcq.lcq_device_status(wss) == 0
+    flops_sweep = float(m) * n * n            # m n^2 / 2 fused multiply-adds of the error feedback
+    flops_factor = float(n) ** 3 / 3.0        # block U D U^T of an n x n matrix
+    k_s = sweep_ms * 1e-3 / sweep_calls if sweep_calls else t_s
+    out = {"workload": "llama3-70b gate 28672x8192 LDLQ initialisation, d=8, synthetic proxy Hessian "
+                       "(AR(0.9) + rank-8, 1% outlier channels x20, 1% dampening); W ~N(0,0.015) + 0.1% Student-t(4)",
+           "factor_ms": t_f * 1e3, "factor_TFLOP/s": flops_factor / t_f / 1e12,
+           "sweep_ms": t_s * 1e3, "sweep_TFLOP/s": flops_sweep / t_s / 1e12, "mse": float(mse.item()),
+           "roofline": {"kernel": "ldlq_sweep_kernel (fp32 FMA feedback GEMM + in-chunk rounding)", "bound": "alu",
+                        "achieved": flops_sweep / k_s / 1e12, "peak": FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
+                        "frac": flops_sweep / k_s / 1e12 / FP32_PEAK_TFLOPS,
+                        "peak_kind": "derived: 152 SMs x 128 fp32 FMA lanes x 2 x 2.07 GHz", "traffic": None}}
+    del H, W, U, wsf, wss, packed
+    torch.cuda.empty_cache()
+    return out
+
+
 # ----------------------------------------------------------------------------- CPU oracle
 
 def oracle_sample(seed, budget_s, tokens=64, max_linears=7):
@@ -497,6 +552,7 @@ def main():
         torch.cuda.empty_cache()
         line["encode"] = time_encode_70b(torch, lcq, wl, args.seed, device, pk)
         line["packed_decode"] = time_gemv_70b(torch, lcq, wl, args.seed, device, pk)
+        line["ldlq_init"] = time_ldlq_70b(torch, lcq, wl, args.seed, device, pk)
         line["other_training_workloads"] = time_training_sets(torch, lcq, wl, args.seed, device, pk)
         torch.cuda.empty_cache()
         layer = None
@@ -588,6 +644,21 @@ def profile_case(args):
         def run():
             lcq.lcq_encode(W, A, b, mx.d, ws, packed=pk_, mse=mse)
         wss = [ws]
+    elif args.case == "ldlq":
+        mx = wl.llama3_8b_gate_ldlq()[0]
+        m, n, d = 152 * 64, mx.n, mx.d            # one 64-row tile per SM: one full wave
+        H = wl.torch_hessian(torch, n, args.seed, 0, device)
+        W = wl.torch_W(torch, mx, args.seed, 0, device)[:m].contiguous()
+        A, b = wl.torch_A(torch, mx, args.seed, 0, device), wl.torch_b(torch, mx, args.seed, 0, device)
+        U = torch.empty((n, n), dtype=torch.float32, device=device)
+        wsf = lcq.workspace(lcq.LCQ_OP_LDL_FACTOR, 0, 0, n, d, device)
+        lcq.lcq_ldl_factor(H, d, U, wsf)
+        pk_ = torch.empty((m, n // 4), dtype=torch.uint8, device=device)
+        ws = lcq.workspace(lcq.LCQ_OP_LDLQ, 0, m, n, d, device)
+
+        def run():
+            lcq.lcq_ldlq(W, A, b, U, d, ws, packed=pk_)
+        wss = [wsf, ws]
     else:
         mx = wl.llama3_70b_gate_decode(args.tokens or GEMV_TOKENS)[0]
         packed = wl.torch_packed_codes(torch, mx, args.seed, 0, device)

@@ -181,14 +181,16 @@ lcq_status lcq_ldl_factor(const float *H, int64_t n, int d, float *U, float *D, 
  * U       [n][n] fp32; only the entries above the block diagonal are read.
  * packed  [m][n/4] uint8 output, or NULL.
  * codes   [m][n] uint8 output (one code per byte), or NULL.
+ * latent  [m][n] fp32 output: u = A^{-1}(T_k - b), the value each code was rounded from, or NULL.
  * mse     device double, receives mean((W - W_hat)^2) (0 when m*n == 0), or NULL.
- * Arithmetic is fp32 (the targets' feedback sums run in another order than a sequential
- * evaluation). If A is singular the status word becomes LCQ_ERR_SINGULAR and every code is 0.
+ * Arithmetic is fp32; the feedback sums of a target run over up to n terms, in another order than a
+ * sequential evaluation. If A is singular the status word becomes LCQ_ERR_SINGULAR and every code is 0.
  * Needs lcq_workspace_size(LCQ_OP_LDLQ, 0, m, n, d) bytes of ws (the error history, 4 n bytes per
  * row of m rounded up to 64 rows).
  */
 lcq_status lcq_ldlq(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, const float *U,
-                    uint8_t *packed, uint8_t *codes, double *mse, void *ws, size_t ws_bytes, void *stream);
+                    uint8_t *packed, uint8_t *codes, float *latent, double *mse, void *ws, size_t ws_bytes,
+                    void *stream);
 
 /*
  * lcq_decode - affine decode of packed codes (Sec. 3.2 Eq. def:forward):

@@ -66,7 +66,7 @@ _SIG = {
                                         ctypes.c_size_t, _P]),
     "lcq_decode": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
     "lcq_ldl_factor": (ctypes.c_int, [_P, _I64, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
-    "lcq_ldlq": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "lcq_ldlq": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "lcq_pack2b": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
     "lcq_linear_fwd": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P,
                                       ctypes.c_size_t, _P]),
@@ -175,10 +175,10 @@ def lcq_ldl_factor(H, d: int, U, ws, D=None, stream=None):
            "lcq_ldl_factor")
 
 
-def lcq_ldlq(W, A, b, U, d: int, ws, packed=None, codes=None, mse=None, stream=None):
+def lcq_ldlq(W, A, b, U, d: int, ws, packed=None, codes=None, latent=None, mse=None, stream=None):
     m, n = W.shape
-    _check(lib().lcq_ldlq(_ptr(W), m, n, d, _ptr(A), _ptr(b), _ptr(U), _ptr(packed), _ptr(codes), _ptr(mse),
-                          _ptr(ws), ws.numel(), _stream(stream)), "lcq_ldlq")
+    _check(lib().lcq_ldlq(_ptr(W), m, n, d, _ptr(A), _ptr(b), _ptr(U), _ptr(packed), _ptr(codes), _ptr(latent),
+                          _ptr(mse), _ptr(ws), ws.numel(), _stream(stream)), "lcq_ldlq")
 
 
 def lcq_decode(packed, n: int, d: int, A, b, W_hat_f32=None, W_hat_bf16=None, stream=None):

@@ -70,6 +70,7 @@ struct LdlqArgs {
     int d;
     const float *A, *b, *U;
     uint8_t *packed, *codes;
+    float *latent;
     double *mse;
     float *E;                 // error history, ldlq_history_bytes(m, n)
     double *partials;         // [ldlq_tiles(m)]

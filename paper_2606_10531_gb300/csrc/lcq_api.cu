@@ -315,13 +315,15 @@ lcq_status lcq_ldl_factor(const float *H, int64_t n, int d, float *U, float *D, 
 }
 
 lcq_status lcq_ldlq(const float *W, int64_t m, int64_t n, int d, const float *A, const float *b, const float *U,
-                    uint8_t *packed, uint8_t *codes, double *mse, void *ws, size_t ws_bytes, void *stream) {
+                    uint8_t *packed, uint8_t *codes, float *latent, double *mse, void *ws, size_t ws_bytes,
+                    void *stream) {
     LCQ_TRY(check_common(m, n, d));
     const int64_t mn = m * n;
     LCQ_TRY(check_tensor(W, mn));
     LCQ_TRY(check_tensor(U, n * n));
     LCQ_TRY(check_tensor(packed, mn, false));
     LCQ_TRY(check_tensor(codes, mn, false));
+    LCQ_TRY(check_tensor(latent, mn, false));
     if (!A || !b) return LCQ_ERR_NULL;
     if (ldlq_tiles(m) * n >= (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
     LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_LDLQ, 0, m, n, d)));
@@ -329,7 +331,7 @@ lcq_status lcq_ldlq(const float *W, int64_t m, int64_t n, int d, const float *A,
     if (mn == 0) return mse ? cuda_status(cudaMemsetAsync(mse, 0, sizeof(double), st)) : LCQ_OK;
     Header *h = static_cast<Header *>(ws);
     uint8_t *base = static_cast<uint8_t *>(ws) + kHeader;
-    LdlqArgs a{W, m, n, d, A, b, U, packed, codes, mse, reinterpret_cast<float *>(base),
+    LdlqArgs a{W, m, n, d, A, b, U, packed, codes, latent, mse, reinterpret_cast<float *>(base),
                reinterpret_cast<double *>(base + align256(ldlq_history_bytes(m, n))), &h->status};
     trace_begin(LCQ_K_LDLQ, st);
     const cudaError_t e = launch_ldlq(a, st);

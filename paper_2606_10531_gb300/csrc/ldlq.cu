@@ -219,17 +219,17 @@ constexpr int kSwBK = 32;             // rows of U / of the error history per ri
 constexpr int kSwStages = 4;
 constexpr int kSwWarps = 8;           // compute warps; + 1 producer warp
 constexpr int kSwThreads = 32 * (kSwWarps + 1);
-constexpr int kSwExLd = 33;           // padded row of the per-slice error exchange (conflict-free scalar access)
+constexpr int kSwTLd = kSwC + 4;      // padded row of the target tile (conflict-free 16-byte access)
 
 struct SweepSmem {
     float ring_u[kSwStages][kSwBK][kSwC];    // U[k0 .. k0+31][c0 .. c0+127]
     float ring_e[kSwStages][kSwBK][kSwR];    // E[k0 .. k0+31][64 rows] (history, k-major)
-    float T[kSwR][kSwC + 4];                 // feedback of the earlier chunks, then the chunk's weights
-    float ex[kSwC / 32][kSwR][kSwExLd];      // errors of one slice, for the later slices
+    float W[kSwC / 32][kSwR][32];            // the chunk's weights: one 128B-swizzled box per slice
+    float T[kSwR][kSwTLd];                   // targets minus weights, then the errors
     float A[64], Ainv[64], b[8];
     InvScratch inv;
     double red[kSwWarps];
-    uint64_t full[kSwStages], empty[kSwStages], edone;
+    uint64_t full[kSwStages], empty[kSwStages], edone, wfull;
 };
 
 __device__ __forceinline__ void sweep_bar() {
@@ -248,12 +248,16 @@ __device__ __forceinline__ float lds_nohoist(const float *p) {
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
+// 16-byte chunk c16 of row r of a 128B-swizzled box (rows of 128 bytes)
+__device__ __forceinline__ const float4 *swz128(const float (*box)[32], int r, int c16) {
+    return reinterpret_cast<const float4 *>(&box[r][0]) + (c16 ^ (r & 7));
+}
 
 struct SweepParams {
-    const float *W;
-    int64_t m, n;
     const float *A, *b;
+    int64_t m, n;
     uint8_t *packed, *codes;
+    float *latent;             // [m][n] latent coordinates of the targets, or null
     float *E;                  // [tiles][n][kSwR] error history
     double *partials;          // [tiles] per-CTA sum of squared errors, or null
     int32_t *status;
@@ -261,7 +265,8 @@ struct SweepParams {
 
 template <int D>
 __global__ void __launch_bounds__(kSwThreads, 1)
-ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmE, const SweepParams p) {
+ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmE,
+                  const __grid_constant__ CUtensorMap tmW, const SweepParams p) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
     SweepSmem &s = *reinterpret_cast<SweepSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -273,6 +278,7 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             mbar_init(&s.empty[i], kSwWarps);
         }
         mbar_init(&s.edone, 32 * kSwWarps);
+        mbar_init(&s.wfull, 1);
         fence_barrier_init();
     }
     if (tid < D * D) s.A[tid] = s.inv.A[tid] = p.A[tid];
@@ -284,6 +290,7 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         if (lane == 0) {
             prefetch_tensormap(&tmU);
             prefetch_tensormap(&tmE);
+            prefetch_tensormap(&tmW);
             int st = 0;
             uint32_t ph = 0;
             for (int c = 0; c < nchunks; ++c) {
@@ -291,7 +298,15 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                 const int cend = static_cast<int>(n < c0 + kSwC ? n : c0 + kSwC);
                 for (int k0 = 0; k0 < cend; k0 += kSwBK) {
                     const bool gemm = k0 < c0;
-                    if (gemm && k0 == c0 - kSwC && !mbar_wait(&s.edone, (c - 1) & 1, p.status)) return;
+                    if (k0 == (c0 > 0 ? c0 - kSwC : 0)) {
+                        // the previous chunk is done (its errors published, its weights read):
+                        // this chunk's weights may replace them
+                        if (c > 0 && !mbar_wait(&s.edone, (c - 1) & 1, p.status)) return;
+                        const int nbox = (cend - c0 + 31) / 32;
+                        mbar_arrive_expect_tx(&s.wfull, nbox * sizeof(s.W[0]));
+                        for (int q = 0; q < nbox; ++q)
+                            tma_load_2d(&s.W[q][0][0], &tmW, c0 + 32 * q, static_cast<int32_t>(tile * kSwR), &s.wfull);
+                    }
                     if (!mbar_wait(&s.empty[st], ph ^ 1, p.status)) return;
                     mbar_arrive_expect_tx(&s.full[st], gemm ? sizeof(s.ring_u[0]) + sizeof(s.ring_e[0]) : sizeof(s.ring_u[0]));
                     tma_load_2d(&s.ring_u[st][0][0], &tmU, c0, k0, &s.full[st]);
@@ -314,6 +329,7 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
     const int q = warp >> 1, r = (warp & 1) * 32 + lane;   // rounding: row r, slice q (columns 32q .. 32q+31)
     const int64_t grow = tile * kSwR + r;
     const bool row_ok = grow < p.m;
+    float *trow = &s.T[r][0];
     int st = 0;
     uint32_t ph = 0;
     bool ok = true;
@@ -323,19 +339,12 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         const int c0 = c * kSwC;
         const int cw = static_cast<int>(n - c0 < kSwC ? n - c0 : kSwC);
         const int col0 = c0 + 32 * q;                  // this thread's first column
-        float w[32];
-#pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (row_ok && col0 + i < n) v = *reinterpret_cast<const float4 *>(p.W + grow * n + col0 + i);
-            w[i] = v.x; w[i + 1] = v.y; w[i + 2] = v.z; w[i + 3] = v.w;
-        }
-        // feedback of the earlier chunks: F = E_{<c0} U_{<c0, chunk}
-        float acc[4][8];
+        // feedback of the earlier chunks: F = E_{<c0} U_{<c0, chunk}, packed fp32 FMAs (two columns each)
+        float2 acc[4][4];
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+            for (int j = 0; j < 4; ++j) acc[i][j] = make_float2(0.0f, 0.0f);
         for (int k0 = 0; k0 < c0; k0 += kSwBK) {
             if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
             if (ok) {
@@ -345,11 +354,14 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                     const float4 b0 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][4 * tx]);
                     const float4 b1 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][64 + 4 * tx]);
                     const float av[4] = {a.x, a.y, a.z, a.w};
-                    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+                    const float2 bv[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
+                                          make_float2(b1.z, b1.w)};
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)
+                    for (int i = 0; i < 4; ++i) {
+                        const float2 ai = make_float2(av[i], av[i]);
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                        for (int j = 0; j < 4; ++j) acc[i][j] = __ffma2_rn(ai, bv[j], acc[i][j]);
+                    }
                 }
             }
             __syncwarp();
@@ -359,103 +371,132 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         sweep_bar();                                   // the previous chunk's readers of T are done
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][4 * tx]) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][64 + 4 * tx]) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][4 * tx]) = make_float4(acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y);
+            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][64 + 4 * tx]) = make_float4(acc[i][2].x, acc[i][2].y, acc[i][3].x, acc[i][3].y);
         }
         sweep_bar();
-        float t[32];
-#pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-            float4 *tp = reinterpret_cast<float4 *>(&s.T[r][32 * q + i]);
-            const float4 v = *tp;
-            t[i] = w[i] + v.x; t[i + 1] = w[i + 1] + v.y; t[i + 2] = w[i + 2] + v.z; t[i + 3] = w[i + 3] + v.w;
-            *tp = make_float4(w[i], w[i + 1], w[i + 2], w[i + 3]);   // own region: the weights, for the errors
-        }
+        if (ok && !mbar_wait(&s.wfull, c & 1, p.status)) ok = false;
         uint32_t bits0 = 0, bits1 = 0;
         float csq = 0.0f;
-        // the chunk's slices in order: slice s is rounded by warps 2s, 2s+1 (its columns are theirs);
-        // its errors then reach the later slices through U's diagonal block
+        // the chunk's slices in order: slice s is rounded by warps 2s, 2s+1 (its columns are theirs), in
+        // place in T (target - weight -> error); its errors then reach the later slices through U's
+        // diagonal block
         for (int sl = 0; sl * 32 < cw; ++sl) {
             if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
             const float(*Us)[kSwC] = s.ring_u[st];
             if (q == sl) {
+                float4 *t4 = reinterpret_cast<float4 *>(trow + 32 * sl);
 #pragma unroll 1
                 for (int j = 0; j < 32 / D; ++j) {
+                    float t[D], w[D];
+#pragma unroll
+                    for (int h = 0; h < D / 4; ++h) {
+                        const float4 fv = t4[j * (D / 4) + h];
+                        const float4 wv = *swz128(s.W[sl], r, j * (D / 4) + h);
+                        w[4 * h] = wv.x; w[4 * h + 1] = wv.y; w[4 * h + 2] = wv.z; w[4 * h + 3] = wv.w;
+                        t[4 * h] = wv.x + fv.x; t[4 * h + 1] = wv.y + fv.y; t[4 * h + 2] = wv.z + fv.z; t[4 * h + 3] = wv.w + fv.w;
+                    }
                     float u[D], e[D];
 #pragma unroll
                     for (int i = 0; i < D; ++i) {
                         float v = 0.0f;
 #pragma unroll
-                        for (int jj = 0; jj < D; ++jj) v = fmaf(lds_nohoist(&s.Ainv[i * D + jj]), t[j * D + jj] - lds_nohoist(&s.b[jj]), v);
+                        for (int jj = 0; jj < D; ++jj) v = fmaf(lds_nohoist(&s.Ainv[i * D + jj]), t[jj] - lds_nohoist(&s.b[jj]), v);
                         u[i] = v;
                     }
                     uint32_t z[D];
 #pragma unroll
                     for (int i = 0; i < D; ++i) z[i] = round_clamp3(u[i]);
+                    if (p.latent && row_ok && col0 + j * D < n) {
+#pragma unroll
+                        for (int i = 0; i < D; ++i) p.latent[grow * n + col0 + j * D + i] = u[i];
+                    }
 #pragma unroll
                     for (int i = 0; i < D; ++i) {
                         float wh = lds_nohoist(&s.b[i]);
 #pragma unroll
                         for (int jj = 0; jj < D; ++jj) wh = fmaf(lds_nohoist(&s.A[i * D + jj]), static_cast<float>(z[jj]), wh);
-                        e[i] = lds_nohoist(&s.T[r][32 * sl + j * D + i]) - wh;
+                        e[i] = w[i] - wh;
+                    }
+                    uint32_t zb = 0;
+#pragma unroll
+                    for (int i = 0; i < D; ++i) zb |= z[i] << (2 * i);
+                    const int sh = 2 * ((j * D) & 15);
+                    if (j * D < 16) bits0 |= zb << sh;
+                    else bits1 |= zb << sh;
+                    if (col0 + j * D < n) {
+#pragma unroll
+                        for (int i = 0; i < D; ++i) csq = fmaf(e[i], e[i], csq);
                     }
 #pragma unroll
-                    for (int i = 0; i < D; ++i) {
-                        const int cc = j * D + i;
-                        if (cc < 16) bits0 |= z[i] << (2 * cc);
-                        else bits1 |= z[i] << (2 * (cc - 16));
-                        if (col0 + cc < n) csq = fmaf(e[i], e[i], csq);
-                    }
-                    // later groups of this slice, one row of U at a time (the empty asm keeps the
-                    // compiler from hoisting every row's loads at once)
+                    for (int h = 0; h < D / 4; ++h)
+                        t4[j * (D / 4) + h] = make_float4(e[4 * h], e[4 * h + 1], e[4 * h + 2], e[4 * h + 3]);
+                    // later groups of this slice, 16 bytes of the row at a time
+                    for (int c4 = (j + 1) * (D / 4); c4 < 8; ++c4) {
+                        float4 v = t4[c4];
 #pragma unroll
-                    for (int i = 0; i < D; ++i) {
-                        const float4 *urow = reinterpret_cast<const float4 *>(&Us[j * D + i][32 * sl]);
-#pragma unroll
-                        for (int c4 = (j + 1) * D / 4; c4 < 8; ++c4) {
-                            const float4 uv = urow[c4];
-                            t[4 * c4] = fmaf(e[i], uv.x, t[4 * c4]);
-                            t[4 * c4 + 1] = fmaf(e[i], uv.y, t[4 * c4 + 1]);
-                            t[4 * c4 + 2] = fmaf(e[i], uv.z, t[4 * c4 + 2]);
-                            t[4 * c4 + 3] = fmaf(e[i], uv.w, t[4 * c4 + 3]);
+                        for (int i = 0; i < D; ++i) {
+                            const float4 uv = *reinterpret_cast<const float4 *>(&Us[j * D + i][32 * sl + 4 * c4]);
+                            v.x = fmaf(e[i], uv.x, v.x);
+                            v.y = fmaf(e[i], uv.y, v.y);
+                            v.z = fmaf(e[i], uv.z, v.z);
+                            v.w = fmaf(e[i], uv.w, v.w);
                         }
-                        asm volatile("" ::: "memory");
+                        t4[c4] = v;
                     }
-#pragma unroll
-                    for (int i = 0; i < D; ++i) t[j * D + i] = e[i];
-                }
-                if (sl < kSwC / 32 - 1) {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) s.ex[sl][r][i] = t[i];
                 }
             }
             if (sl < kSwC / 32 - 1 && q >= sl) slice_bar(sl);
             if (q > sl) {
-                // t += e_slice U[slice rows][this thread's columns]
-#pragma unroll 2
-                for (int i = 0; i < 32; ++i) {
-                    const float ei = s.ex[sl][r][i];
-                    const float4 *urow = reinterpret_cast<const float4 *>(&Us[i][32 * q]);
+                // T[r][this slice] += e_slice U[slice rows][this thread's columns]
+                float acc2[32];
+                const float4 *own = reinterpret_cast<const float4 *>(trow + 32 * q);
 #pragma unroll
-                    for (int c4 = 0; c4 < 8; ++c4) {
-                        const float4 uv = urow[c4];
-                        t[4 * c4] = fmaf(ei, uv.x, t[4 * c4]);
-                        t[4 * c4 + 1] = fmaf(ei, uv.y, t[4 * c4 + 1]);
-                        t[4 * c4 + 2] = fmaf(ei, uv.z, t[4 * c4 + 2]);
-                        t[4 * c4 + 3] = fmaf(ei, uv.w, t[4 * c4 + 3]);
+                for (int c4 = 0; c4 < 8; ++c4) {
+                    const float4 v = own[c4];
+                    acc2[4 * c4] = v.x; acc2[4 * c4 + 1] = v.y; acc2[4 * c4 + 2] = v.z; acc2[4 * c4 + 3] = v.w;
+                }
+                const float4 *es = reinterpret_cast<const float4 *>(trow + 32 * sl);
+#pragma unroll 1
+                for (int i4 = 0; i4 < 8; ++i4) {
+                    const float4 e4 = es[i4];
+                    const float ev[4] = {e4.x, e4.y, e4.z, e4.w};
+#pragma unroll
+                    for (int ii = 0; ii < 4; ++ii) {
+                        const float4 *urow = reinterpret_cast<const float4 *>(&Us[4 * i4 + ii][32 * q]);
+#pragma unroll
+                        for (int c4 = 0; c4 < 8; ++c4) {
+                            const float4 uv = urow[c4];
+                            acc2[4 * c4] = fmaf(ev[ii], uv.x, acc2[4 * c4]);
+                            acc2[4 * c4 + 1] = fmaf(ev[ii], uv.y, acc2[4 * c4 + 1]);
+                            acc2[4 * c4 + 2] = fmaf(ev[ii], uv.z, acc2[4 * c4 + 2]);
+                            acc2[4 * c4 + 3] = fmaf(ev[ii], uv.w, acc2[4 * c4 + 3]);
+                        }
+                        asm volatile("" ::: "memory");
                     }
                 }
+                float4 *ownw = reinterpret_cast<float4 *>(trow + 32 * q);
+#pragma unroll
+                for (int c4 = 0; c4 < 8; ++c4)
+                    ownw[c4] = make_float4(acc2[4 * c4], acc2[4 * c4 + 1], acc2[4 * c4 + 2], acc2[4 * c4 + 3]);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.empty[st]);
             if (++st == kSwStages) { st = 0; ph ^= 1; }
         }
-        // this thread's columns: error history (k-major), codes
+        // this thread's columns: error history (k-major) from T, codes
         if (col0 < n) {
             float *Eh = p.E + (tile * n + col0) * kSwR + r;
+            const float4 *ev = reinterpret_cast<const float4 *>(trow + 32 * q);
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-                if (col0 + i < n) Eh[static_cast<int64_t>(i) * kSwR] = t[i];
+            for (int c4 = 0; c4 < 8; ++c4) {
+                if (col0 + 4 * c4 >= n) break;
+                const float4 v = ev[c4];
+                Eh[(4 * c4 + 0) * kSwR] = v.x;
+                Eh[(4 * c4 + 1) * kSwR] = v.y;
+                Eh[(4 * c4 + 2) * kSwR] = v.z;
+                Eh[(4 * c4 + 3) * kSwR] = v.w;
+            }
             if (row_ok && p.packed) {
                 uint8_t *pk = p.packed + grow * (n / 4) + col0 / 4;
                 if (col0 + 32 <= n && (reinterpret_cast<uintptr_t>(pk) & 7u) == 0) {
@@ -465,12 +506,10 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                         pk[i / 4] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 0xFFu);
                 }
             }
-            if (row_ok) {
-                if (p.codes) {
-                    uint8_t *cd = p.codes + grow * n + col0;
-                    for (int i = 0; i < 32 && col0 + i < n; ++i)
-                        cd[i] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 3u);
-                }
+            if (row_ok && p.codes) {
+                uint8_t *cd = p.codes + grow * n + col0;
+                for (int i = 0; i < 32 && col0 + i < n; ++i)
+                    cd[i] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 3u);
             }
         }
         if (row_ok) sq += static_cast<double>(csq);
@@ -509,30 +548,32 @@ size_t ldlq_history_bytes(int64_t m, int64_t n) {
 }
 
 static bool make_map_f32(CUtensorMap *map, const float *base, uint64_t inner, uint64_t outer, uint64_t ld_elems,
-                         uint32_t box_inner, uint32_t box_outer) {
+                         uint32_t box_inner, uint32_t box_outer, bool swizzle128 = false) {
     auto enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
     if (!enc) return false;
     cuuint64_t dims[2] = {inner, outer};
     cuuint64_t strides[1] = {ld_elems * 4};
     cuuint32_t box[2] = {box_inner, box_outer}, estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 cudaError_t launch_ldlq(const LdlqArgs &a, cudaStream_t st) {
     const int64_t tiles = ldlq_tiles(a.m);
-    CUtensorMap tmU, tmE;
+    CUtensorMap tmU, tmE, tmW;
     if (!make_map_f32(&tmU, a.U, a.n, a.n, a.n, kSwC, kSwBK) ||
-        !make_map_f32(&tmE, a.E, kSwR, static_cast<uint64_t>(tiles * a.n), kSwR, kSwR, kSwBK))
+        !make_map_f32(&tmE, a.E, kSwR, static_cast<uint64_t>(tiles * a.n), kSwR, kSwR, kSwBK) ||
+        !make_map_f32(&tmW, a.W, a.n, a.m, a.n, 32, kSwR, true))
         return cudaErrorInvalidValue;
-    SweepParams p{a.W, a.m, a.n, a.A, a.b, a.packed, a.codes, a.E, a.mse ? a.partials : nullptr, a.status};
-    void (*k)(const CUtensorMap, const CUtensorMap, const SweepParams) =
+    SweepParams p{a.A, a.b, a.m, a.n, a.packed, a.codes, a.latent, a.E, a.mse ? a.partials : nullptr, a.status};
+    void (*k)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const SweepParams) =
         a.d == 4 ? ldlq_sweep_kernel<4> : ldlq_sweep_kernel<8>;
     const int smem = static_cast<int>(sizeof(SweepSmem)) + 1024;
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), smem);
     if (e != cudaSuccess) return e;
-    k<<<static_cast<unsigned>(tiles), kSwThreads, smem, st>>>(tmU, tmE, p);
+    k<<<static_cast<unsigned>(tiles), kSwThreads, smem, st>>>(tmU, tmE, tmW, p);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (a.mse) {

@@ -12,7 +12,7 @@ import pytest
 import oracle
 import paper_2606_10531_gb300 as lcq
 from paper_2606_10531_gb300 import workloads as wl
-from tests.gpu_util import TOL_BF16, dev, dev_bf16, empty_bf16, host_bf16, max_rel
+from tests.gpu_util import TOL_BF16, dev, dev_bf16, empty_bf16, host_bf16, ldlq_latent_bound, max_rel
 
 pytestmark = pytest.mark.gpu
 
@@ -130,3 +130,64 @@ def test_llama3_70b_gate_bulk_encode_full_size():
     ref_mse = sq / (mx.m * mx.n)
     assert abs(mse.item() - ref_mse) <= 1e-4 * ref_mse
     print(f"near-boundary codes excluded: {near} of {mx.m * mx.n}")
+
+
+def test_llama3_70b_gate_ldlq_full_size():
+    """LDLQ of the Llama-3-70B gate (28672 x 8192, d = 8) with the synthetic proxy Hessian, through the
+    calls bench.py times. The factor is checked by reconstructing sampled entries of H from U and D
+    (any size); the sweep, on sampled rows, by its decisions against its own fp32 latents (exact) and
+    those latents against the oracle's fp64 latents of the same history and U (fp32 error bound), and
+    by its MSE over all rows."""
+    import torch
+    mx = wl.llama3_70b_gate_ldlq()[0]
+    m, n, d = mx.m, mx.n, mx.d
+    H = wl.draw_hessian(n, SEED, 0)
+    W = wl.draw_W(mx, SEED, 0)
+    A, b = wl.draw_A(mx, SEED, 0), wl.draw_b(mx, SEED, 0)
+    U = torch.empty((n, n), dtype=torch.float32, device="cuda")
+    D = torch.empty((n // d, d, d), dtype=torch.float32, device="cuda")
+    wsf = lcq.workspace(lcq.LCQ_OP_LDL_FACTOR, 0, 0, n, d)
+    lcq.lcq_ldl_factor(dev(H), d, U, wsf, D=D)
+    codes = torch.empty((m, n), dtype=torch.uint8, device="cuda")
+    latent = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    mse = torch.empty(1, dtype=torch.float64, device="cuda")
+    wss = lcq.workspace(lcq.LCQ_OP_LDLQ, 0, m, n, d)
+    lcq.lcq_ldlq(dev(W), dev(A), dev(b), U, d, wss, packed=packed, codes=codes, latent=latent, mse=mse)
+    assert lcq.lcq_device_status(wsf) == 0 and lcq.lcq_device_status(wss) == 0
+
+    Uh = U.cpu().numpy().astype(np.float64)
+    Dh = D.cpu().numpy().astype(np.float64)
+    M = Uh + np.eye(n)
+    rng = np.random.default_rng(4242)
+    pairs = [(int(i), int(j)) for i, j in zip(rng.integers(0, n, 64), rng.integers(0, n, 64))] + [(0, 0), (n - 1, n - 1)]
+    Hmax = float(np.abs(H).max())
+    worst = 0.0
+    for i, j in pairs:
+        kmin = max(i, j) // d
+        acc = 0.0
+        for k in range(kmin, n // d):
+            s = slice(k * d, (k + 1) * d)
+            acc += M[i, s] @ Dh[k] @ M[j, s]
+        worst = max(worst, abs(acc - float(H[i, j])) / Hmax)
+    print(f"factor: max sampled |(M D M^T - H)_ij| / max|H| = {worst:.2e}")
+    assert worst < 1e-4
+
+    rows = np.concatenate([[0, m - 1], rng.choice(m, 30, replace=False)])
+    Z = codes.cpu().numpy()
+    assert np.array_equal(packed.cpu().numpy()[rows], oracle.pack2b(Z[rows]))
+    lat_gpu = latent[torch.as_tensor(rows, device="cuda")].cpu().numpy()
+    assert np.array_equal(oracle.round_clamp(lat_gpu), Z[rows])
+    lat = oracle.ldlq_latent_given_codes(W[rows], Z[rows], Uh, A, b, d)
+    bound = ldlq_latent_bound(W[rows], Z[rows], Uh, A, b, d)
+    err = np.abs(lat_gpu.astype(np.float64) - lat)
+    flips = int(np.sum(oracle.round_clamp(lat) != Z[rows]))
+    print(f"sweep: latent error max {err.max():.2e} (median bound {np.median(bound):.2e}), "
+          f"max error / bound {np.max(err / bound):.3f}; {flips} of {lat.size} decisions round otherwise "
+          f"in fp64, all within the bound of a boundary")
+    assert np.all(err <= bound)
+    sq = 0.0
+    for r0 in range(0, m, 2048):
+        sq += float(np.sum((W[r0:r0 + 2048].astype(np.float64) - oracle.decode(Z[r0:r0 + 2048], A, b, d)) ** 2))
+    ref_mse = sq / (m * n)
+    assert abs(mse.item() - ref_mse) <= 1e-5 * ref_mse
