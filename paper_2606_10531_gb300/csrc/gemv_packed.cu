@@ -527,6 +527,7 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
 constexpr int kDpMaxTokens = 1;            // two tokens measured slower than the tensor-core kernel
 constexpr int kDpWarps = 16;               // consumer warps (a multiple of 8)
 constexpr int64_t kDpMaxN = 32768;         // integer row sums stay below 2^31
+constexpr int kDpPrefill = 2;              // ring stages filled before the activations are loaded
 constexpr size_t kDpSmemLimit = 227 * 1024;
 
 struct GemvDpParams {
@@ -549,7 +550,7 @@ __host__ __device__ inline DpSmemLayout dp_smem_layout(int R, int stages, int nk
     L.red = L.xq + static_cast<size_t>(nkc) * 1024;
     L.ab = L.red + 2 * kDpWarps * 4;                                 // per-warp max|X| and sum X_g . b
     L.bars = (L.ab + (64 + 8 + 1) * 4 + 15) / 16 * 16;               // A (d x d), b (d), max_k sum_j |A|
-    L.total = L.bars + 2 * kTmaStages * 8;
+    L.total = L.bars + (2 * kTmaStages + 1) * 8;    // full[], empty[], xready
     return L;
 }
 
@@ -589,10 +590,33 @@ __device__ __forceinline__ void dp_word(uint32_t w, const uint4 &xa, const uint4
 template <int D>
 __device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *ab_s, uint8_t *xq_s, float inv, int tile,
                                             int lane, float &r) {
-    const float(&Am)[D * D] = *reinterpret_cast<const float(*)[D * D]>(ab_s);
-    const float(&bv)[D] = *reinterpret_cast<const float(*)[D]>(ab_s + D * D);
+    // X'_g = X_g A, one row of A (16-byte loads from shared memory) at a time, so that the loads of
+    // the next row overlap the FMAs of this one
     float xp[16];
-    xform_block<D>(x, Am, bv, xp, r);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) xp[i] = 0.0f;
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+        float arow[D];
+#pragma unroll
+        for (int h = 0; h < D / 4; ++h) {
+            const float4 v = reinterpret_cast<const float4 *>(ab_s + j * D)[h];
+            arow[4 * h] = v.x; arow[4 * h + 1] = v.y; arow[4 * h + 2] = v.z; arow[4 * h + 3] = v.w;
+        }
+        const float bj = ab_s[D * D + j];
+#pragma unroll
+        for (int g = 0; g < 16 / D; ++g) {
+            const float xj = x[g * D + j];
+            const float2 xx = make_float2(xj, xj);
+#pragma unroll
+            for (int k = 0; k < D; k += 2) {
+                const float2 v = __ffma2_rn(xx, make_float2(arow[k], arow[k + 1]), make_float2(xp[g * D + k], xp[g * D + k + 1]));
+                xp[g * D + k] = v.x;
+                xp[g * D + k + 1] = v.y;
+            }
+            r = fmaf(xj, bj, r);
+        }
+    }
     constexpr int kFirst[8] = {0, 8, 1, 9, 2, 10, 3, 11};
     uint32_t words[8];
 #pragma unroll
@@ -626,6 +650,7 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
     float *ab_s = reinterpret_cast<float *>(base + L.ab);
     uint64_t *full = reinterpret_cast<uint64_t *>(base + L.bars);
     uint64_t *empty = full + kTmaStages;
+    uint64_t *xready = empty + kTmaStages;    // the consumers have loaded X
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t stage_bytes = static_cast<uint32_t>(p.R) * 128u;
     if (threadIdx.x == 0) {
@@ -634,6 +659,7 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], CW);
         }
+        mbar_init(xready, 1);
         fence_barrier_init();
     }
     __syncthreads();
@@ -651,6 +677,10 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
                     if (!mbar_wait(&empty[st], ph ^ 1, p.status)) return;
                     mbar_arrive_expect_tx(&full[st], stage_bytes);
                     tma_load_2d(base + static_cast<size_t>(st) * stage_bytes, &tmC, kc * 128, u * p.R, &full[st]);
+                    // only a short head start of the code stream before the consumers' X loads: a full
+                    // ring in flight delays those loads (measured)
+                    if (u == static_cast<int>(blockIdx.x) && kc == kDpPrefill - 1 && !mbar_wait(xready, 0, p.status))
+                        return;
                     if (++st == p.stages) { st = 0; ph ^= 1; }
                 }
             }
@@ -661,13 +691,14 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
     // -------------------------------------------------------------------- consumers
     const int cw = warp - 1, ct = threadIdx.x - 32;
     const auto bar_consumers = [] { asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory"); };
-    asm volatile("griddepcontrol.wait;" ::: "memory");   // X comes from the previous kernel
+    // A and b are weights like the codes: read before the wait, only X comes from the previous kernel
+    if (ct < p.d * p.d + p.d) ab_s[ct] = ct < p.d * p.d ? __ldg(p.A + ct) : __ldg(p.b + (ct - p.d * p.d));
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     float scale, corr;
     {
         // pass 1: A, b to shared memory; max|X| per warp. Lane l of warp cw reads the 16-column block l
         // of tiles cw, cw + CW, ...; the first block stays in registers for pass 2.
         const int D = p.d;
-        if (ct < D * D + D) ab_s[ct] = ct < D * D ? __ldg(p.A + ct) : __ldg(p.b + (ct - D * D));
         const bool f32in = p.f32in != 0;
         float x0[16];
         float mx = 0.0f;
@@ -683,14 +714,17 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
         for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
         if (lane == 0) red_s[cw] = mx;
         bar_consumers();
+        if (ct == 0) mbar_arrive(xready);
         // pass 2: the token's scale s = max|X| * max_k sum_j |A[j][k]| / 32767 (a bound on max|X'|),
-        // then X' -> int16
-        float xmax = 0.0f, acol = 0.0f;
-        for (int w = 0; w < CW; ++w) xmax = fmaxf(xmax, red_s[w]);
-        for (int k = 0; k < D; ++k) {
-            float cs = 0.0f;
-            for (int j = 0; j < D; ++j) cs += fabsf(ab_s[j * D + k]);
-            acol = fmaxf(acol, cs);
+        // then X' -> int16. Both maxima by warp shuffles (no serial chains of shared-memory loads).
+        float xmax = lane < CW ? red_s[lane] : 0.0f;
+        float acol = 0.0f;
+        if (lane < D) {
+            for (int j = 0; j < D; ++j) acol += fabsf(ab_s[j * D + lane]);
+        }
+        for (int o = 16; o; o >>= 1) {
+            xmax = fmaxf(xmax, __shfl_xor_sync(0xffffffffu, xmax, o));
+            acol = fmaxf(acol, __shfl_xor_sync(0xffffffffu, acol, o));
         }
         const float bound = xmax * acol;
         scale = bound / 32767.0f;
@@ -710,8 +744,8 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
         for (int o = 16; o; o >>= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
         if (lane == 0) red_s[CW + cw] = r;
         bar_consumers();
-        corr = 0.0f;
-        for (int w = 0; w < CW; ++w) corr += red_s[CW + w];
+        corr = lane < CW ? red_s[CW + lane] : 0.0f;
+        for (int o = 16; o; o >>= 1) corr += __shfl_xor_sync(0xffffffffu, corr, o);
     }
 
     // this lane's word in any of its rows: 16-byte chunk (lane / 4) ^ (row % 8), row % 8 = warp % 8
