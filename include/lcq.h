@@ -139,10 +139,13 @@ typedef struct lcq_encode_item {
  * initialisation, per-step requantisation). Every output is exactly the one lcq_encode gives for the
  * same matrix. The matrices share the group size d. When no item asks for the MSE they stream through
  * one persistent launch, so the per-call costs (launch, forming A^{-1}, filling the ring) are paid
- * once for the batch; when any item asks for it, each matrix gets its own launch (measured faster).
+ * once for the batch; when any item asks for it, each matrix gets its own launch (measured faster),
+ * and each launch after the first starts while the previous one drains (programmatic dependent
+ * launch); work enqueued after the call still sees every output.
  *
  * items  host array of `count` matrices, 1 <= count <= LCQ_ENCODE_BATCH_MAX; each item is
- *        validated as lcq_encode validates its arguments.
+ *        validated as lcq_encode validates its arguments. The items must be independent: no item's
+ *        outputs may overlap another item's inputs or outputs.
  * Needs lcq_workspace_size(LCQ_OP_ENCODE_BATCH, count, 0, 0, d) bytes of ws. The workspace header
  * holds one counter per matrix, which returns to zero at the end of every call (the header must be
  * zero before first use). If any A is singular the status word becomes LCQ_ERR_SINGULAR and that

@@ -75,6 +75,37 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int32_
     }
 }
 
+// The same operations on a shared-memory address already converted to 32 bits (hot loops).
+__device__ __forceinline__ void mbar_arrive_u32(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_u32(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+static __device__ __noinline__ bool mbar_wait_slow_u32(uint32_t bar, uint32_t parity, int32_t *status) {
+    const uint64_t t0 = globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait_u32(bar, parity)) return true;
+        if ((it & 63u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
+            set_status(status, LCQ_ERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+// Bounded wait as mbar_wait; the rarely taken retry loop is kept out of line.
+__device__ __forceinline__ bool mbar_wait_u32(uint32_t bar, uint32_t parity, int32_t *status) {
+    if (mbar_try_wait_u32(bar, parity)) return true;
+    return mbar_wait_slow_u32(bar, parity, status);
+}
+
 // ------------------------------------------------------------------ bulk copies (TMA engine)
 
 // 1-D bulk copy global -> shared, completing `bytes` on the mbarrier.

@@ -554,15 +554,12 @@ __host__ __device__ inline DpSmemLayout dp_smem_layout(int R, int stages, int nk
     return L;
 }
 
-__device__ __forceinline__ int32_t dp2a_lo(uint32_t a, uint32_t b, int32_t c) {
-    int32_t d;
-    asm("dp2a.lo.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
-    return d;
+// acc += the two int16 halves of a times bytes 0, 1 (lo) or 2, 3 (hi) of b, accumulated in place
+__device__ __forceinline__ void dp2a_lo(uint32_t a, uint32_t b, int32_t &acc) {
+    asm("dp2a.lo.s32.u32 %0, %1, %2, %0;" : "+r"(acc) : "r"(a), "r"(b));
 }
-__device__ __forceinline__ int32_t dp2a_hi(uint32_t a, uint32_t b, int32_t c) {
-    int32_t d;
-    asm("dp2a.hi.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
-    return d;
+__device__ __forceinline__ void dp2a_hi(uint32_t a, uint32_t b, int32_t &acc) {
+    asm("dp2a.hi.s32.u32 %0, %1, %2, %0;" : "+r"(acc) : "r"(a), "r"(b));
 }
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     uint4 v;
@@ -574,14 +571,14 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
 __device__ __forceinline__ void dp_word(uint32_t w, const uint4 &xa, const uint4 &xb, int32_t &acc0, int32_t &acc1) {
     const uint32_t w4 = w >> 4;
     const uint32_t s0 = w & 0x03030303u, s1 = w & 0x0C0C0C0Cu, s2 = w4 & 0x03030303u, s3 = w4 & 0x0C0C0C0Cu;
-    acc0 = dp2a_lo(xa.x, s0, acc0);
-    acc1 = dp2a_hi(xa.y, s0, acc1);
-    acc0 = dp2a_lo(xa.z, s1, acc0);
-    acc1 = dp2a_hi(xa.w, s1, acc1);
-    acc0 = dp2a_lo(xb.x, s2, acc0);
-    acc1 = dp2a_hi(xb.y, s2, acc1);
-    acc0 = dp2a_lo(xb.z, s3, acc0);
-    acc1 = dp2a_hi(xb.w, s3, acc1);
+    dp2a_lo(xa.x, s0, acc0);
+    dp2a_hi(xa.y, s0, acc1);
+    dp2a_lo(xa.z, s1, acc0);
+    dp2a_hi(xa.w, s1, acc1);
+    dp2a_lo(xb.x, s2, acc0);
+    dp2a_hi(xb.y, s2, acc1);
+    dp2a_lo(xb.z, s3, acc0);
+    dp2a_hi(xb.w, s3, acc1);
 }
 
 // int16 activations of one 16-column block (lane l of tile `tile`): X' = X_g A, scaled by inv
@@ -752,27 +749,38 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
     const int lane_word = (((lane >> 2) ^ (cw & 7)) << 2) + (lane & 3);
     const uint32_t *ring_w = reinterpret_cast<const uint32_t *>(base) + cw * 32 + lane_word;
     const uint4 *xq_v = reinterpret_cast<const uint4 *>(base + L.xq) + lane;
+    // per-tile bookkeeping kept to a minimum (the loop is issue-bound): barrier addresses as 32-bit
+    // shared addresses, the tile pointer advanced instead of recomputed
+    const uint32_t full_a = smem_u32(full), empty_a = smem_u32(empty);
     int st = 0;
     uint32_t ph = 0;
+    const uint32_t *tile = ring_w;
     bool ok = true;
     for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
         int32_t acc[RPT][2];
 #pragma unroll
         for (int j = 0; j < RPT; ++j) acc[j][0] = acc[j][1] = 0;
 
+        const uint4 *xv = xq_v;
         for (int kc = 0; kc < p.nkc; ++kc) {
             // this lane's 16 activation columns of tile kc (fetched before waiting for the code tile)
-            const uint4 xa = xq_v[kc * 64], xb = xq_v[kc * 64 + 32];
-            if (!mbar_wait(&full[st], ph, p.status)) { ok = false; break; }
-            const uint32_t *tile = ring_w + static_cast<size_t>(st) * (RPT * CW * 32);
+            const uint4 xa = xv[0], xb = xv[32];
+            xv += 64;
+            if (!mbar_wait_u32(full_a + 8u * st, ph, p.status)) { ok = false; break; }
             uint32_t w[RPT];
 #pragma unroll
             for (int j = 0; j < RPT; ++j) w[j] = tile[j * CW * 32];
 #pragma unroll
             for (int j = 0; j < RPT; ++j) dp_word(w[j], xa, xb, acc[j][0], acc[j][1]);
             __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[st]);
-            if (++st == p.stages) { st = 0; ph ^= 1; }
+            if (lane == 0) mbar_arrive_u32(empty_a + 8u * st);
+            if (++st == p.stages) {
+                st = 0;
+                ph ^= 1;
+                tile = ring_w;
+            } else {
+                tile += RPT * CW * 32;
+            }
         }
         if (!ok) break;
         // sum the 32 lanes of each row (exact integer warp reductions: each accumulator covers half the

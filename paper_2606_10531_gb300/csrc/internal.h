@@ -26,6 +26,10 @@ struct EncodeArgs {
     double *partials;     // [grid] per-CTA sums of squared residuals
     unsigned *counter;    // zero between calls: the last CTA wraps it back (atomicInc)
     int32_t *status;
+    // programmatic dependent launch inside lcq_encode_batch (independent matrices): bit 0 = let the
+    // next launch start early, bit 1 = launched early (waits for the previous grid before it exits,
+    // so completion stays in stream order). 0 for a single lcq_encode.
+    int pdl = 0;
 };
 
 constexpr int kEncodeBatchMax = 16;   // = LCQ_ENCODE_BATCH_MAX

@@ -271,9 +271,11 @@ encode_kernel(EncodeArgs a) {
     if (threadIdx.x < D * D) s.A[threadIdx.x] = a.A[threadIdx.x];
     if (threadIdx.x < D) s.b[threadIdx.x] = a.b[threadIdx.x];
     __syncthreads();
+    if (a.pdl & 1) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == 0) {
         if (lane == 0) stream_producer(s, a.W, total, a.status);
+        if (a.pdl & 2) asm volatile("griddepcontrol.wait;" ::: "memory");
         return;
     }
     // compute warps
@@ -301,6 +303,7 @@ encode_kernel(EncodeArgs a) {
         if (lane == 0) mbar_arrive(&s.empty[st]);
     }
     if (kMse) mse_flush(sq, s.dred, a.partials, a.counter, a.mse, total);
+    if (a.pdl & 2) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // ------------------------------------------------------------------ batched encode (codes, latents)
@@ -726,10 +729,25 @@ cudaError_t launch_encode(const EncodeArgs &a, int d, int num_sms, cudaStream_t 
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     trace_begin(LCQ_K_ENCODE, st);
-    k<<<grid, kStreamThreads, smem, st>>>(a);
+    if (a.pdl & 2) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(kStreamThreads);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, k, a);
+    } else {
+        k<<<grid, kStreamThreads, smem, st>>>(a);
+        e = cudaSuccess;
+    }
     trace_end(LCQ_K_ENCODE, st);
     count_launch();
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 int64_t encode_chunk_size() { return kChunk; }
@@ -743,22 +761,32 @@ cudaError_t launch_encode_batch(const EncodeBatchArgs &a, int d, int num_sms, cu
     if (mse) {
         // With the reconstruction MSE, the single-matrix kernel measured faster per matrix than the
         // fused batch kernel (whose MSE variant compiles to ~25% more instructions per group), so each
-        // matrix gets its own launch, with its own partials and counter in the batch workspace.
+        // matrix gets its own launch, with its own partials and counter in the batch workspace. The
+        // matrices are independent, so each launch after the first is a programmatic dependent launch
+        // that starts as the previous one drains; the last one does not let anything start early, so
+        // the work after the batch sees all of it.
+        int last = -1;
         for (int i = 0; i < a.count; ++i) {
             const EncodeBatchItem &it = a.item[i];
-            if (it.m * it.n == 0) {
-                if (it.mse) {
-                    const cudaError_t e = cudaMemsetAsync(it.mse, 0, sizeof(double), st);
-                    if (e != cudaSuccess) return e;
-                }
-                continue;
+            if (it.m * it.n != 0) {
+                last = i;
+            } else if (it.mse) {
+                const cudaError_t e = cudaMemsetAsync(it.mse, 0, sizeof(double), st);
+                if (e != cudaSuccess) return e;
             }
+        }
+        bool first = true;
+        for (int i = 0; i < a.count; ++i) {
+            const EncodeBatchItem &it = a.item[i];
+            if (it.m * it.n == 0) continue;
             EncodeArgs e;
             e.W = it.W; e.m = it.m; e.n = it.n; e.A = it.A; e.b = it.b;
             e.packed = it.packed; e.codes = it.codes; e.latent = it.latent; e.mse = it.mse;
             e.partials = a.partials + static_cast<int64_t>(i) * kEncodeBatchPartials;
             e.counter = a.counters + i;
             e.status = a.status;
+            e.pdl = (i != last ? 1 : 0) | (first ? 0 : 2);
+            first = false;
             const cudaError_t r = launch_encode(e, d, num_sms, st);
             if (r != cudaSuccess) return r;
         }
