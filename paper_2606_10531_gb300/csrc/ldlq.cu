@@ -214,18 +214,21 @@ cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
 // ================================================================== sweep
 
 constexpr int kSwR = 64;              // rows per CTA
-constexpr int kSwC = 128;             // columns per chunk (4 slices of 32)
-constexpr int kSwBK = 32;             // rows of U / of the error history per ring stage
+constexpr int kSwC = 256;             // columns per chunk (8 slices of 32)
+constexpr int kSwBK = 16;             // rows of U / of the error history per ring stage
 constexpr int kSwStages = 4;
 constexpr int kSwWarps = 8;           // compute warps; + 1 producer warp
 constexpr int kSwThreads = 32 * (kSwWarps + 1);
+constexpr int kSwS = 32;              // columns of a rounding slice: warp q rounds slice q
+constexpr int kSwSlices = kSwC / kSwS;
 constexpr int kSwTLd = kSwC + 4;      // padded row of the target tile (conflict-free 16-byte access)
+static_assert(kSwSlices == kSwWarps, "one rounding slice per compute warp");
 
 struct SweepSmem {
-    float ring_u[kSwStages][kSwBK][kSwC];    // U[k0 .. k0+31][c0 .. c0+127]
-    float ring_e[kSwStages][kSwBK][kSwR];    // E[k0 .. k0+31][64 rows] (history, k-major)
-    float W[kSwC / 32][kSwR][32];            // the chunk's weights: one 128B-swizzled box per slice
-    float T[kSwR][kSwTLd];                   // targets minus weights, then the errors
+    float ring_u[kSwStages][kSwBK][kSwC];    // U[k0 .. k0+15][c0 .. c0+255]
+    float ring_e[kSwStages][kSwBK][kSwR];    // E[k0 .. k0+15][64 rows] (history, k-major)
+    float W[kSwSlices][kSwR][32];            // the chunk's weights: one 128B-swizzled box per slice
+    float T[kSwR][kSwTLd];                   // feedback of the earlier chunks, then targets - weights, then errors
     float A[64], Ainv[64], b[8];
     InvScratch inv;
     double red[kSwWarps];
@@ -235,14 +238,19 @@ struct SweepSmem {
 __device__ __forceinline__ void sweep_bar() {
     asm volatile("bar.sync 1, %0;" ::"r"(32 * kSwWarps) : "memory");
 }
-// the warps taking part in the errors of slice s: warps 2s .. 7
+// the warps taking part in the errors of slice s: warps s .. 7
 __device__ __forceinline__ void slice_bar(int s) {
-    asm volatile("bar.sync %0, %1;" ::"r"(2 + s), "r"(32 * (kSwWarps - 2 * s)) : "memory");
+    asm volatile("bar.sync %0, %1;" ::"r"(2 + s), "r"(32 * (kSwWarps - s)) : "memory");
 }
 // shared-memory load the compiler must not hoist (keeps the d x d constants out of registers)
 __device__ __forceinline__ float lds_nohoist(const float *p) {
     float v;
     asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(smem_u32(p)));
+    return v;
+}
+__device__ __forceinline__ float4 lds4_nohoist(const float *p) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(smem_u32(p)));
     return v;
 }
 __device__ __forceinline__ void fence_proxy_async_global() {
@@ -325,11 +333,9 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
     if (tid == 0 && s.inv.singular && blockIdx.x == 0) set_status(p.status, LCQ_ERR_SINGULAR);
     sweep_bar();
 
-    const int ty = tid >> 4, tx = tid & 15;           // feedback GEMM: rows 4ty.., cols 4tx.. and 64+4tx..
-    const int q = warp >> 1, r = (warp & 1) * 32 + lane;   // rounding: row r, slice q (columns 32q .. 32q+31)
-    const int64_t grow = tile * kSwR + r;
-    const bool row_ok = grow < p.m;
-    float *trow = &s.T[r][0];
+    // feedback GEMM: warp w computes rows 8w .. 8w+7, lane l columns 4l .. 4l+3 and 128+4l .. 128+4l+3.
+    // rounding: warp q owns slice q (columns 32q .. 32q+31) of rows l and l + 32.
+    const int q = warp;
     int st = 0;
     uint32_t ph = 0;
     bool ok = true;
@@ -338,26 +344,27 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
     for (int c = 0; c < nchunks; ++c) {
         const int c0 = c * kSwC;
         const int cw = static_cast<int>(n - c0 < kSwC ? n - c0 : kSwC);
-        const int col0 = c0 + 32 * q;                  // this thread's first column
+        const int col0 = c0 + kSwS * q;                // this thread's first column
         // feedback of the earlier chunks: F = E_{<c0} U_{<c0, chunk}, packed fp32 FMAs (two columns each)
-        float2 acc[4][4];
+        float2 acc[8][4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
+        for (int i = 0; i < 8; ++i)
 #pragma unroll
             for (int j = 0; j < 4; ++j) acc[i][j] = make_float2(0.0f, 0.0f);
         for (int k0 = 0; k0 < c0; k0 += kSwBK) {
             if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
             if (ok) {
-#pragma unroll 8
+#pragma unroll 4
                 for (int kk = 0; kk < kSwBK; ++kk) {
-                    const float4 a = *reinterpret_cast<const float4 *>(&s.ring_e[st][kk][4 * ty]);
-                    const float4 b0 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][4 * tx]);
-                    const float4 b1 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][64 + 4 * tx]);
-                    const float av[4] = {a.x, a.y, a.z, a.w};
+                    const float4 a0 = *reinterpret_cast<const float4 *>(&s.ring_e[st][kk][8 * warp]);
+                    const float4 a1 = *reinterpret_cast<const float4 *>(&s.ring_e[st][kk][8 * warp + 4]);
+                    const float4 b0 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][4 * lane]);
+                    const float4 b1 = *reinterpret_cast<const float4 *>(&s.ring_u[st][kk][128 + 4 * lane]);
+                    const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
                     const float2 bv[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
                                           make_float2(b1.z, b1.w)};
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
+                    for (int i = 0; i < 8; ++i) {
                         const float2 ai = make_float2(av[i], av[i]);
 #pragma unroll
                         for (int j = 0; j < 4; ++j) acc[i][j] = __ffma2_rn(ai, bv[j], acc[i][j]);
@@ -370,149 +377,217 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         }
         sweep_bar();                                   // the previous chunk's readers of T are done
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][4 * tx]) = make_float4(acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y);
-            *reinterpret_cast<float4 *>(&s.T[4 * ty + i][64 + 4 * tx]) = make_float4(acc[i][2].x, acc[i][2].y, acc[i][3].x, acc[i][3].y);
+        for (int i = 0; i < 8; ++i) {
+            *reinterpret_cast<float4 *>(&s.T[8 * warp + i][4 * lane]) = make_float4(acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y);
+            *reinterpret_cast<float4 *>(&s.T[8 * warp + i][128 + 4 * lane]) = make_float4(acc[i][2].x, acc[i][2].y, acc[i][3].x, acc[i][3].y);
         }
         sweep_bar();
         if (ok && !mbar_wait(&s.wfull, c & 1, p.status)) ok = false;
-        uint32_t bits0 = 0, bits1 = 0;
+        uint32_t bits[2][2] = {{0u, 0u}, {0u, 0u}};
         float csq = 0.0f;
-        // the chunk's slices in order: slice s is rounded by warps 2s, 2s+1 (its columns are theirs), in
-        // place in T (target - weight -> error); its errors then reach the later slices through U's
-        // diagonal block
-        for (int sl = 0; sl * 32 < cw; ++sl) {
+        // the chunk's slices in order: slice s (its 32 rows of U's diagonal block in one or two ring
+        // stages) is rounded by warp s in place in T (target - weight -> error); its errors then reach
+        // the later slices through U's diagonal block
+        for (int sl = 0; sl * kSwS < cw; ++sl) {
+            const int span = cw - kSwS * sl < kSwS ? cw - kSwS * sl : kSwS;   // valid columns of the slice
+            const int nst = (span + kSwBK - 1) / kSwBK;
+            const int stA = st;
             if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
-            const float(*Us)[kSwC] = s.ring_u[st];
+            if (++st == kSwStages) { st = 0; ph ^= 1; }
+            int stB = stA;
+            if (nst == 2) {
+                stB = st;
+                if (ok && !mbar_wait(&s.full[st], ph, p.status)) ok = false;
+                if (++st == kSwStages) { st = 0; ph ^= 1; }
+            }
+            // row i (0 .. 31) of the slice in U's diagonal block
+            const auto urow = [&](int i) -> const float * {
+                return i < kSwBK ? &s.ring_u[stA][i][0] : &s.ring_u[stB][i - kSwBK][0];
+            };
             if (q == sl) {
-                float4 *t4 = reinterpret_cast<float4 *>(trow + 32 * sl);
+                // both rows of this lane, group by group; each row of A^{-1} and A is loaded once (16-byte
+                // shared-memory loads) for the two rows
+                float4 *t4[2] = {reinterpret_cast<float4 *>(&s.T[lane][kSwS * sl]),
+                                 reinterpret_cast<float4 *>(&s.T[lane + 32][kSwS * sl])};
+                float bb[D];
+#pragma unroll
+                for (int hh = 0; hh < D / 4; ++hh) {
+                    const float4 v = lds4_nohoist(&s.b[4 * hh]);
+                    bb[4 * hh] = v.x; bb[4 * hh + 1] = v.y; bb[4 * hh + 2] = v.z; bb[4 * hh + 3] = v.w;
+                }
 #pragma unroll 1
-                for (int j = 0; j < 32 / D; ++j) {
-                    float t[D], w[D];
+                for (int j = 0; j < span / D; ++j) {
+                    float tb[2][D], w[2][D];
 #pragma unroll
-                    for (int h = 0; h < D / 4; ++h) {
-                        const float4 fv = t4[j * (D / 4) + h];
-                        const float4 wv = *swz128(s.W[sl], r, j * (D / 4) + h);
-                        w[4 * h] = wv.x; w[4 * h + 1] = wv.y; w[4 * h + 2] = wv.z; w[4 * h + 3] = wv.w;
-                        t[4 * h] = wv.x + fv.x; t[4 * h + 1] = wv.y + fv.y; t[4 * h + 2] = wv.z + fv.z; t[4 * h + 3] = wv.w + fv.w;
+                    for (int rr = 0; rr < 2; ++rr) {
+                        const int r = lane + 32 * rr;
+#pragma unroll
+                        for (int hh = 0; hh < D / 4; ++hh) {
+                            const float4 fv = t4[rr][j * (D / 4) + hh];
+                            const float4 wv = *swz128(s.W[sl], r, j * (D / 4) + hh);
+                            w[rr][4 * hh] = wv.x; w[rr][4 * hh + 1] = wv.y; w[rr][4 * hh + 2] = wv.z; w[rr][4 * hh + 3] = wv.w;
+                            tb[rr][4 * hh] = (wv.x + fv.x) - bb[4 * hh];
+                            tb[rr][4 * hh + 1] = (wv.y + fv.y) - bb[4 * hh + 1];
+                            tb[rr][4 * hh + 2] = (wv.z + fv.z) - bb[4 * hh + 2];
+                            tb[rr][4 * hh + 3] = (wv.w + fv.w) - bb[4 * hh + 3];
+                        }
                     }
-                    float u[D], e[D];
+                    // u = A^{-1} (t - b) and z = clip(round(u), 0, 3)
+                    float u[2][D];
+                    uint32_t z[2][D];
 #pragma unroll
                     for (int i = 0; i < D; ++i) {
-                        float v = 0.0f;
+                        float ar[D];
 #pragma unroll
-                        for (int jj = 0; jj < D; ++jj) v = fmaf(lds_nohoist(&s.Ainv[i * D + jj]), t[jj] - lds_nohoist(&s.b[jj]), v);
-                        u[i] = v;
+                        for (int hh = 0; hh < D / 4; ++hh) {
+                            const float4 v = lds4_nohoist(&s.Ainv[i * D + 4 * hh]);
+                            ar[4 * hh] = v.x; ar[4 * hh + 1] = v.y; ar[4 * hh + 2] = v.z; ar[4 * hh + 3] = v.w;
+                        }
+#pragma unroll
+                        for (int rr = 0; rr < 2; ++rr) {
+                            float v = 0.0f;
+#pragma unroll
+                            for (int jj = 0; jj < D; ++jj) v = fmaf(ar[jj], tb[rr][jj], v);
+                            u[rr][i] = v;
+                            z[rr][i] = round_clamp3(v);
+                        }
                     }
-                    uint32_t z[D];
-#pragma unroll
-                    for (int i = 0; i < D; ++i) z[i] = round_clamp3(u[i]);
-                    if (p.latent && row_ok && col0 + j * D < n) {
-#pragma unroll
-                        for (int i = 0; i < D; ++i) p.latent[grow * n + col0 + j * D + i] = u[i];
-                    }
+                    // e = w - (A z + b)
+                    float e[2][D];
 #pragma unroll
                     for (int i = 0; i < D; ++i) {
-                        float wh = lds_nohoist(&s.b[i]);
+                        float ar[D];
 #pragma unroll
-                        for (int jj = 0; jj < D; ++jj) wh = fmaf(lds_nohoist(&s.A[i * D + jj]), static_cast<float>(z[jj]), wh);
-                        e[i] = w[i] - wh;
+                        for (int hh = 0; hh < D / 4; ++hh) {
+                            const float4 v = lds4_nohoist(&s.A[i * D + 4 * hh]);
+                            ar[4 * hh] = v.x; ar[4 * hh + 1] = v.y; ar[4 * hh + 2] = v.z; ar[4 * hh + 3] = v.w;
+                        }
+#pragma unroll
+                        for (int rr = 0; rr < 2; ++rr) {
+                            float wh = bb[i];
+#pragma unroll
+                            for (int jj = 0; jj < D; ++jj) wh = fmaf(ar[jj], static_cast<float>(z[rr][jj]), wh);
+                            e[rr][i] = w[rr][i] - wh;
+                        }
                     }
-                    uint32_t zb = 0;
 #pragma unroll
-                    for (int i = 0; i < D; ++i) zb |= z[i] << (2 * i);
-                    const int sh = 2 * ((j * D) & 15);
-                    if (j * D < 16) bits0 |= zb << sh;
-                    else bits1 |= zb << sh;
-                    if (col0 + j * D < n) {
+                    for (int rr = 0; rr < 2; ++rr) {
+                        const int64_t grow = tile * kSwR + lane + 32 * rr;
+                        if (p.latent && grow < p.m) {
 #pragma unroll
-                        for (int i = 0; i < D; ++i) csq = fmaf(e[i], e[i], csq);
+                            for (int i = 0; i < D; ++i) p.latent[grow * n + col0 + j * D + i] = u[rr][i];
+                        }
+                        uint32_t zb = 0;
+#pragma unroll
+                        for (int i = 0; i < D; ++i) zb |= z[rr][i] << (2 * i);
+                        bits[rr][(j * D) >> 4] |= zb << (2 * ((j * D) & 15));
+                        if (grow < p.m) {
+#pragma unroll
+                            for (int i = 0; i < D; ++i) csq = fmaf(e[rr][i], e[rr][i], csq);
+                        }
+#pragma unroll
+                        for (int hh = 0; hh < D / 4; ++hh)
+                            t4[rr][j * (D / 4) + hh] = make_float4(e[rr][4 * hh], e[rr][4 * hh + 1], e[rr][4 * hh + 2], e[rr][4 * hh + 3]);
                     }
-#pragma unroll
-                    for (int h = 0; h < D / 4; ++h)
-                        t4[j * (D / 4) + h] = make_float4(e[4 * h], e[4 * h + 1], e[4 * h + 2], e[4 * h + 3]);
-                    // later groups of this slice, 16 bytes of the row at a time
-                    for (int c4 = (j + 1) * (D / 4); c4 < 8; ++c4) {
-                        float4 v = t4[c4];
+                    // later groups of this slice, 16 bytes of the rows at a time (U shared by the two rows)
+                    for (int c4 = (j + 1) * (D / 4); c4 < span / 4; ++c4) {
+                        float4 v0 = t4[0][c4], v1 = t4[1][c4];
 #pragma unroll
                         for (int i = 0; i < D; ++i) {
-                            const float4 uv = *reinterpret_cast<const float4 *>(&Us[j * D + i][32 * sl + 4 * c4]);
-                            v.x = fmaf(e[i], uv.x, v.x);
-                            v.y = fmaf(e[i], uv.y, v.y);
-                            v.z = fmaf(e[i], uv.z, v.z);
-                            v.w = fmaf(e[i], uv.w, v.w);
+                            const float4 uv = *reinterpret_cast<const float4 *>(urow(j * D + i) + kSwS * sl + 4 * c4);
+                            v0.x = fmaf(e[0][i], uv.x, v0.x); v0.y = fmaf(e[0][i], uv.y, v0.y);
+                            v0.z = fmaf(e[0][i], uv.z, v0.z); v0.w = fmaf(e[0][i], uv.w, v0.w);
+                            v1.x = fmaf(e[1][i], uv.x, v1.x); v1.y = fmaf(e[1][i], uv.y, v1.y);
+                            v1.z = fmaf(e[1][i], uv.z, v1.z); v1.w = fmaf(e[1][i], uv.w, v1.w);
                         }
-                        t4[c4] = v;
+                        t4[0][c4] = v0;
+                        t4[1][c4] = v1;
                     }
                 }
             }
-            if (sl < kSwC / 32 - 1 && q >= sl) slice_bar(sl);
+            if (sl < kSwSlices - 1 && q >= sl) slice_bar(sl);
             if (q > sl) {
-                // T[r][this slice] += e_slice U[slice rows][this thread's columns]
-                float acc2[32];
-                const float4 *own = reinterpret_cast<const float4 *>(trow + 32 * q);
+                // T[r][this slice] += e_slice U[slice rows][this thread's columns], both rows per U load
+                float2 acc2[2][kSwS / 2];
 #pragma unroll
-                for (int c4 = 0; c4 < 8; ++c4) {
-                    const float4 v = own[c4];
-                    acc2[4 * c4] = v.x; acc2[4 * c4 + 1] = v.y; acc2[4 * c4 + 2] = v.z; acc2[4 * c4 + 3] = v.w;
+                for (int rr = 0; rr < 2; ++rr) {
+                    const float4 *own = reinterpret_cast<const float4 *>(&s.T[lane + 32 * rr][kSwS * q]);
+#pragma unroll
+                    for (int c4 = 0; c4 < kSwS / 4; ++c4) {
+                        const float4 v = own[c4];
+                        acc2[rr][2 * c4] = make_float2(v.x, v.y);
+                        acc2[rr][2 * c4 + 1] = make_float2(v.z, v.w);
+                    }
                 }
-                const float4 *es = reinterpret_cast<const float4 *>(trow + 32 * sl);
 #pragma unroll 1
-                for (int i4 = 0; i4 < 8; ++i4) {
-                    const float4 e4 = es[i4];
-                    const float ev[4] = {e4.x, e4.y, e4.z, e4.w};
+                for (int i4 = 0; i4 < span / 4; ++i4) {
+                    const float4 e0 = reinterpret_cast<const float4 *>(&s.T[lane][kSwS * sl])[i4];
+                    const float4 e1 = reinterpret_cast<const float4 *>(&s.T[lane + 32][kSwS * sl])[i4];
+                    const float ev0[4] = {e0.x, e0.y, e0.z, e0.w}, ev1[4] = {e1.x, e1.y, e1.z, e1.w};
 #pragma unroll
                     for (int ii = 0; ii < 4; ++ii) {
-                        const float4 *urow = reinterpret_cast<const float4 *>(&Us[4 * i4 + ii][32 * q]);
+                        const float4 *ur = reinterpret_cast<const float4 *>(urow(4 * i4 + ii) + kSwS * q);
+                        const float2 x0 = make_float2(ev0[ii], ev0[ii]), x1 = make_float2(ev1[ii], ev1[ii]);
 #pragma unroll
-                        for (int c4 = 0; c4 < 8; ++c4) {
-                            const float4 uv = urow[c4];
-                            acc2[4 * c4] = fmaf(ev[ii], uv.x, acc2[4 * c4]);
-                            acc2[4 * c4 + 1] = fmaf(ev[ii], uv.y, acc2[4 * c4 + 1]);
-                            acc2[4 * c4 + 2] = fmaf(ev[ii], uv.z, acc2[4 * c4 + 2]);
-                            acc2[4 * c4 + 3] = fmaf(ev[ii], uv.w, acc2[4 * c4 + 3]);
+                        for (int c4 = 0; c4 < kSwS / 4; ++c4) {
+                            const float4 uv = ur[c4];
+                            const float2 ua = make_float2(uv.x, uv.y), ub = make_float2(uv.z, uv.w);
+                            acc2[0][2 * c4] = __ffma2_rn(x0, ua, acc2[0][2 * c4]);
+                            acc2[0][2 * c4 + 1] = __ffma2_rn(x0, ub, acc2[0][2 * c4 + 1]);
+                            acc2[1][2 * c4] = __ffma2_rn(x1, ua, acc2[1][2 * c4]);
+                            acc2[1][2 * c4 + 1] = __ffma2_rn(x1, ub, acc2[1][2 * c4 + 1]);
                         }
                         asm volatile("" ::: "memory");
                     }
                 }
-                float4 *ownw = reinterpret_cast<float4 *>(trow + 32 * q);
 #pragma unroll
-                for (int c4 = 0; c4 < 8; ++c4)
-                    ownw[c4] = make_float4(acc2[4 * c4], acc2[4 * c4 + 1], acc2[4 * c4 + 2], acc2[4 * c4 + 3]);
+                for (int rr = 0; rr < 2; ++rr) {
+                    float4 *ownw = reinterpret_cast<float4 *>(&s.T[lane + 32 * rr][kSwS * q]);
+#pragma unroll
+                    for (int c4 = 0; c4 < kSwS / 4; ++c4)
+                        ownw[c4] = make_float4(acc2[rr][2 * c4].x, acc2[rr][2 * c4].y, acc2[rr][2 * c4 + 1].x, acc2[rr][2 * c4 + 1].y);
+                }
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(&s.empty[st]);
-            if (++st == kSwStages) { st = 0; ph ^= 1; }
+            if (lane == 0) {
+                mbar_arrive(&s.empty[stA]);
+                if (nst == 2) mbar_arrive(&s.empty[stB]);
+            }
         }
         // this thread's columns: error history (k-major) from T, codes
         if (col0 < n) {
-            float *Eh = p.E + (tile * n + col0) * kSwR + r;
-            const float4 *ev = reinterpret_cast<const float4 *>(trow + 32 * q);
 #pragma unroll
-            for (int c4 = 0; c4 < 8; ++c4) {
-                if (col0 + 4 * c4 >= n) break;
-                const float4 v = ev[c4];
-                Eh[(4 * c4 + 0) * kSwR] = v.x;
-                Eh[(4 * c4 + 1) * kSwR] = v.y;
-                Eh[(4 * c4 + 2) * kSwR] = v.z;
-                Eh[(4 * c4 + 3) * kSwR] = v.w;
-            }
-            if (row_ok && p.packed) {
-                uint8_t *pk = p.packed + grow * (n / 4) + col0 / 4;
-                if (col0 + 32 <= n && (reinterpret_cast<uintptr_t>(pk) & 7u) == 0) {
-                    *reinterpret_cast<uint2 *>(pk) = make_uint2(bits0, bits1);
-                } else {
-                    for (int i = 0; i < 32 && col0 + i < n; i += 4)
-                        pk[i / 4] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 0xFFu);
+            for (int rr = 0; rr < 2; ++rr) {
+                const int r = lane + 32 * rr;
+                const int64_t grow = tile * kSwR + r;
+                float *Eh = p.E + (tile * n + col0) * kSwR + r;
+                const float4 *ev = reinterpret_cast<const float4 *>(&s.T[r][kSwS * q]);
+#pragma unroll
+                for (int c4 = 0; c4 < kSwS / 4; ++c4) {
+                    if (col0 + 4 * c4 >= n) break;
+                    const float4 v = ev[c4];
+                    Eh[(4 * c4 + 0) * kSwR] = v.x;
+                    Eh[(4 * c4 + 1) * kSwR] = v.y;
+                    Eh[(4 * c4 + 2) * kSwR] = v.z;
+                    Eh[(4 * c4 + 3) * kSwR] = v.w;
+                }
+                if (grow < p.m && p.packed) {
+                    uint8_t *pk = p.packed + grow * (n / 4) + col0 / 4;
+                    if (col0 + kSwS <= n && (reinterpret_cast<uintptr_t>(pk) & 7u) == 0) {
+                        *reinterpret_cast<uint2 *>(pk) = make_uint2(bits[rr][0], bits[rr][1]);
+                    } else {
+                        for (int i = 0; i < kSwS && col0 + i < n; i += 4)
+                            pk[i / 4] = static_cast<uint8_t>((bits[rr][i >> 4] >> (2 * (i & 15))) & 0xFFu);
+                    }
+                }
+                if (grow < p.m && p.codes) {
+                    uint8_t *cd = p.codes + grow * n + col0;
+                    for (int i = 0; i < kSwS && col0 + i < n; ++i)
+                        cd[i] = static_cast<uint8_t>((bits[rr][i >> 4] >> (2 * (i & 15))) & 3u);
                 }
             }
-            if (row_ok && p.codes) {
-                uint8_t *cd = p.codes + grow * n + col0;
-                for (int i = 0; i < 32 && col0 + i < n; ++i)
-                    cd[i] = static_cast<uint8_t>(((i < 16 ? bits0 : bits1) >> (2 * (i & 15))) & 3u);
-            }
         }
-        if (row_ok) sq += static_cast<double>(csq);
+        sq += static_cast<double>(csq);
         fence_proxy_async_global();
         mbar_arrive(&s.edone);
     }
