@@ -6,18 +6,18 @@
 // so the integer codes themselves are the weight operand and A acts on the few activation rows.
 //
 // prep kernel  (256 16-column blocks per CTA): X' in bf16, written in the column order and scale
-//              the main kernel's register fragments expect, and per-CTA partials of the per-token
-//              constant corr[t].
+//              the main kernel's register fragments expect (tile-major for the tma variant), and
+//              per-CTA partials of the per-token constant corr[t].
 // main kernel  streams the codes once from HBM, turns each 32-bit word of 16 codes into eight
 //              bf16x2 tensor-core fragments with one LOP3 each (no table) and accumulates with
 //              mma.sync m16n8k16 (16 rows of W x 8 tokens). The codes operand is converted in
 //              registers, so the bandwidth-bound stream never round-trips through a bf16 copy.
 //   tma variant (n % 64 == 0): persistent CTAs; one producer thread streams (rows x 512 columns)
-//              code tiles through an 8-stage shared-memory ring with 2-D TMA copies (128-byte
-//              swizzle, bank-conflict-free fragment reads); eight consumer warps each own a 64-column
-//              slice of every tile and reuse its activation fragments over all rows of the unit.
-//              Launched with programmatic dependent launch so the code stream starts while the
-//              prep kernel still runs; consumers wait for it (griddepcontrol.wait) before reading X'.
+//              code tiles, each with the tile's 512 columns of X' (one bulk copy), through a
+//              shared-memory ring (2-D TMA copies, 128-byte swizzle, bank-conflict-free fragment
+//              reads); each consumer warp owns whole rows of the unit over all columns, so a row's
+//              sum stays in registers. Launched with programmatic dependent launch so the code
+//              stream starts while the prep kernel still runs; the X' copies wait for it.
 //   generic variant: plain 16-byte loads (byte loads at a ragged row end), any n % 8 == 0.
 //
 // Code -> bf16 conversion: OR-ing a 2-bit field into the mantissa of bf16 128.0 (0x4300) gives
@@ -37,6 +37,9 @@ constexpr int kGemvWarps = 8;                     // generic variant: K is split
 constexpr int kSuper = 256;                       // generic variant: columns per warp step
 constexpr int kPadCols = 512;                     // X' rows are zero-padded to a multiple of this
 constexpr int kPrepCols = 4096;                   // columns per prep CTA (256 threads x 16)
+constexpr int kTmaStages = 8;                     // ring stages (at most)
+constexpr int kTileCols = 512;                    // 128 bytes of codes per row per stage
+constexpr size_t kGemvSmemLimit = 227 * 1024;
 
 __host__ __device__ inline int64_t gemv_npad(int64_t n) { return (n + kPadCols - 1) / kPadCols * kPadCols; }
 __host__ __device__ inline int64_t gemv_nprep(int64_t n) { return (gemv_npad(n) + kPrepCols - 1) / kPrepCols; }
@@ -123,7 +126,9 @@ __device__ __forceinline__ void block_sum_256(float v, float *out) {
     }
 }
 
-template <int D, bool F32IN>
+// TILED: X' in the tile-major order of the TMA variant ([npad / 512][N][512], 16-byte chunks of a
+// token's tile row permuted as its consumers read them); otherwise [N][npad] in block order.
+template <int D, bool F32IN, bool TILED>
 __global__ void __launch_bounds__(256)
 gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const float *__restrict__ A,
                  const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ corrpart) {
@@ -135,7 +140,6 @@ gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const flo
     for (int i = 0; i < D * D; ++i) Am[i] = __ldg(A + i);
 #pragma unroll
     for (int i = 0; i < D; ++i) bv[i] = __ldg(b + i);
-    uint32_t *out = reinterpret_cast<uint32_t *>(Xp + t * npad);
     float S = 0.0f, r = 0.0f;
     const int64_t blk = static_cast<int64_t>(blockIdx.y) * 256 + threadIdx.x;
     if (blk < npad / 16) {
@@ -151,9 +155,21 @@ gemv_prep_kernel(const void *__restrict__ Xv, int64_t n, int64_t npad, const flo
             words[k] = static_cast<uint32_t>(*reinterpret_cast<const uint16_t *>(&lo)) |
                        (static_cast<uint32_t>(*reinterpret_cast<const uint16_t *>(&hi)) << 16);
         }
-        uint4 *dst = reinterpret_cast<uint4 *>(out + blk * 8);
-        dst[0] = make_uint4(words[0], words[1], words[2], words[3]);
-        dst[1] = make_uint4(words[4], words[5], words[6], words[7]);
+        const uint4 c0 = make_uint4(words[0], words[1], words[2], words[3]);
+        const uint4 c1 = make_uint4(words[4], words[5], words[6], words[7]);
+        if (TILED) {
+            // block bi of tile kc: chunks 2 (bi % 8) and 2 (bi % 8) + 1 of lane group bi / 8
+            const int64_t kc = blk / 32;
+            const int bi = static_cast<int>(blk % 32), q4 = bi / 8;
+            const int sig = (2 * q4 + static_cast<int>(t & 1)) & 7;
+            uint4 *row = reinterpret_cast<uint4 *>(Xp + (kc * gridDim.x + t) * kTileCols);
+            row[16 * q4 + ((2 * (bi % 8)) ^ sig)] = c0;
+            row[16 * q4 + ((2 * (bi % 8) + 1) ^ sig)] = c1;
+        } else {
+            uint4 *dst = reinterpret_cast<uint4 *>(Xp + t * npad) + blk * 2;
+            dst[0] = c0;
+            dst[1] = c1;
+        }
     }
     block_sum_256(r - 128.0f * S, corrpart + t * gridDim.y + blockIdx.y);
 }
@@ -292,207 +308,279 @@ packed_gemv_kernel(const uint8_t *__restrict__ packed, int64_t m, int64_t n, int
 
 // ------------------------------------------------------------------ TMA-streamed variant
 //
-// Persistent CTAs: one producer thread streams (R rows x 512 columns) code tiles through a ring of 2-D
-// TMA copies (128-byte swizzle, bank-conflict-free fragment reads). CW consumer warps: warp w owns the
-// 64-column slice w % 8 of every tile and the RBW consecutive 16-row blocks of row group w / 8, so a
-// unit has R = (CW / 8) * 16 * RBW rows. mma.sync is latency-bound per warp here, so the warp count
-// is what hides the conversion and MMA latencies; the eight slices of a row are summed through
-// shared memory in a fixed order at the end of each unit.
+// Persistent CTAs. One producer thread streams each (R rows x 512 columns) code tile (2-D TMA copy,
+// 128-byte swizzle) together with the matching 512 columns of X' of the launch's tokens (one bulk
+// copy) through a shared-memory ring. Consumer warp w owns RBW 16-row blocks of every tile, over all
+// 512 columns, so a row's sum stays in one warp's registers (with KS = 2 two warps split the tiles of
+// a unit by parity and add their sums once per unit).
+//
+// Fragment reads. Lane (g, q4) (g = lane / 4, q4 = lane % 4) reads the 16-byte chunks 2 q4 and
+// 2 q4 + 1 of its rows g and g + 8 of a block: a chunk holds four 16-column code words, and word v of
+// chunk c supplies the lane's A fragments of four MMAs (16 columns x 16 rows each). The swizzle puts
+// chunk c of row r at c ^ (r % 8), so a quarter-warp's eight 16-byte reads hit eight distinct bank
+// groups. X' of a tile is stored per token as 64 chunks of 16 bytes; lane (g, q4) reads token g's
+// chunks [16 q4, 16 q4 + 16) (the activations of its own 128 columns, in word order), each at
+// position 16 q4 + (i ^ ((2 q4 + g % 2) % 8)) so that those reads are conflict-free as well; the prep
+// kernel writes X' in exactly this order.
+//
+// Two accumulators per (row block, token tile) alternate over the four MMAs of a word, which halves
+// the dependent-MMA chains a warp waits on.
 
-constexpr int kTmaStages = 8;
-constexpr int kColGroups = 8;         // 64-column slices of a 512-column tile
-constexpr int kTileCols = 512;        // 128 bytes of codes per row per stage
-constexpr size_t kGemvSmemLimit = 227 * 1024;
 
 struct GemvTmaParams {
-    int64_t m, N, npad, nprep;
-    int R, units, nkc, stages;
-    const uint16_t *Xp;       // [N][npad] (token 0 of this launch)
-    const float *corrpart;    // [N][nprep]
-    uint16_t *Y;              // [N][m]
+    int64_t m, ntok_all, npad, nprep;
+    int ntok, t0, units, nkc, stages;
+    const uint16_t *Xp;       // tile-major X': [npad / 512][ntok_all][512]
+    const float *corrpart;    // [ntok][nprep] (token t0 of this launch)
+    uint16_t *Y;              // [ntok][m] (token t0 of this launch)
     int32_t *status;
 };
 
-// Shared-memory layout (offsets from the 1024-byte aligned base): ring, slice partial sums
-// [8][R][8 NT + 1], barriers, per-token constants.
+// Shared-memory layout (offsets from the 1024-byte aligned base): code ring, X' ring, KS = 2
+// exchange buffer, barriers.
 struct GemvTmaLayout {
-    size_t red, bars, corr, total;
+    size_t acts, red, bars, total;
 };
-__host__ __device__ inline GemvTmaLayout gemv_tma_layout(int R, int stages, int nt) {
+__host__ __device__ inline GemvTmaLayout gemv_tma_layout(int R, int stages, int nt, int cwr, int rbw, int ks) {
     GemvTmaLayout L;
-    L.red = static_cast<size_t>(stages) * static_cast<size_t>(R) * 128;
-    L.bars = L.red + static_cast<size_t>(kColGroups) * static_cast<size_t>(R) * (8 * nt + 1) * 4;
-    L.bars = (L.bars + 15) / 16 * 16;
-    L.corr = L.bars + 2 * kTmaStages * 8;
-    L.total = L.corr + 16 * 4;
+    L.acts = static_cast<size_t>(stages) * static_cast<size_t>(R) * 128;
+    L.red = L.acts + static_cast<size_t>(stages) * static_cast<size_t>(8 * nt) * 1024;
+    L.bars = L.red + (ks > 1 ? static_cast<size_t>(cwr) * 32 * static_cast<size_t>(rbw * nt * 8) * 4 : 0);
+    L.total = L.bars + 2 * kTmaStages * 8;
     return L;
 }
 
-__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
-    uint32_t v;
-    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
+// Named-barrier arrival that also tells whether any participating thread had pred set.
+__device__ __forceinline__ bool bar_any(int id, int count, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(count)
+        : "memory");
+    return r != 0;
 }
 
-// NT: 8-token MMA tiles (1: N <= 8, 2: N <= 16). CW: consumer warps (a multiple of 8). RBW: 16-row
-// blocks per warp per tile.
-template <int NT, int CW, int RBW>
-__global__ void __launch_bounds__(32 * (CW + 1), 1)
+// NT: 8-token MMA tiles (1: <= 8 tokens, 2: <= 16). CWR: consumer warps per K phase; RBW: 16-row
+// blocks per warp; KS: K phases (tiles of a unit split by kc % KS). Unit rows R = CWR * 16 * RBW.
+template <int NT, int CWR, int RBW, int KS>
+__global__ void __launch_bounds__(32 * (CWR * KS + 1), 1)
 packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaParams p) {
-    static_assert(CW % kColGroups == 0, "consumer warps must cover the 8 slices");
-    constexpr int R = (CW / kColGroups) * 16 * RBW;
-    constexpr int LD = 8 * NT + 1;
+    constexpr int CW = CWR * KS;
+    constexpr int R = CWR * 16 * RBW;
+    constexpr uint32_t kCodeBytes = static_cast<uint32_t>(R) * 128u;
+    constexpr uint32_t kActStride = 8u * NT * 1024u;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const GemvTmaLayout L = gemv_tma_layout(R, p.stages, NT);
-    float *red = reinterpret_cast<float *>(base + L.red);          // [8][R][LD]
+    const GemvTmaLayout L = gemv_tma_layout(R, p.stages, NT, CWR, RBW, KS);
+    uint8_t *acts = base + L.acts;
+    float *red = reinterpret_cast<float *>(base + L.red);
     uint64_t *full = reinterpret_cast<uint64_t *>(base + L.bars);
     uint64_t *empty = full + kTmaStages;
-    float *corr_s = reinterpret_cast<float *>(base + L.corr);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    constexpr uint32_t kStageBytes = static_cast<uint32_t>(R) * 128u;
+    const uint32_t act_bytes = static_cast<uint32_t>(p.ntok) * 1024u;
+    const int my_units = p.units > static_cast<int>(blockIdx.x)
+                             ? (p.units - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1
+                             : 0;
+    const int tiles = my_units * p.nkc;
     if (threadIdx.x == 0) {
         prefetch_tensormap(&tmC);
         for (int i = 0; i < p.stages; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], CW);
+            mbar_init(&empty[i], CWR);
         }
         fence_barrier_init();
     }
     __syncthreads();
 
     if (warp == 0) {
-        // ---------------------------------------------------------------- producer: code tiles -> ring
+        // ---------------------------------------------------------------- producer
         if (lane == 0) {
-            int st = 0;
-            uint32_t ph = 0;
-            for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
-                for (int kc = 0; kc < p.nkc; ++kc) {
-                    if (!mbar_wait(&empty[st], ph ^ 1, p.status)) return;
-                    mbar_arrive_expect_tx(&full[st], kStageBytes);
-                    tma_load_2d(base + static_cast<size_t>(st) * kStageBytes, &tmC, kc * 128, u * R, &full[st]);
-                    if (++st == p.stages) { st = 0; ph ^= 1; }
-                }
+            auto tile_at = [&](int T, int &u, int &kc) {
+                u = static_cast<int>(blockIdx.x) + (T / p.nkc) * static_cast<int>(gridDim.x);
+                kc = T % p.nkc;
+            };
+            auto act_src = [&](int kc) {
+                return p.Xp + (static_cast<int64_t>(kc) * p.ntok_all + p.t0) * kTileCols;
+            };
+            // The code tiles of the first stages go out before X' exists (the prep kernel may still
+            // be running); their X' copies follow once it has completed.
+            const int P = tiles < p.stages ? tiles : p.stages;
+            for (int T = 0; T < P; ++T) {
+                int u, kc;
+                tile_at(T, u, kc);
+                mbar_arrive_expect_tx(&full[T], kCodeBytes + act_bytes);
+                tma_load_2d(base + static_cast<size_t>(T) * kCodeBytes, &tmC, kc * 128, u * R, &full[T]);
+            }
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            for (int T = 0; T < P; ++T) {
+                int u, kc;
+                tile_at(T, u, kc);
+                bulk_g2s(acts + static_cast<size_t>(T) * kActStride, act_src(kc), act_bytes, &full[T]);
+            }
+            int st = P % p.stages;
+            uint32_t ph = P == p.stages ? 1u : 0u;
+            for (int T = P; T < tiles; ++T) {
+                int u, kc;
+                tile_at(T, u, kc);
+                if (!mbar_wait(&empty[st], ph ^ 1, p.status)) return;
+                mbar_arrive_expect_tx(&full[st], kCodeBytes + act_bytes);
+                tma_load_2d(base + static_cast<size_t>(st) * kCodeBytes, &tmC, kc * 128, u * R, &full[st]);
+                bulk_g2s(acts + static_cast<size_t>(st) * kActStride, act_src(kc), act_bytes, &full[st]);
+                if (++st == p.stages) { st = 0; ph ^= 1; }
             }
         }
         return;
     }
 
     // -------------------------------------------------------------------- consumers
-    asm volatile("griddepcontrol.wait;" ::: "memory");   // X' and corr partials of the prep kernel
-    const int cw = (warp - 1) % kColGroups;              // 64-column slice
-    const int rb0 = ((warp - 1) / kColGroups) * RBW;
-    const int g = lane >> 2, tid = lane & 3;
-    const int ct = threadIdx.x - 32;
-    if (ct < p.N) corr_s[ct] = token_corr(p.corrpart, ct, p.nprep);
-    asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
-    const bool has0 = g < p.N, has1 = (g + 8) < p.N;
-    const uint32_t *xp0 = reinterpret_cast<const uint32_t *>(p.Xp + (has0 ? g : 0) * p.npad);
-    const uint32_t *xp1 = reinterpret_cast<const uint32_t *>(p.Xp + (has1 ? g + 8 : 0) * p.npad);
-    // this lane's word in its rows (row % 8 == g): 16-byte chunk cw ^ g, word tid
-    const uint32_t swz = static_cast<uint32_t>((cw ^ g) << 4) + 4u * tid + static_cast<uint32_t>((rb0 * 16 + g) * 128);
-    const uint32_t ring0 = smem_u32(base);
-
-    // activation fragments of this warp's 64 columns of tile kc (16-column block of this lane's word);
-    // the next tile's fragments are fetched while the current tile is multiplied.
-    auto load_frags = [&](int kc, uint2 (&bq)[4][NT]) {
-        const int64_t blk = static_cast<int64_t>(kc) * (kTileCols / 16) + cw * 4 + tid;
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-            bq[h][0] = has0 ? __ldg(reinterpret_cast<const uint2 *>(xp0 + blk * 8 + 2 * h)) : make_uint2(0, 0);
-            if (NT == 2)
-                bq[h][NT - 1] = has1 ? __ldg(reinterpret_cast<const uint2 *>(xp1 + blk * 8 + 2 * h)) : make_uint2(0, 0);
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // corr partials of the prep kernel
+    const int cwarp = warp - 1;
+    const int rg = cwarp % CWR, ks = cwarp / CWR;
+    const int g = lane >> 2, q4 = lane & 3;
+    // X' rows of the tile's unused token slots are zero in every stage (the copies never write them),
+    // so the lanes of those tokens read zero fragments without a select
+    {
+        const int zrows = 8 * NT - p.ntok;
+        for (int o = threadIdx.x - 32; o < p.stages * zrows * 64; o += 32 * CW) {
+            const int s_ = o / (zrows * 64), rem = o % (zrows * 64);
+            reinterpret_cast<uint4 *>(acts + static_cast<size_t>(s_) * kActStride +
+                                      static_cast<size_t>(p.ntok + rem / 64) * 1024)[rem % 64] = make_uint4(0, 0, 0, 0);
         }
-    };
-    uint2 bcur[4][NT], bnext[4][NT];
-    load_frags(0, bcur);
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+    }
+    float corr[NT][2];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int t = 8 * nt + 2 * q4 + e;
+            corr[nt][e] = t < p.ntok ? token_corr(p.corrpart, t, p.nprep) : 0.0f;
+        }
+    }
+    // byte offsets inside a stage: this lane's first code chunk (row g of its first block) and its
+    // X' chunks (token g); the chunk index i of X' is stored at i ^ sig
+    const uint32_t code_off = static_cast<uint32_t>((rg * RBW * 16 + g) * 128);
+    const uint32_t act_off = static_cast<uint32_t>(g * 1024 + q4 * 256);
+    const uint32_t sig = static_cast<uint32_t>((2 * q4 + (g & 1)) & 7);
 
     int st = 0;
     uint32_t ph = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-        float acc[RBW][NT][4];
+    for (int ul = 0; ul < my_units && ok; ++ul) {
+        const int u = static_cast<int>(blockIdx.x) + ul * static_cast<int>(gridDim.x);
+        float acc[RBW][NT][2][4];
 #pragma unroll
         for (int i = 0; i < RBW; ++i)
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) acc[i][nt][e] = 0.0f;
+                for (int a = 0; a < 2; ++a)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[i][nt][a][e] = 0.0f;
 
         for (int kc = 0; kc < p.nkc; ++kc) {
-            load_frags(kc + 1 < p.nkc ? kc + 1 : 0, bnext);
-            if (!mbar_wait(&full[st], ph, p.status)) { ok = false; break; }
-            const uint32_t tbase = ring0 + static_cast<uint32_t>(st) * kStageBytes + swz;
-            // row blocks in pairs: two blocks' fragments converted, then their MMAs interleaved (h outer)
-#pragma unroll
-            for (int rp = 0; rp < (RBW + 1) / 2; ++rp) {
-                constexpr int kLast = RBW - 1;
-                const bool second = 2 * rp + 1 <= kLast;
-                uint32_t w[2][2];
+            if (KS == 1 || kc % KS == ks) {
+                if (!mbar_wait(&full[st], ph, p.status)) { ok = false; break; }
+                const uint8_t *ctile = base + static_cast<size_t>(st) * kCodeBytes + code_off;
+                const uint8_t *atile = acts + static_cast<size_t>(st) * kActStride + act_off;
 #pragma unroll
                 for (int j = 0; j < 2; ++j) {
-                    const uint32_t rbase = static_cast<uint32_t>((2 * rp + j) * 16 * 128);
-                    w[j][0] = (j == 0 || second) ? lds32(tbase + rbase) : 0u;
-                    w[j][1] = (j == 0 || second) ? lds32(tbase + rbase + 8u * 128u) : 0u;
-                }
-                uint32_t f[2][2][8];
+                    const uint32_t cchunk = static_cast<uint32_t>(((2 * q4 + j) ^ g) << 4);
+                    uint4 cw[RBW][2];
 #pragma unroll
-                for (int j = 0; j < 2; ++j) {
-                    if (j == 0 || second) {
-                        codes_to_frags(w[j][0], f[j][0]);
-                        codes_to_frags(w[j][1], f[j][1]);
-                    }
-                }
+                    for (int i = 0; i < RBW; ++i)
 #pragma unroll
-                for (int h = 0; h < 4; ++h) {
+                        for (int r8 = 0; r8 < 2; ++r8)
+                            cw[i][r8] = *reinterpret_cast<const uint4 *>(ctile + (i * 16 + 8 * r8) * 128 + cchunk);
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        if (j == 0 || second) {
+                    for (int v = 0; v < 4; ++v) {
+                        uint4 bx[NT][2];
 #pragma unroll
-                            for (int nt = 0; nt < NT; ++nt)
-                                mma_bf16_16816(acc[2 * rp + j][nt], f[j][0][2 * h], f[j][1][2 * h], f[j][0][2 * h + 1],
-                                               f[j][1][2 * h + 1], bcur[h][nt].x, bcur[h][nt].y);
+                        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                            for (int hf = 0; hf < 2; ++hf) {
+                                const uint32_t ci = static_cast<uint32_t>(8 * j) + ((static_cast<uint32_t>(2 * v + hf)) ^ sig);
+                                bx[nt][hf] = *reinterpret_cast<const uint4 *>(atile + nt * 8 * 1024 + ci * 16);
+                            }
+                        // all blocks' fragments first, then the MMAs with the blocks innermost, so
+                        // consecutive MMAs are independent
+                        uint32_t f0[RBW][8], f8[RBW][8];
+#pragma unroll
+                        for (int i = 0; i < RBW; ++i) {
+                            const uint32_t w0 = v == 0 ? cw[i][0].x : v == 1 ? cw[i][0].y : v == 2 ? cw[i][0].z : cw[i][0].w;
+                            const uint32_t w8 = v == 0 ? cw[i][1].x : v == 1 ? cw[i][1].y : v == 2 ? cw[i][1].z : cw[i][1].w;
+                            codes_to_frags(w0, f0[i]);
+                            codes_to_frags(w8, f8[i]);
                         }
+#pragma unroll
+                        for (int h = 0; h < 4; ++h)
+#pragma unroll
+                            for (int i = 0; i < RBW; ++i)
+#pragma unroll
+                                for (int nt = 0; nt < NT; ++nt) {
+                                    const uint4 &b = bx[nt][h >> 1];
+                                    const uint32_t b0 = (h & 1) ? b.z : b.x, b1 = (h & 1) ? b.w : b.y;
+                                    mma_bf16_16816(acc[i][nt][h & 1], f0[i][2 * h], f8[i][2 * h], f0[i][2 * h + 1],
+                                                   f8[i][2 * h + 1], b0, b1);
+                                }
                     }
                 }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&empty[st]);
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[st]);
             if (++st == p.stages) { st = 0; ph ^= 1; }
-#pragma unroll
-            for (int h = 0; h < 4; ++h)
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) bcur[h][nt] = bnext[h][nt];
         }
-        if (!ok) break;
-        // cross-slice reduction (fixed order), + corr, bf16 store
+        if (KS == 1 && !ok) break;
+        // sum of the two accumulators; with KS = 2 the second phase's warps hand theirs over
 #pragma unroll
-        for (int i = 0; i < RBW; ++i) {
-            const int r = 16 * (rb0 + i) + g;
+        for (int i = 0; i < RBW; ++i)
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                float *r0 = red + (static_cast<size_t>(cw) * R + r) * LD + nt * 8 + 2 * tid;
-                float *r8 = r0 + 8 * LD;
-                r0[0] = acc[i][nt][0];
-                r0[1] = acc[i][nt][1];
-                r8[0] = acc[i][nt][2];
-                r8[1] = acc[i][nt][3];
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[i][nt][0][e] += acc[i][nt][1][e];
+        if (KS > 1) {
+            float *mine = red + static_cast<size_t>(rg) * 32 * (RBW * NT * 4) + lane;
+            if (ks == 1 && ok) {
+#pragma unroll
+                for (int i = 0; i < RBW; ++i)
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) mine[32 * ((i * NT + nt) * 4 + e)] = acc[i][nt][0][e];
             }
-        }
-        asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
-        const int64_t row0 = static_cast<int64_t>(u) * R;
-        for (int o = ct; o < R * p.N; o += 32 * CW) {
-            const int rl = o % R, tl = o / R;
-            const int64_t row = row0 + rl;
-            if (row >= p.m) continue;
-            float v = 0.0f;
+            // every consumer warp reaches both barriers of a unit, also after a failed wait, and
+            // all of them leave together if any wait failed
+            const bool failed = bar_any(1, 32 * CW, !ok);
+            if (ks == 0 && !failed) {
 #pragma unroll
-            for (int w = 0; w < kColGroups; ++w) v += red[(static_cast<size_t>(w) * R + rl) * LD + tl];
-            v += corr_s[tl];
-            const __nv_bfloat16 h = __float2bfloat16_rn(v);
-            p.Y[static_cast<int64_t>(tl) * p.m + row] = *reinterpret_cast<const uint16_t *>(&h);
+                for (int i = 0; i < RBW; ++i)
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) acc[i][nt][0][e] += mine[32 * ((i * NT + nt) * 4 + e)];
+            }
+            asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+            if (failed) break;
+            if (ks != 0) continue;
         }
-        asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory");
+        const int64_t row0 = static_cast<int64_t>(u) * R + (rg * RBW) * 16 + g;
+#pragma unroll
+        for (int i = 0; i < RBW; ++i)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int64_t row = row0 + 16 * i + 8 * (e >> 1);
+                    const int t = 8 * nt + 2 * q4 + (e & 1);
+                    if (row < p.m && t < p.ntok) {
+                        const __nv_bfloat16 hv = __float2bfloat16_rn(acc[i][nt][0][e] + corr[nt][e & 1]);
+                        p.Y[static_cast<int64_t>(t) * p.m + row] = *reinterpret_cast<const uint16_t *>(&hv);
+                    }
+                }
     }
 }
 
@@ -972,21 +1060,18 @@ size_t packed_gemv_corr_offset(int64_t N, int64_t n) {
     return ((xp + 255) / 256) * 256;
 }
 
-// Tensor-core variant configurations: (token groups, consumer warps, row blocks per warp). The unit
-// has (CW / 8) * 16 * RBW rows; the launcher picks the configuration whose units balance best over
-// the CTAs.
+// Tensor-core variant configurations: (token tiles, warps per K phase, row blocks per warp, K
+// phases). The unit has CWR * 16 * RBW rows; the launcher picks the configuration whose units
+// balance best over the CTAs.
 struct GemvTmaConfig {
-    int nt, cw, rbw;
+    int nt, cwr, rbw, ks;
     void (*kernel)(const CUtensorMap, const GemvTmaParams);
 };
-// In order of preference (measured on the 70B gate: 24 x 2 at 1-8 tokens, 8 x 4 at 9-16 tokens);
-// a later entry wins only if its units balance at least half a percent better.
+// In order of preference; a later entry wins only if its units balance at least half a percent better.
 static const GemvTmaConfig kGemvTmaConfigs[] = {
-    {1, 24, 2, packed_gemv_tma_kernel<1, 24, 2>}, {1, 16, 4, packed_gemv_tma_kernel<1, 16, 4>},
-    {1, 24, 4, packed_gemv_tma_kernel<1, 24, 4>}, {1, 16, 2, packed_gemv_tma_kernel<1, 16, 2>},
-    {1, 24, 1, packed_gemv_tma_kernel<1, 24, 1>}, {1, 16, 1, packed_gemv_tma_kernel<1, 16, 1>},
-    {2, 8, 4, packed_gemv_tma_kernel<2, 8, 4>},   {2, 8, 2, packed_gemv_tma_kernel<2, 8, 2>},
-    {2, 16, 2, packed_gemv_tma_kernel<2, 16, 2>}, {2, 16, 1, packed_gemv_tma_kernel<2, 16, 1>},
+    {1, 4, 3, 2, packed_gemv_tma_kernel<1, 4, 3, 2>}, {1, 4, 2, 2, packed_gemv_tma_kernel<1, 4, 2, 2>},
+    {1, 4, 1, 2, packed_gemv_tma_kernel<1, 4, 1, 2>}, {2, 4, 3, 2, packed_gemv_tma_kernel<2, 4, 3, 2>},
+    {2, 4, 2, 2, packed_gemv_tma_kernel<2, 4, 2, 2>}, {2, 4, 1, 2, packed_gemv_tma_kernel<2, 4, 1, 2>},
 };
 
 static const GemvTmaConfig *choose_tma_config(int64_t m, int ctas, int nt) {
@@ -994,7 +1079,7 @@ static const GemvTmaConfig *choose_tma_config(int64_t m, int ctas, int nt) {
     double best_eff = -1.0;
     for (const GemvTmaConfig &c : kGemvTmaConfigs) {
         if (c.nt != nt) continue;
-        const int R = (c.cw / kColGroups) * 16 * c.rbw;
+        const int R = c.cwr * 16 * c.rbw;
         const int64_t units = (m + R - 1) / R;
         const int64_t rounds = (units + ctas - 1) / ctas;
         const double eff = static_cast<double>(units) / static_cast<double>(rounds * (units < ctas ? units : ctas));
@@ -1117,44 +1202,50 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
             return cudaGetLastError();
         }
     }
+    const bool tiled = a.n % 64 == 0 && a.m >= 16;
     dim3 pgrid(static_cast<unsigned>(a.N), static_cast<unsigned>(nprep));
-    if (a.Xf) {
-        if (d == 4) gemv_prep_kernel<4, true><<<pgrid, 256, 0, st>>>(a.Xf, a.n, npad, a.A, a.b, a.Xp, a.corr);
-        else gemv_prep_kernel<8, true><<<pgrid, 256, 0, st>>>(a.Xf, a.n, npad, a.A, a.b, a.Xp, a.corr);
-    } else {
-        if (d == 4) gemv_prep_kernel<4, false><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
-        else gemv_prep_kernel<8, false><<<pgrid, 256, 0, st>>>(a.X, a.n, npad, a.A, a.b, a.Xp, a.corr);
-    }
+    using PrepFn = void (*)(const void *, int64_t, int64_t, const float *, const float *, uint16_t *, float *);
+    PrepFn prep;
+    if (a.Xf)
+        prep = d == 4 ? (tiled ? gemv_prep_kernel<4, true, true> : gemv_prep_kernel<4, true, false>)
+                      : (tiled ? gemv_prep_kernel<8, true, true> : gemv_prep_kernel<8, true, false>);
+    else
+        prep = d == 4 ? (tiled ? gemv_prep_kernel<4, false, true> : gemv_prep_kernel<4, false, false>)
+                      : (tiled ? gemv_prep_kernel<8, false, true> : gemv_prep_kernel<8, false, false>);
+    prep<<<pgrid, 256, 0, st>>>(a.Xf ? static_cast<const void *>(a.Xf) : static_cast<const void *>(a.X), a.n, npad,
+                                a.A, a.b, a.Xp, a.corr);
     count_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    if (a.n % 64 == 0 && a.m >= 16) {
+    if (tiled) {
         for (int64_t t0 = 0; t0 < a.N; t0 += 16) {
             const int64_t ntok = (a.N - t0) < 16 ? (a.N - t0) : 16;
             const GemvTmaConfig *c = choose_tma_config(a.m, num_sms, ntok > 8 ? 2 : 1);
-            const int R = (c->cw / kColGroups) * 16 * c->rbw;
+            const int R = c->cwr * 16 * c->rbw;
             CUtensorMap map;
             if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
             int stages = kTmaStages;
-            while (stages > 2 && gemv_tma_layout(R, stages, c->nt).total + 1024 > kGemvSmemLimit) --stages;
+            while (stages > 2 && gemv_tma_layout(R, stages, c->nt, c->cwr, c->rbw, c->ks).total + 1024 > kGemvSmemLimit)
+                --stages;
             GemvTmaParams p;
             p.m = a.m;
-            p.N = ntok;
+            p.ntok_all = a.N;
             p.npad = npad;
             p.nprep = nprep;
-            p.R = R;
+            p.ntok = static_cast<int>(ntok);
+            p.t0 = static_cast<int>(t0);
             p.units = static_cast<int>((a.m + R - 1) / R);
             p.nkc = static_cast<int>(npad / kTileCols);
             p.stages = stages;
-            p.Xp = a.Xp + t0 * npad;
+            p.Xp = a.Xp;
             p.corrpart = a.corr + t0 * nprep;
             p.Y = a.Y + t0 * a.m;
             p.status = a.status;
             const int grid = p.units < num_sms ? p.units : num_sms;
-            const size_t smem = gemv_tma_layout(R, stages, c->nt).total + 1024;
+            const size_t smem = gemv_tma_layout(R, stages, c->nt, c->cwr, c->rbw, c->ks).total + 1024;
             e = ensure_dynamic_smem(reinterpret_cast<const void *>(c->kernel), static_cast<int>(smem));
             if (e != cudaSuccess) return e;
-            e = launch_pdl(c->kernel, dim3(grid), dim3(32 * (c->cw + 1)), smem, st, map, p);
+            e = launch_pdl(c->kernel, dim3(grid), dim3(32 * (c->cwr * c->ks + 1)), smem, st, map, p);
             count_launch();
             if (e != cudaSuccess) return e;
         }
