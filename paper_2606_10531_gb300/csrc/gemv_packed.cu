@@ -702,15 +702,19 @@ __device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *a
             r = fmaf(xj, bj, r);
         }
     }
+    // round to int16: v + 1.5 * 2^23 holds round(v) (ties to even) in its low mantissa bits for
+    // |v| < 2^22, so the low 16 bits are the two's-complement int16; |v| <= 32767 by the choice of inv
+    // (clamped all the same)
     constexpr int kFirst[8] = {0, 8, 1, 9, 2, 10, 3, 11};
+    constexpr float kMagic = 12582912.0f;
     uint32_t words[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         const int cc = kFirst[k];
         const float f = (cc & 1) ? 0.25f * inv : inv;
-        const int lo = max(-32767, min(32767, __float2int_rn(xp[cc] * f)));
-        const int hi = max(-32767, min(32767, __float2int_rn(xp[cc + 4] * f)));
-        words[k] = (static_cast<uint32_t>(lo) & 0xFFFFu) | (static_cast<uint32_t>(hi) << 16);
+        const float lo = fminf(fmaxf(xp[cc] * f, -32767.0f), 32767.0f) + kMagic;
+        const float hi = fminf(fmaxf(xp[cc + 4] * f, -32767.0f), 32767.0f) + kMagic;
+        words[k] = __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x5410);
     }
     uint4 *dst = reinterpret_cast<uint4 *>(xq_s + static_cast<size_t>(tile) * 1024);
     dst[lane] = make_uint4(words[0], words[1], words[2], words[3]);
@@ -776,8 +780,13 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
     // -------------------------------------------------------------------- consumers
     const int cw = warp - 1, ct = threadIdx.x - 32;
     const auto bar_consumers = [] { asm volatile("bar.sync 1, %0;" ::"r"(32 * CW) : "memory"); };
-    // A and b are weights like the codes: read before the wait, only X comes from the previous kernel
+    // A and b are weights like the codes: read before the wait, only X comes from the previous kernel;
+    // so is max_k sum_j |A[j][k]| (lane k of every warp)
     if (ct < p.d * p.d + p.d) ab_s[ct] = ct < p.d * p.d ? __ldg(p.A + ct) : __ldg(p.b + (ct - p.d * p.d));
+    float acol = 0.0f;
+    if (lane < p.d)
+        for (int j = 0; j < p.d; ++j) acol += fabsf(__ldg(p.A + j * p.d + lane));
+    for (int o = 16; o; o >>= 1) acol = fmaxf(acol, __shfl_xor_sync(0xffffffffu, acol, o));
     asm volatile("griddepcontrol.wait;" ::: "memory");
     float scale, corr;
     {
@@ -801,19 +810,13 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
         bar_consumers();
         if (ct == 0) mbar_arrive(xready);
         // pass 2: the token's scale s = max|X| * max_k sum_j |A[j][k]| / 32767 (a bound on max|X'|),
-        // then X' -> int16. Both maxima by warp shuffles (no serial chains of shared-memory loads).
+        // then X' -> int16. The maxima by warp shuffles (no serial chains of shared-memory loads).
         float xmax = lane < CW ? red_s[lane] : 0.0f;
-        float acol = 0.0f;
-        if (lane < D) {
-            for (int j = 0; j < D; ++j) acol += fabsf(ab_s[j * D + lane]);
-        }
-        for (int o = 16; o; o >>= 1) {
-            xmax = fmaxf(xmax, __shfl_xor_sync(0xffffffffu, xmax, o));
-            acol = fmaxf(acol, __shfl_xor_sync(0xffffffffu, acol, o));
-        }
+        for (int o = 16; o; o >>= 1) xmax = fmaxf(xmax, __shfl_xor_sync(0xffffffffu, xmax, o));
         const float bound = xmax * acol;
-        scale = bound / 32767.0f;
-        const float inv = bound > 0.0f ? 32767.0f / bound : 0.0f;
+        scale = bound * (1.0f / 32767.0f);
+        // inv need not be exactly 1 / scale: |X'| * inv stays <= 32767 up to rounding (clamped)
+        const float inv = bound > 0.0f ? __fdividef(32767.0f, bound) : 0.0f;
         uint8_t *xq_s = base + L.xq;
         float r = 0.0f;
         if (cw < p.nkc) {
