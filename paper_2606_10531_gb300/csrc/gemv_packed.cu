@@ -623,6 +623,7 @@ struct GemvDpParams {
     const float *A, *b;
     int64_t m, n;
     int d, f32in;
+    int hb;                   // > 0: rotate X by the block Walsh-Hadamard transform of this block size first
     int R, units, nkc, stages;
     uint16_t *Y;              // [m]
     int32_t *status;
@@ -727,6 +728,39 @@ __device__ __forceinline__ float absmax16(const float (&x)[16], float mx) {
     return mx;
 }
 
+// Block Walsh-Hadamard rotation of the token in the prologue (Sec. 3.3 rotated deployment), for
+// n = 32 * 16 * kDpWarps: consumer thread t holds columns 16 t .. 16 t + 15, so the bits of a column
+// index are (warp, lane, register). H_B factors over the index bits (one (u, v) -> (u + v, u - v)
+// stage per bit below log2 B): the 4 register bits in registers, the 5 lane bits by warp shuffles, the
+// warp bits after one exchange through shared memory (thread t then holds columns t + 512 w, w = 0..15)
+// and one back. Unnormalised; the caller scales by 1 / sqrt(B).
+__device__ __forceinline__ void wht_reg16(float (&x)[16], int step0, int hb) {
+    // butterflies over the register index for element strides step0 * {1, 2, 4, 8} below hb
+#pragma unroll
+    for (int r = 1; r < 16; r *= 2) {
+        if (step0 * r >= hb) break;
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+            if ((i & r) == 0) {
+                const float u = x[i], v = x[i + r];
+                x[i] = u + v;
+                x[i + r] = u - v;
+            }
+    }
+}
+__device__ __forceinline__ void wht_lanes(float (&x)[16], int lane, int hb) {
+#pragma unroll
+    for (int s = 1; s < 32; s *= 2) {
+        if (16 * s >= hb) break;
+        const bool upper = (lane & s) != 0;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float v = __shfl_xor_sync(0xffffffffu, x[i], s);
+            x[i] = upper ? v - x[i] : x[i] + v;
+        }
+    }
+}
+
 // RPT: rows per thread per tile (a unit has R = kDpWarps * RPT rows).
 template <int RPT>
 __global__ void __launch_bounds__(32 * (kDpWarps + 1), 1)
@@ -768,8 +802,12 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
                     tma_load_2d(base + static_cast<size_t>(st) * stage_bytes, &tmC, kc * 128, u * p.R, &full[st]);
                     // only a short head start of the code stream before the consumers' X loads: a full
                     // ring in flight delays those loads (measured)
-                    if (u == static_cast<int>(blockIdx.x) && kc == kDpPrefill - 1 && !mbar_wait(xready, 0, p.status))
-                        return;
+                    if (u == static_cast<int>(blockIdx.x) && kc == kDpPrefill - 1) {
+                        if (!mbar_wait(xready, 0, p.status)) return;
+                        // the consumers' generic accesses to the later stages (the rotation's
+                        // exchange buffer) come before the copies that refill them
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    }
                     if (++st == p.stages) { st = 0; ph ^= 1; }
                 }
             }
@@ -796,10 +834,39 @@ packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParam
         const bool f32in = p.f32in != 0;
         float x0[16];
         float mx = 0.0f;
-        if (cw < p.nkc) {
-            load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(cw) * 32 + lane) * 16, x0);
-            mx = absmax16(x0, mx);
+        if (cw < p.nkc) load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(cw) * 32 + lane) * 16, x0);
+        if (p.hb > 0) {
+            // the rotation (launcher: nkc == CW, so every consumer thread holds one 16-column block);
+            // ring stages kDpPrefill.. are still empty (the producer waits for xready before filling
+            // them) and serve as the exchange buffer
+            wht_reg16(x0, 1, p.hb);
+            wht_lanes(x0, lane, p.hb);
+            if (p.hb > 32 * 16) {
+                float *xs = reinterpret_cast<float *>(base + static_cast<size_t>(kDpPrefill) * stage_bytes);
+                const int t = cw * 32 + lane;
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    reinterpret_cast<float4 *>(xs + 16 * t)[q] = make_float4(x0[4 * q], x0[4 * q + 1], x0[4 * q + 2], x0[4 * q + 3]);
+                bar_consumers();
+                float y[16];
+#pragma unroll
+                for (int w = 0; w < 16; ++w) y[w] = w < CW ? xs[t + 512 * w] : 0.0f;
+                wht_reg16(y, 512, p.hb);
+#pragma unroll
+                for (int w = 0; w < 16; ++w)
+                    if (w < CW) xs[t + 512 * w] = y[w];
+                bar_consumers();
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 v = reinterpret_cast<const float4 *>(xs + 16 * t)[q];
+                    x0[4 * q] = v.x; x0[4 * q + 1] = v.y; x0[4 * q + 2] = v.z; x0[4 * q + 3] = v.w;
+                }
+            }
+            const float nrm = rsqrtf(static_cast<float>(p.hb));
+#pragma unroll
+            for (int i = 0; i < 16; ++i) x0[i] *= nrm;
         }
+        if (cw < p.nkc) mx = absmax16(x0, mx);
         for (int tile = cw + CW; tile < p.nkc; tile += CW) {
             float x[16];
             load_block(p.X, f32in, p.n, 0, (static_cast<int64_t>(tile) * 32 + lane) * 16, x);
@@ -1148,13 +1215,31 @@ static cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t
 
 // dp2a variant for one token. Leaves `done` false (and launches nothing) when the activations do
 // not fit in shared memory next to a ring of at least three stages.
+// Rows per unit, ring stages and rotation block of the dp kernel for this call; false when the kernel
+// does not apply (the activations would not fit next to a ring of three stages, or a requested
+// prologue rotation lacks its one-block-per-thread layout or exchange buffer).
+static bool dp_plan(const PackedGemvArgs &a, int num_sms, int &R, int &stages, int &nkc, int &hb) {
+    nkc = static_cast<int>(gemv_npad(a.n) / kTileCols);
+    R = choose_rows_dp(a.m, num_sms);
+    stages = kTmaStages;
+    while (stages >= 3 && dp_smem_layout(R, stages, nkc).total + 1024 > kDpSmemLimit) --stages;
+    if (stages < 3) return false;
+    hb = 0;
+    if (a.rotate) {
+        // the prologue rotation wants one 16-column block per consumer thread and an exchange buffer
+        // in the ring stages the producer fills only after the activations are in
+        if (a.Xf || nkc != kDpWarps ||
+            static_cast<size_t>(stages - kDpPrefill) * static_cast<size_t>(R) * 128 < static_cast<size_t>(a.n) * 4)
+            return false;
+        hb = hadamard_block_size(a.n);
+    }
+    return true;
+}
+
 static cudaError_t launch_packed_gemv_dp(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, bool &done) {
     done = false;
-    const int nkc = static_cast<int>(gemv_npad(a.n) / kTileCols);
-    const int R = choose_rows_dp(a.m, num_sms);
-    int stages = kTmaStages;
-    while (stages >= 3 && dp_smem_layout(R, stages, nkc).total + 1024 > kDpSmemLimit) --stages;
-    if (stages < 3) return cudaSuccess;
+    int R, stages, nkc, hb;
+    if (!dp_plan(a, num_sms, R, stages, nkc, hb)) return cudaSuccess;
     CUtensorMap map;
     if (!make_codes_map(&map, a.packed, a.m, a.n, R)) return cudaErrorInvalidValue;
     GemvDpParams p;
@@ -1165,6 +1250,7 @@ static cudaError_t launch_packed_gemv_dp(const PackedGemvArgs &a, int d, int num
     p.n = a.n;
     p.d = d;
     p.f32in = a.Xf != nullptr;
+    p.hb = hb;
     p.R = R;
     p.units = static_cast<int>((a.m + R - 1) / R);
     p.nkc = nkc;
@@ -1191,6 +1277,24 @@ static cudaError_t launch_packed_gemv_dp(const PackedGemvArgs &a, int d, int num
     if (e != cudaSuccess) return e;
     done = true;
     return cudaSuccess;
+}
+
+bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err) {
+    err = cudaSuccess;
+    if (!(a.n % 64 == 0 && a.n <= kDpMaxN && a.m >= 16 && a.N == kDpMaxTokens)) return false;
+    PackedGemvArgs r = a;
+    r.rotate = true;
+    r.Xf = nullptr;
+    int R, stages, nkc, hb;
+    if (!dp_plan(r, num_sms, R, stages, nkc, hb)) return false;
+    bool done = false;
+    trace_begin(LCQ_K_GEMV, st);
+    err = launch_packed_gemv_dp(r, d, num_sms, st, done);
+    if (err == cudaSuccess) {
+        trace_end(LCQ_K_GEMV, st);
+        err = cudaGetLastError();
+    }
+    return true;
 }
 
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st) {

@@ -168,10 +168,14 @@ struct PackedGemvArgs {
     uint16_t *Xp;            // workspace: transformed activations [N][npad]
     float *corr;             // workspace: per-token constant, partial sums [N][nprep]
     int32_t *status;
+    bool rotate = false;     // rotate X by the block Walsh-Hadamard transform in the product's prologue
 };
 size_t packed_gemv_workspace(int64_t N, int64_t n);
 size_t packed_gemv_corr_offset(int64_t N, int64_t n);
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);
+// The rotated product with the rotation in the one-token kernel's prologue. Returns false (nothing
+// launched) when that kernel does not apply; err holds a launch error otherwise.
+bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err);
 // Row-wise normalized block Walsh-Hadamard rotation (block = largest power of two dividing n, <= 32768).
 int hadamard_block_size(int64_t n);
 cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t n, float *out, cudaStream_t st);

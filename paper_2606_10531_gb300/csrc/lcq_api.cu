@@ -284,6 +284,17 @@ lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_
     Header *h = static_cast<Header *>(ws);
     float *Xr = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kHeader);
     uint8_t *base = static_cast<uint8_t *>(ws) + kHeader + align256(static_cast<size_t>(N) * static_cast<size_t>(n) * 4);
+    {
+        // one token: the rotation runs in the product kernel's prologue
+        PackedGemvArgs a;
+        a.X = X; a.Xf = nullptr; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
+        a.Xp = reinterpret_cast<uint16_t *>(base);
+        a.corr = reinterpret_cast<float *>(base + packed_gemv_corr_offset(N, n));
+        a.status = &h->status;
+        cudaError_t err;
+        if (launch_packed_gemv_rotated(a, d, num_sms_current(), st, err)) return cuda_status(err);
+        LCQ_TRY(cuda_status(err));
+    }
     trace_begin(LCQ_K_GEMV, st);
     const cudaError_t e = launch_hadamard(X, true, N, n, Xr, st);
     trace_end(LCQ_K_GEMV, st);

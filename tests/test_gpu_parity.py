@@ -454,6 +454,27 @@ def test_hadamard_rotation_matches_oracle(rows, n):
     np.testing.assert_allclose(out.cpu().numpy(), X, rtol=1e-4, atol=1e-5)
 
 
+# One token, n = 8192 and enough rows per unit: the rotation runs in the one-token kernel's prologue
+# (one launch instead of two), in fp32 before the int16 activations, so the dp bound applies.
+@pytest.mark.parametrize("d", [4, 8])
+def test_gemm_packed2b_hadamard_fused_prologue(d):
+    m, n, N = 7296, 8192, 1
+    rng = np.random.default_rng(31 + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n))
+    X[:, rng.random(n) < 0.01] *= 50.0
+    Xb = wl.bf16_bits(X.astype(np.float32))
+    ref = oracle.gemm_packed2b_hadamard(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)
+    before = lcq.lcq_launch_count()
+    lcq.lcq_gemm_packed2b_hadamard(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_launch_count() - before == 1          # no separate rotation kernel
+    assert lcq.lcq_device_status(ws) == 0
+    assert max_rel(host_bf16(Y), ref) <= TOL_DP
+
+
 @pytest.mark.parametrize("N", [1, 16])
 @pytest.mark.parametrize("m,n,d", [(200, 512, 8), (70, 200, 4), (300, 8192, 8)])
 def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
