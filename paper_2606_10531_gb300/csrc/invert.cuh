@@ -94,7 +94,10 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) 
 //  3. If the residual does not reach the acceptance bound within four steps (A badly conditioned, or
 //     non-finite), the fp64 elimination runs instead.
 // Sets s.singular if a pivot is (relatively) zero.
-template <int D, typename Smem>
+// kSpd: A is symmetric positive definite (the diagonal blocks of LDLQ's factorisation), so the
+// elimination takes the diagonal pivots without a search or row swaps, and M is not formed; the
+// refinement and its fp64 fallback are the same.
+template <int D, typename Smem, bool kSpd = false>
 __device__ void invert_warp(Smem &s) {
     constexpr int H = 2 * D / 8;                 // 8-column blocks of [A | I]
     const int lane = threadIdx.x & 31;
@@ -106,11 +109,13 @@ __device__ void invert_warp(Smem &s) {
         const int c = 8 * h + j;
         row[j] = !act ? 0.0f : (c < D ? s.A[r * D + c] : (c - D == r ? 1.0f : 0.0f));
     }
-    for (int e = lane; e < D * D; e += 32) {
-        const int i = e / D, j = e % D;
-        float acc = 0.0f;
-        for (int k = 0; k < D; ++k) acc = fmaf(s.A[k * D + i], s.A[k * D + j], acc);
-        s.M[e] = acc;
+    if (!kSpd) {
+        for (int e = lane; e < D * D; e += 32) {
+            const int i = e / D, j = e % D;
+            float acc = 0.0f;
+            for (int k = 0; k < D; ++k) acc = fmaf(s.A[k * D + i], s.A[k * D + j], acc);
+            s.M[e] = acc;
+        }
     }
     float amax = 0.0f;
 #pragma unroll
@@ -121,21 +126,28 @@ __device__ void invert_warp(Smem &s) {
 #pragma unroll
     for (int c = 0; c < D; ++c) {
         if (singular) break;
-        // pivot: largest |a[r][c]| over rows r >= c (column c sits in block 0, lane r)
-        float v = (act && h == 0 && r >= c) ? fabsf(row[c]) : -1.0f;
-        int idx = r;
-        for (int o = 16; o; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-            if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
-        }
-        if (!(static_cast<double>(v) > 1e-12 * static_cast<double>(amax)) || !isfinite(v)) { singular = 1; break; }
-        const int prow = idx;
-        // swap rows c and prow, within each column block
-        const int src = (r == c) ? prow : (r == prow ? c : r);
+        float piv;
+        if (kSpd) {
+            // the diagonal pivot (positive for a positive definite A)
+            piv = __shfl_sync(0xffffffffu, row[c], c);
+            if (!(static_cast<double>(piv) > 1e-12 * static_cast<double>(amax)) || !isfinite(piv)) { singular = 1; break; }
+        } else {
+            // pivot: largest |a[r][c]| over rows r >= c (column c sits in block 0, lane r)
+            float v = (act && h == 0 && r >= c) ? fabsf(row[c]) : -1.0f;
+            int idx = r;
+            for (int o = 16; o; o >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+                if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
+            }
+            if (!(static_cast<double>(v) > 1e-12 * static_cast<double>(amax)) || !isfinite(v)) { singular = 1; break; }
+            const int prow = idx;
+            // swap rows c and prow, within each column block
+            const int src = (r == c) ? prow : (r == prow ? c : r);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src + D * h);
-        const float piv = __shfl_sync(0xffffffffu, row[c], c);     // a[c][c], block 0
+            for (int j = 0; j < 8; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src + D * h);
+            piv = __shfl_sync(0xffffffffu, row[c], c);     // a[c][c], block 0
+        }
         const float rinv = 1.0f / piv;
         if (r == c) {
 #pragma unroll

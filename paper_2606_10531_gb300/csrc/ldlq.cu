@@ -58,20 +58,25 @@ ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, floa
         s.Up[i][j] = 0.0f;
     }
     __syncthreads();
-    for (int k = G - 1; k >= 0; --k) {
+    // D_k^{-1} of the last group; then per group k (from the last): U_{<k,k} = S_{<k,k} D_k^{-1}, the
+    // next diagonal block D_{k-1} updated first, and its inversion (warp 0) overlapped with the rest of
+    // the Schur update S_{<k,<k} -= U_{<k,k} S_{k,<k} (warps 1..). Only the block-upper triangle is
+    // kept current (S_{k,<k} is read as S_{<k,k}^T).
+    const auto invert_group = [&](int k) {
         const int kd = k * D;
-        if (warp == 0) {
-            for (int e = tid; e < D * D; e += 32) s.inv.A[e] = s.S[kd + e / D][kd + e % D];
-            __syncwarp();
-            invert_warp<D>(s.inv);
-            for (int e = tid; e < D * D; e += 32) {
-                s.Dinv[k][e] = s.inv.Ainv[e];
-                if (Dout) Dout[(c0 / D + k) * D * D + e] = s.inv.A[e];
-            }
-            if (tid == 0 && s.inv.singular) set_status(status, LCQ_ERR_SINGULAR);
+        for (int e = tid; e < D * D; e += 32) s.inv.A[e] = s.S[kd + e / D][kd + e % D];
+        __syncwarp();
+        invert_warp<D, InvScratch, true>(s.inv);
+        for (int e = tid; e < D * D; e += 32) {
+            s.Dinv[k][e] = s.inv.Ainv[e];
+            if (Dout) Dout[(c0 / D + k) * D * D + e] = s.inv.A[e];
         }
-        __syncthreads();
-        if (k == 0) break;
+        if (tid == 0 && s.inv.singular) set_status(status, LCQ_ERR_SINGULAR);
+    };
+    if (warp == 0) invert_group(G - 1);
+    __syncthreads();
+    for (int k = G - 1; k >= 1; --k) {
+        const int kd = k * D, kp = kd - D;
         // U_{<k,k} = S_{<k,k} D_k^{-1}
         for (int e = tid; e < kd * D; e += kLdlThreads) {
             const int i = e / D, j = e % D;
@@ -81,13 +86,28 @@ ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, floa
             s.Up[i][kd + j] = acc;
         }
         __syncthreads();
-        // S_{<k,<k} -= U_{<k,k} S_{k,<k}
-        for (int e = tid; e < kd * kd; e += kLdlThreads) {
-            const int i = e / kd, j = e % kd;
+        // the next diagonal block, D_{k-1} -= U_{k-1,k} S_{k,k-1}
+        for (int e = tid; e < D * D; e += kLdlThreads) {
+            const int i = kp + e / D, j = kp + e % D;
             float acc = s.S[i][j];
 #pragma unroll
-            for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[kd + q][j], acc);
+            for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[j][kd + q], acc);
             s.S[i][j] = acc;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            invert_group(k - 1);
+        } else {
+            // the rest of the block-upper triangle of S_{<k,<k}
+            for (int e = tid - 32; e < kd * kd; e += kLdlThreads - 32) {
+                const int i = e / kd, j = e % kd;
+                const int bi = i / D, bj = j / D;
+                if (bi > bj || (bi == k - 1 && bj == k - 1)) continue;
+                float acc = s.S[i][j];
+#pragma unroll
+                for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[j][kd + q], acc);
+                s.S[i][j] = acc;
+            }
         }
         __syncthreads();
     }
@@ -96,13 +116,24 @@ ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, floa
         const int i = e / P, j = e % P;
         if (i / D < j / D) U[(c0 + i) * n + c0 + j] = s.Up[i][j];
     }
-    // X = M^-1, M = I + Up unit upper: X_k = E_k - sum_{j>k} Up_{k,j} X_j, block rows from the last
+    // X = M^-1, M = I + Up unit block-upper triangular: X_k = E_k - sum_{j>k} Up_{k,j} X_j, block rows
+    // from the last; X is block-upper triangular too, so X_k[., col] needs the blocks up to col's only
     for (int k = G - 1; k >= 0; --k) {
         const int kd = k * D;
         for (int e = tid; e < D * P; e += kLdlThreads) {
             const int r = kd + e / P, col = e % P;
-            float acc = (r == col) ? 1.0f : 0.0f;
-            for (int c = kd + D; c < P; ++c) acc = fmaf(-s.Up[r][c], s.S[c][col], acc);
+            float acc;
+            if (col < kd + D) {
+                acc = (r == col) ? 1.0f : 0.0f;
+            } else {
+                // four partial sums (the block boundaries are multiples of D >= 4)
+                float a4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                const int cend = (col / D + 1) * D;
+                for (int c = kd + D; c < cend; c += 4)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) a4[q] = fmaf(-s.Up[r][c + q], s.S[c + q][col], a4[q]);
+                acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+            }
             s.S[r][col] = acc;
         }
         __syncthreads();
