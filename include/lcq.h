@@ -168,6 +168,10 @@ lcq_status lcq_encode_batch(const lcq_encode_item *items, int count, int d, void
  * D  [n/d][d][d] fp32 output (block k is D_k), or NULL.
  * If a block D_k is singular (H not positive definite) the status word becomes LCQ_ERR_SINGULAR.
  * Needs lcq_workspace_size(LCQ_OP_LDL_FACTOR, 0, 0, n, d) bytes of ws (a copy of H, about 4 n^2 bytes).
+ * Streams: each panel's factorisation runs on a library-owned high-priority stream (one per device),
+ * forked from and joined back to `stream` by events, so work enqueued on `stream` after the call sees
+ * every output and the call can be captured into a CUDA graph. Concurrent calls are safe; they share
+ * that stream's order.
  */
 lcq_status lcq_ldl_factor(const float *H, int64_t n, int d, float *U, float *D, void *ws, size_t ws_bytes,
                           void *stream);

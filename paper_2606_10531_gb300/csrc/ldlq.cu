@@ -20,6 +20,8 @@
 // phase per chunk, after a generic-to-async proxy fence).
 #include <cudaTypedefs.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 #include "invert.cuh"
@@ -212,6 +214,36 @@ static cudaError_t gemm_nt(const float *A, int64_t lda, const float *B, int64_t 
     return cudaGetLastError();
 }
 
+// The side stream of the factorisation's look-ahead: one per device, created once with the highest
+// priority. Calls enqueue
+// under a lock and fork/join through events of their own, so concurrent calls only share its order.
+static std::mutex g_ldl_side_mu;
+static cudaError_t ldl_side_stream(cudaStream_t &out) {
+    static cudaStream_t per_device[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!per_device[dev]) {
+        // the highest priority: the one-CTA panel takes the first SM slot the trailing GEMM frees
+        int lo = 0, hi = 0;
+        if ((e = cudaDeviceGetStreamPriorityRange(&lo, &hi)) != cudaSuccess) return e;
+        if ((e = cudaStreamCreateWithPriority(&per_device[dev], cudaStreamNonBlocking, hi)) != cudaSuccess) return e;
+    }
+    out = per_device[dev];
+    return cudaSuccess;
+}
+struct LdlEvents {
+    cudaEvent_t fork = nullptr, join = nullptr;
+    ~LdlEvents() {
+        if (fork) cudaEventDestroy(fork);
+        if (join) cudaEventDestroy(join);
+    }
+};
+
+// Right-looking from the last panel. After a panel, its column block (Y = S_QP M^-T, U_QP) and the
+// update of the next panel's columns run first; the next panel's factorisation then runs on a side
+// stream while the rest of the Schur update (the leading square) runs on the caller's stream.
 cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
     const int64_t n = a.n;
     const size_t nn = static_cast<size_t>(n);
@@ -225,20 +257,45 @@ cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
     const int smem = static_cast<int>(sizeof(LdlPanelSmem));
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(panel), smem);
     if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_ldl_side_mu);
+    cudaStream_t side;
+    if ((e = ldl_side_stream(side)) != cudaSuccess) return e;
+    LdlEvents ev;
+    if ((e = cudaEventCreateWithFlags(&ev.fork, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&ev.join, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaMemcpyAsync(S, a.H, nn * nn * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
     if ((e = cudaMemsetAsync(a.U, 0, nn * nn * 4, st)) != cudaSuccess) return e;
-    for (int64_t c1 = n; c1 > 0; c1 -= kLdlPanel) {
-        const int64_t c0 = c1 > kLdlPanel ? c1 - kLdlPanel : 0;
+    int64_t c1 = n;
+    int64_t c0 = c1 > kLdlPanel ? c1 - kLdlPanel : 0;
+    panel<<<1, kLdlThreads, smem, st>>>(S, n, c0, static_cast<int>(c1 - c0), a.U, a.D, Minv, Binv, a.status);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    bool side_pending = false;
+    while (c0 > 0) {
         const int P = static_cast<int>(c1 - c0);
-        panel<<<1, kLdlThreads, smem, st>>>(S, n, c0, P, a.U, a.D, Minv, Binv, a.status);
-        count_launch();
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        if (c0 == 0) break;
-        // Y = S_QP M^-T, U_QP = S_QP (D^-1 M^-1)^T, S_QQ -= Y U_QP^T (P = kLdlPanel here)
+        const int64_t p0 = c0 > kLdlPanel ? c0 - kLdlPanel : 0;
+        const int Pn = static_cast<int>(c0 - p0);
+        if (side_pending && (e = cudaStreamWaitEvent(st, ev.join, 0)) != cudaSuccess) return e;
+        // Y = S_QP M^-T, U_QP = S_QP (D^-1 M^-1)^T (P = kLdlPanel here)
         if ((e = gemm_nt(S + c0, n, Minv, kLdlPanel, Y, kLdlPanel, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
         if ((e = gemm_nt(S + c0, n, Binv, kLdlPanel, a.U + c0, n, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
-        if ((e = gemm_nt(Y, kLdlPanel, a.U + c0, n, S, n, c0, c0, P, -1.0f, 1.0f, true, st)) != cudaSuccess) return e;
+        // the next panel's columns of S_QQ -= Y U_QP^T (rows 0 .. c0, columns p0 .. c0)
+        if ((e = gemm_nt(Y, kLdlPanel, a.U + p0 * n + c0, n, S + p0, n, c0, Pn, P, -1.0f, 1.0f, false, st)) != cudaSuccess)
+            return e;
+        // the next panel on the side stream, after all of the above (it overwrites M^-1, D^-1 M^-1)
+        if ((e = cudaEventRecord(ev.fork, st)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(side, ev.fork, 0)) != cudaSuccess) return e;
+        panel<<<1, kLdlThreads, smem, side>>>(S, n, p0, Pn, a.U, a.D, Minv, Binv, a.status);
+        count_launch();
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = cudaEventRecord(ev.join, side)) != cudaSuccess) return e;
+        side_pending = true;
+        // the rest of the update, the leading p0 x p0 square (upper tiles), meanwhile
+        if ((e = gemm_nt(Y, kLdlPanel, a.U + c0, n, S, n, p0, p0, P, -1.0f, 1.0f, true, st)) != cudaSuccess) return e;
+        c1 = c0;
+        c0 = p0;
     }
+    if (side_pending && (e = cudaStreamWaitEvent(st, ev.join, 0)) != cudaSuccess) return e;
     return cudaSuccess;
 }
 
