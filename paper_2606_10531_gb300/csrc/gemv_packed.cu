@@ -650,11 +650,6 @@ __device__ __forceinline__ void dp2a_lo(uint32_t a, uint32_t b, int32_t &acc) {
 __device__ __forceinline__ void dp2a_hi(uint32_t a, uint32_t b, int32_t &acc) {
     asm("dp2a.hi.s32.u32 %0, %1, %2, %0;" : "+r"(acc) : "r"(a), "r"(b));
 }
-__device__ __forceinline__ uint4 lds128(uint32_t addr) {
-    uint4 v;
-    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
-    return v;
-}
 
 // acc0/acc1 += the 16 columns of code word w times one 16-column block (two uint4) of activations.
 __device__ __forceinline__ void dp_word(uint32_t w, const uint4 &xa, const uint4 &xb, int32_t &acc0, int32_t &acc1) {
