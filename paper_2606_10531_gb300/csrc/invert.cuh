@@ -84,6 +84,64 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) 
     err = (a - (s - bb)) + (b - bb);
 }
 
+// One thread: X = A^{-1} of a symmetric positive definite A (row-major in smem) by Cholesky, A = L L^T,
+// X = L^{-T} L^{-1}, all in registers (fp32; the caller refines). Returns false if a pivot is not
+// (relatively) positive.
+template <int D>
+__device__ __forceinline__ bool spd_inverse_thread(const float *A, float (&X)[8][16], float amax) {
+    float L[D][D];
+#pragma unroll
+    for (int i = 0; i < D; ++i)
+#pragma unroll
+        for (int j = 0; j < D; ++j) L[i][j] = 0.0f;
+    float dinv[D];
+    bool ok = true;
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+        float dj = A[j * D + j];
+#pragma unroll
+        for (int k = 0; k < j; ++k) dj = fmaf(-L[j][k], L[j][k], dj);
+        ok = ok && (dj > 1e-12f * amax) && isfinite(dj);
+        const float ljj = sqrtf(fmaxf(dj, 1e-30f));
+        L[j][j] = ljj;
+        dinv[j] = 1.0f / ljj;
+#pragma unroll
+        for (int i = j + 1; i < D; ++i) {
+            float v = A[i * D + j];
+#pragma unroll
+            for (int k = 0; k < j; ++k) v = fmaf(-L[i][k], L[j][k], v);
+            L[i][j] = v * dinv[j];
+        }
+    }
+    // W = L^{-1} (lower triangular), column by column
+    float W[D][D];
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+#pragma unroll
+        for (int i = 0; i < D; ++i) W[i][j] = 0.0f;
+        W[j][j] = dinv[j];
+#pragma unroll
+        for (int i = j + 1; i < D; ++i) {
+            float v = 0.0f;
+#pragma unroll
+            for (int k = j; k < i; ++k) v = fmaf(L[i][k], W[k][j], v);
+            W[i][j] = -v * dinv[i];
+        }
+    }
+    // X = W^T W (symmetric)
+#pragma unroll
+    for (int i = 0; i < D; ++i)
+#pragma unroll
+        for (int j = i; j < D; ++j) {
+            float v = 0.0f;
+#pragma unroll
+            for (int k = j; k < D; ++k) v = fmaf(W[k][i], W[k][j], v);
+            X[i][j] = v;
+            X[j][i] = v;
+        }
+    return ok;
+}
+
 // One warp: A^{-1} and M = A^T A (fp32).
 //  1. Gauss-Jordan elimination with partial pivoting in fp32, in registers: lane r + D h (r < D,
 //     h < 2D/8) holds columns 8h .. 8h+7 of row r of [A | I]; pivots, row swaps and the pivot row
@@ -94,9 +152,9 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) 
 //  3. If the residual does not reach the acceptance bound within four steps (A badly conditioned, or
 //     non-finite), the fp64 elimination runs instead.
 // Sets s.singular if a pivot is (relatively) zero.
-// kSpd: A is symmetric positive definite (the diagonal blocks of LDLQ's factorisation), so the
-// elimination takes the diagonal pivots without a search or row swaps, and M is not formed; the
-// refinement and its fp64 fallback are the same.
+// kSpd: A is symmetric positive definite (the diagonal blocks of LDLQ's factorisation): the first
+// approximation is lane 0's Cholesky-based inverse (spd_inverse_thread) instead of the elimination,
+// and M is not formed; the refinement and its fp64 fallback are the same.
 template <int D, typename Smem, bool kSpd = false>
 __device__ void invert_warp(Smem &s) {
     constexpr int H = 2 * D / 8;                 // 8-column blocks of [A | I]
@@ -123,9 +181,16 @@ __device__ void invert_warp(Smem &s) {
         if (8 * h + j < D) amax = fmaxf(amax, fabsf(row[j]));
     for (int o = 16; o; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
     int singular = !(amax > 0.0f) || !isfinite(amax);
+    if (kSpd) {
+        if (!singular) {
+            int bad = 0;
+            if (lane == 0) bad = spd_inverse_thread<D>(s.A, s.gjf, amax) ? 0 : 1;
+            singular = __shfl_sync(0xffffffffu, bad, 0);
+        }
+    }
 #pragma unroll
     for (int c = 0; c < D; ++c) {
-        if (singular) break;
+        if (singular || kSpd) break;
         float piv;
         if (kSpd) {
             // the diagonal pivot (positive for a positive definite A)
@@ -166,11 +231,13 @@ __device__ void invert_warp(Smem &s) {
         __syncwarp();
         return;
     }
-    // X = right half of [I | A^{-1}]
+    // X = right half of [I | A^{-1}] (kSpd: lane 0 has written it)
+    if (!kSpd) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int c = 8 * h + j;
-        if (act && c >= D) s.gjf[r][c - D] = row[j];
+        for (int j = 0; j < 8; ++j) {
+            const int c = 8 * h + j;
+            if (act && c >= D) s.gjf[r][c - D] = row[j];
+        }
     }
     __syncwarp();
     // Acceptance: the residual of any fp32-stored inverse has a rounding floor of about
