@@ -211,3 +211,32 @@ def test_ldlq_empty():
     U = torch.zeros((n, n), dtype=torch.float32, device="cuda")
     lcq.lcq_ldlq(W, dev(config_A(d, np.random.default_rng(1))), dev(np.zeros(d, np.float32)), U, d, ws, mse=mse)
     assert float(mse.item()) == 0.0
+
+
+def test_ldl_factor_captured_in_a_cuda_graph():
+    """The factorisation forks each panel onto a library side stream and joins it back with events:
+    captured into a CUDA graph and replayed it gives the eager result, and work after the replay on
+    the capturing stream sees every output."""
+    torch = T()
+    n, d = 520, 8
+    H = dev(wl.draw_hessian(n, 17, n))
+    U_eager, D_eager = gpu_factor(H.cpu().numpy(), d)
+    U = torch.empty((n, n), dtype=torch.float32, device="cuda")
+    D = torch.empty((n // d, d, d), dtype=torch.float32, device="cuda")
+    ws = lcq.workspace(lcq.LCQ_OP_LDL_FACTOR, 0, 0, n, d)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        lcq.lcq_ldl_factor(H, d, U, ws, D=D)          # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    U.zero_(), D.zero_()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        lcq.lcq_ldl_factor(H, d, U, ws, D=D)
+        checksum = U.abs().sum() + D.abs().sum()      # on the capturing stream, after the join
+    g.replay()
+    torch.cuda.synchronize()
+    assert lcq.lcq_device_status(ws) == 0
+    assert torch.equal(U, U_eager) and torch.equal(D, D_eager)
+    assert float(checksum) == pytest.approx(float(U_eager.abs().sum() + D_eager.abs().sum()), rel=1e-6)
