@@ -672,12 +672,16 @@ template <int D>
 __device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *ab_s, uint8_t *xq_s, float inv, int tile,
                                             int lane, float &r) {
     // X'_g = X_g A, one row of A (16-byte loads from shared memory) at a time, so that the loads of
-    // the next row overlap the FMAs of this one
-    float xp[16];
+    // the next row overlap the FMAs of this one; the rows j < D/2 and j >= D/2 accumulate separately
+    // (half-length dependency chains), added at the end
+    float xp[16], xq[16];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) xp[i] = 0.0f;
+    for (int i = 0; i < 16; ++i) xp[i] = xq[i] = 0.0f;
+    float r2 = 0.0f;
 #pragma unroll
     for (int j = 0; j < D; ++j) {
+        float (&acc)[16] = j < D / 2 ? xp : xq;
+        float &racc = j < D / 2 ? r : r2;
         float arow[D];
 #pragma unroll
         for (int h = 0; h < D / 4; ++h) {
@@ -691,16 +695,24 @@ __device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *a
             const float2 xx = make_float2(xj, xj);
 #pragma unroll
             for (int k = 0; k < D; k += 2) {
-                const float2 v = __ffma2_rn(xx, make_float2(arow[k], arow[k + 1]), make_float2(xp[g * D + k], xp[g * D + k + 1]));
-                xp[g * D + k] = v.x;
-                xp[g * D + k + 1] = v.y;
+                const float2 v = __ffma2_rn(xx, make_float2(arow[k], arow[k + 1]), make_float2(acc[g * D + k], acc[g * D + k + 1]));
+                acc[g * D + k] = v.x;
+                acc[g * D + k + 1] = v.y;
             }
-            r = fmaf(xj, bj, r);
+            racc = fmaf(xj, bj, racc);
         }
     }
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+        const float2 v = __fadd2_rn(make_float2(xp[i], xp[i + 1]), make_float2(xq[i], xq[i + 1]));
+        xp[i] = v.x;
+        xp[i + 1] = v.y;
+    }
+    r += r2;
     // round to int16: v + 1.5 * 2^23 holds round(v) (ties to even) in its low mantissa bits for
-    // |v| < 2^22, so the low 16 bits are the two's-complement int16; |v| <= 32767 by the choice of inv
-    // (clamped all the same)
+    // |v| < 2^22, so the low 16 bits are the two's-complement int16. |v| <= 32767 (1 + 16 * 2^-24) for
+    // finite X: |X'| <= max|X| max_k sum_j |A_jk| up to the FMA rounding, and inv is that bound's
+    // 32767 / bound to 2 ulp, so round(v) stays in [-32767, 32767] without a clamp
     constexpr int kFirst[8] = {0, 8, 1, 9, 2, 10, 3, 11};
     constexpr float kMagic = 12582912.0f;
     uint32_t words[8];
@@ -708,8 +720,8 @@ __device__ __forceinline__ void dp_quantize(const float (&x)[16], const float *a
     for (int k = 0; k < 8; ++k) {
         const int cc = kFirst[k];
         const float f = (cc & 1) ? 0.25f * inv : inv;
-        const float lo = fminf(fmaxf(xp[cc] * f, -32767.0f), 32767.0f) + kMagic;
-        const float hi = fminf(fmaxf(xp[cc + 4] * f, -32767.0f), 32767.0f) + kMagic;
+        const float lo = fmaf(xp[cc], f, kMagic);
+        const float hi = fmaf(xp[cc + 4], f, kMagic);
         words[k] = __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x5410);
     }
     uint4 *dst = reinterpret_cast<uint4 *>(xq_s + static_cast<size_t>(tile) * 1024);
