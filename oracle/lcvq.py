@@ -22,7 +22,7 @@ inverse) with no blocking, fusion or reordering:
                         corrected by the earlier groups' errors through the
                         block U D U^T factor of the proxy Hessian (Sec. 2.2)
 
-Readings where the paper is silent or inconsistent (listed in the design doc):
+Readings where the paper is silent or inconsistent:
   * encode maps a real weight group to latent coordinates u = A^{-1}(w - B)
     and rounds/clamps u (Sec. 2.2 "rounding and clamping", Babai rounding);
   * round is round-half-to-even; NaN latent values encode to 0;
