@@ -30,6 +30,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Dynamic shared memory rounded up to a 1024-byte boundary (where the 128-byte swizzle pattern of TMA
+// tiles repeats). The offset comes from the 32-bit shared address and is added to the __shared__
+// pointer itself, so the compiler still knows the result points into shared memory and emits shared
+// loads and stores with 32-bit addresses (a round trip through an integer would leave it generic).
+__device__ __forceinline__ uint8_t *align_smem_1024(uint8_t *raw) {
+    return raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
+}
+
 // ------------------------------------------------------------------ mbarrier
 
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {

@@ -374,7 +374,7 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
     constexpr uint32_t kCodeBytes = static_cast<uint32_t>(R) * 128u;
     constexpr uint32_t kActStride = 8u * NT * 1024u;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *base = align_smem_1024(smem_raw);
     const GemvTmaLayout L = gemv_tma_layout(R, p.stages, NT, CWR, RBW, KS);
     uint8_t *acts = base + L.acts;
     float *red = reinterpret_cast<float *>(base + L.red);
@@ -774,7 +774,7 @@ __global__ void __launch_bounds__(32 * (kDpWarps + 1), 1)
 packed_gemv_dp_kernel(const __grid_constant__ CUtensorMap tmC, const GemvDpParams p) {
     constexpr int CW = kDpWarps;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *base = align_smem_1024(smem_raw);
     const DpSmemLayout L = dp_smem_layout(p.R, p.stages, p.nkc);
     float *red_s = reinterpret_cast<float *>(base + L.red);   // [2][CW]: max|X|, then sum X_g . b
     float *ab_s = reinterpret_cast<float *>(base + L.ab);

@@ -364,7 +364,7 @@ __global__ void __launch_bounds__(kSwThreads, 1)
 ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmE,
                   const __grid_constant__ CUtensorMap tmW, const SweepParams p) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    SweepSmem &s = *reinterpret_cast<SweepSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    SweepSmem &s = *reinterpret_cast<SweepSmem *>(align_smem_1024(smem_raw));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t n = p.n, tile = blockIdx.x;
     const int nchunks = static_cast<int>((n + kSwC - 1) / kSwC);
