@@ -573,7 +573,8 @@ def main():
 
 def e2e_arm(torch, lcq, wl, args, device, world, rank):
     """Same step through the public API with the step's inputs in pinned host memory: every step copies
-    W, X, dY host->device and reads dA, db, MSE and the packed-product output back to the host."""
+    W, X, dY host->device (on a copy stream, overlapping the previous linear's kernels) and reads dA, db,
+    MSE and the packed-product output back to the host."""
     layer = [Linear(torch, lcq, wl, mx, args.seed + 7919 * rank, i, device)
              for i, mx in enumerate(wl.llama3_8b_layer())]
     host = []
@@ -587,18 +588,35 @@ def e2e_arm(torch, lcq, wl, args, device, world, rank):
     h2d = sum(h["W"].numel() * 4 + h["X"].numel() * 2 + h["dY"].numel() * 2 for h in host)
     d2h = sum(h["dA"].numel() * 4 + h["db"].numel() * 4 + 8 + h["Yg"].numel() * 2 for h in host)
 
+    # The host->device copies run on their own stream, so a linear's inputs arrive while the previous
+    # linear computes; events order each linear's compute after its copies, and the next step's copies
+    # into a linear's buffers after that linear's compute. Every step still copies all its inputs and
+    # reads its results back before it ends.
+    main = torch.cuda.current_stream(device)
+    copy_stream = torch.cuda.Stream(device=device)
+    copied = [torch.cuda.Event() for _ in layer]
+    consumed = [torch.cuda.Event() for _ in layer]
+    for ev in consumed:
+        ev.record(main)
+
     def step():
-        for L, h in zip(layer, host):
-            L.W.copy_(h["W"], non_blocking=True)
-            L.X.copy_(h["X"], non_blocking=True)
-            L.dY.copy_(h["dY"], non_blocking=True)
+        with torch.cuda.stream(copy_stream):
+            for L, h, cp, used in zip(layer, host, copied, consumed):
+                copy_stream.wait_event(used)
+                L.W.copy_(h["W"], non_blocking=True)
+                L.X.copy_(h["X"], non_blocking=True)
+                L.dY.copy_(h["dY"], non_blocking=True)
+                cp.record(copy_stream)
+        for L, h, cp, used in zip(layer, host, copied, consumed):
+            main.wait_event(cp)
             L.Xg.copy_(L.X[:GEMV_TOKENS])
             L.step(lcq)
+            used.record(main)
             h["dA"].copy_(L.dA, non_blocking=True)
             h["db"].copy_(L.db, non_blocking=True)
             h["mse"].copy_(L.mse, non_blocking=True)
             h["Yg"].copy_(L.Yg, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        main.synchronize()
 
     from paper_2606_10531_gb300 import dist as lcq_dist
     for _ in range(max(args.warmup, 3)):
