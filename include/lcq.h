@@ -209,9 +209,11 @@ lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const 
                       float *W_hat_f32, uint16_t *W_hat_bf16, void *stream);
 
 /*
- * lcq_pack2b - pack one-code-per-byte codes [m][n] into [m][n/4] bytes in the
- * library's bit order (see the header comment). Only the two low bits of
- * each input byte are used. n must be a multiple of 4. Needs no workspace.
+ * lcq_pack2b - storage of the 2-bit codes (Sec. 2.1: in the 2-bit setting each
+ * dimension takes one of 4 values, so four codes fill a byte). Packs
+ * one-code-per-byte codes [m][n] into [m][n/4] bytes in the library's bit
+ * order (see the header comment). Only the two low bits of each input byte are
+ * used. n must be a multiple of 4. Needs no workspace.
  */
 lcq_status lcq_pack2b(const uint8_t *codes, int64_t m, int64_t n, uint8_t *packed, void *stream);
 
