@@ -137,3 +137,20 @@ def test_encode_batch_validation(L):
     assert L.lcq_workspace_size(6, 0, 0, 0, 8) == 0
     assert L.lcq_workspace_size(6, 17, 0, 0, 8) == 0
     assert 0 < L.lcq_workspace_size(6, 1, 0, 0, 8) < L.lcq_workspace_size(6, 7, 0, 0, 8)
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(ImportError, match="liblcq.so not found"):
+        lcq.load_library(str(tmp_path / "liblcq.so"))
+
+
+def test_product_package_never_reaches_the_oracle():
+    """The binding and the library sources import, link or execute nothing under oracle/."""
+    pkg = os.path.join(ROOT, "paper_2606_10531_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath or "__pycache__" in dirpath:
+            continue
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp", ".c")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b|oracle/|brute\.c|lcvq", text, flags=re.M), f
