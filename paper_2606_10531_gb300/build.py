@@ -25,14 +25,19 @@ def nvcc() -> str:
     raise RuntimeError("nvcc not found")
 
 
+def ptxas_report(src: str) -> str:
+    """Path of the per-kernel resource report (registers, spills, shared memory) ptxas printed for src."""
+    return os.path.join(BUILD, os.path.splitext(src)[0] + ".ptxas.txt")
+
+
 def _compile(src: str, verbose_ptxas: bool) -> str:
     obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
-    cmd = [nvcc(), *ARCH, *NVCC_FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
-    if verbose_ptxas:
-        cmd += ["-Xptxas", "-v"]
+    cmd = [nvcc(), *ARCH, *NVCC_FLAGS, "-Xptxas", "-v", "-c", os.path.join(CSRC, src), "-o", obj]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+    with open(ptxas_report(src), "w") as f:
+        f.write(r.stderr)
     if verbose_ptxas:
         sys.stderr.write(r.stderr)
     return obj
