@@ -527,11 +527,13 @@ def main():
     per_launch_flops = g_flops / g_launch if g_launch else None
     traffic = traffic_from_profile(os.path.join(ROOT, "paper_2606_10531_gb300", "csrc", "gemm_tc.cu"))
     total_trace_ms = sum(v[1] for v in trace.values())
+    # The timed region lasts well under the seconds-long loop the sustained peak was measured over, so
+    # the fraction is taken against the burst peak; the sustained one is reported beside it.
     roofline = {"kernel": "gemm_tc (tcgen05/TMEM, TMA) fwd + dX + dW launches", "bound": "tensor",
-                "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
-                "frac": (achieved / pk["bf16_sustained"]) if achieved else None,
-                "frac_of_burst_peak": (achieved / pk["bf16"]) if achieved else None,
-                "peak_kind": f"bf16_tflops_sustained ({pk['src']}); kernel timed inside a long step",
+                "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+                "frac": (achieved / pk["bf16"]) if achieved else None,
+                "frac_of_sustained_peak": (achieved / pk["bf16_sustained"]) if achieved else None,
+                "peak_kind": f"bf16_tflops burst ({pk['src']}); timed region {elapsed:.2f} s",
                 "traffic": traffic, "flops_per_launch": per_launch_flops, "launches": g_launch,
                 "share_of_kernel_time": g_ms / total_trace_ms if total_trace_ms else None}
     breakdown = {k: {"launches": v[0], "ms_per_step": v[1] / args.steps} for k, v in trace.items()}
@@ -567,56 +569,93 @@ def main():
                                           f"64 of 16384 tokens; {spent:.1f} s of CPU work"}
     lcq_dist.barrier()
     if rank == 0:
+        line["summary"] = summary(line)
         print(json.dumps(line), flush=True)
     lcq_dist.finalize()
 
 
+def summary(line):
+    """Compact headline figures, placed last in the JSON line so that the end of the output holds them."""
+    r3 = lambda x: None if x is None else round(float(x), 3)    # noqa: E731
+    out = {"layer_step_tflops": r3(line["value"]), "layer_frac_bf16_burst": r3(line["frac_bf16_peak"]),
+           "gemm_frac_bf16_burst": r3(line["roofline"]["frac"])}
+    if "e2e" in line:
+        out["e2e_tflops"] = r3(line["e2e"]["value"])
+    enc = line.get("encode")
+    if enc:
+        out["encode70b_mse_ms"] = r3(enc["ms"])
+        out["encode70b_mse_frac_hbm"] = r3(enc["frac_hbm"])
+        out["encode70b_codes_only_frac_hbm"] = r3(enc["codes_only"]["frac_hbm"])
+    pd = line.get("packed_decode")
+    if pd:
+        for k in ("B1", "B2", "B4", "B16", "B1_hadamard"):
+            if k in pd:
+                out[f"packed_{k}_us"] = r3(pd[k]["us"])
+                out[f"packed_{k}_frac_hbm"] = r3(pd[k]["frac_hbm"])
+    ld = line.get("ldlq_init")
+    if ld:
+        out["ldlq_factor_ms"] = r3(ld["factor_ms"])
+        out["ldlq_sweep_ms"] = r3(ld["sweep_ms"])
+        out["ldlq_sweep_frac_fp32"] = r3(ld["roofline"]["frac"])
+    ot = line.get("other_training_workloads")
+    if ot:
+        for k, v in ot.items():
+            if k.startswith("llama2"):
+                out[f"{k}_tflops"] = r3(v["TFLOP/s"])
+    return out
+
+
 def e2e_arm(torch, lcq, wl, args, device, world, rank):
-    """Same step through the public API with the step's inputs in pinned host memory: every step copies
-    W, X, dY host->device (on a copy stream, overlapping the previous linear's kernels) and reads dA, db,
-    MSE and the packed-product output back to the host."""
+    """Same step through the public API with the step's inputs and results in pinned host memory:
+    every step copies W, X, dY host->device and reads every result of the step back device->host
+    (Y, dX, dP, dA, db, the MSE and the packed-product output). Copies run on two copy streams: a
+    linear's inputs arrive while the previous linear computes, and its results leave while the next
+    one computes."""
     layer = [Linear(torch, lcq, wl, mx, args.seed + 7919 * rank, i, device)
              for i, mx in enumerate(wl.llama3_8b_layer())]
+    outs = ("Y", "dX", "dP", "dA", "db", "mse", "Yg")
     host = []
     for L in layer:
-        h = {"W": L.W.cpu().pin_memory(), "X": L.X.cpu().pin_memory(), "dY": L.dY.cpu().pin_memory(),
-             "dA": torch.empty_like(L.dA, device="cpu").pin_memory(),
-             "db": torch.empty_like(L.db, device="cpu").pin_memory(),
-             "mse": torch.empty_like(L.mse, device="cpu").pin_memory(),
-             "Yg": torch.empty_like(L.Yg, device="cpu").pin_memory()}
+        h = {"W": L.W.cpu().pin_memory(), "X": L.X.cpu().pin_memory(), "dY": L.dY.cpu().pin_memory()}
+        for k in outs:
+            t = getattr(L, k)
+            h[k] = torch.empty(t.shape, dtype=t.dtype, device="cpu").pin_memory()
         host.append(h)
-    h2d = sum(h["W"].numel() * 4 + h["X"].numel() * 2 + h["dY"].numel() * 2 for h in host)
-    d2h = sum(h["dA"].numel() * 4 + h["db"].numel() * 4 + 8 + h["Yg"].numel() * 2 for h in host)
+    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("W", "X", "dY"))
+    d2h = sum(h[k].numel() * h[k].element_size() for h in host for k in outs)
 
-    # The host->device copies run on their own stream, so a linear's inputs arrive while the previous
-    # linear computes; events order each linear's compute after its copies, and the next step's copies
-    # into a linear's buffers after that linear's compute. Every step still copies all its inputs and
-    # reads its results back before it ends.
+    # Events order each linear's compute after its input copies and after the previous step's result
+    # copies out of its buffers; the next step's input copies wait for the compute that reads them.
     main = torch.cuda.current_stream(device)
-    copy_stream = torch.cuda.Stream(device=device)
+    cin = torch.cuda.Stream(device=device)
+    cout = torch.cuda.Stream(device=device)
     copied = [torch.cuda.Event() for _ in layer]
-    consumed = [torch.cuda.Event() for _ in layer]
-    for ev in consumed:
+    computed = [torch.cuda.Event() for _ in layer]
+    drained = [torch.cuda.Event() for _ in layer]
+    for ev in computed + drained:
         ev.record(main)
 
     def step():
-        with torch.cuda.stream(copy_stream):
-            for L, h, cp, used in zip(layer, host, copied, consumed):
-                copy_stream.wait_event(used)
+        with torch.cuda.stream(cin):
+            for L, h, cp, done in zip(layer, host, copied, computed):
+                cin.wait_event(done)
                 L.W.copy_(h["W"], non_blocking=True)
                 L.X.copy_(h["X"], non_blocking=True)
                 L.dY.copy_(h["dY"], non_blocking=True)
-                cp.record(copy_stream)
-        for L, h, cp, used in zip(layer, host, copied, consumed):
+                cp.record(cin)
+        for L, h, cp, done, out in zip(layer, host, copied, computed, drained):
             main.wait_event(cp)
+            main.wait_event(out)
             L.Xg.copy_(L.X[:GEMV_TOKENS])
             L.step(lcq)
-            used.record(main)
-            h["dA"].copy_(L.dA, non_blocking=True)
-            h["db"].copy_(L.db, non_blocking=True)
-            h["mse"].copy_(L.mse, non_blocking=True)
-            h["Yg"].copy_(L.Yg, non_blocking=True)
+            done.record(main)
+            with torch.cuda.stream(cout):
+                cout.wait_event(done)
+                for k in outs:
+                    h[k].copy_(getattr(L, k), non_blocking=True)
+                out.record(cout)
         main.synchronize()
+        cout.synchronize()
 
     from paper_2606_10531_gb300 import dist as lcq_dist
     for _ in range(max(args.warmup, 3)):
@@ -632,7 +671,8 @@ def e2e_arm(torch, lcq, wl, args, device, world, rank):
     del layer, host
     torch.cuda.empty_cache()
     return {"value": flops / el / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "ms_per_step": el / args.steps * 1e3, "api": "paper_2606_10531_gb300 ctypes binding of liblcq"}
+            "ms_per_step": el / args.steps * 1e3, "api": "paper_2606_10531_gb300 ctypes binding of liblcq",
+            "copies": "inputs W, X, dY in; results Y, dX, dP, dA, db, MSE, packed-product output out; pinned host"}
 
 
 def profile_case(args):

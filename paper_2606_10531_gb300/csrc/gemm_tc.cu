@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // 1024-byte alignment of the stage buffers is required by the 128B swizzle atoms.
-    GemmSmem &s = *reinterpret_cast<GemmSmem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    GemmSmem &s = *reinterpret_cast<GemmSmem *>(align_smem_1024(smem_raw));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int num_m = (p.M + BM - 1) / BM, num_n = (p.N + BN - 1) / BN;
     const int num_tiles = num_m * num_n;

@@ -50,7 +50,9 @@ extern "C" lcq_status lcq_gemm_packed2b_noalloc(const uint16_t *X, int64_t N, co
                                                 int64_t n, int d, const float *A, const float *b, uint16_t *Y,
                                                 int32_t *device_status, void *stream) {
     using namespace lcq;
-    if (N < 0 || m < 0 || n < 0) return LCQ_ERR_SHAPE;
+    // every argument is checked before the status word is cleared, so a rejected call enqueues nothing
+    const lcq_status arg = check_gemm_packed2b_args(X, N, packed, m, n, d, A, b, Y);
+    if (arg != LCQ_OK) return arg;
     if (N > kNoallocMaxTokens || n > kNoallocMaxN) return LCQ_ERR_LIMIT;
     if (device_status && (reinterpret_cast<uintptr_t>(device_status) & 3u)) return LCQ_ERR_ALIGN;
     const size_t need = lcq_workspace_size(LCQ_OP_GEMM_PACKED2B, N, m, n, d);

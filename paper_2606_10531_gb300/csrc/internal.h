@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "../../include/lcq.h"
+
 namespace lcq {
 
 void count_launch();
@@ -170,6 +172,9 @@ struct PackedGemvArgs {
     int32_t *status;
     bool rotate = false;     // rotate X by the block Walsh-Hadamard transform in the product's prologue
 };
+// Argument checks of lcq_gemm_packed2b other than the workspace (LCQ_OK or the error it returns).
+lcq_status check_gemm_packed2b_args(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n, int d,
+                                    const float *A, const float *b, const uint16_t *Y);
 size_t packed_gemv_workspace(int64_t N, int64_t n);
 size_t packed_gemv_corr_offset(int64_t N, int64_t n);
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);

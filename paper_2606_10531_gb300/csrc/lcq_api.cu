@@ -159,6 +159,20 @@ static lcq_status opts_of(const lcq_opts *o, float &inv_s, float &t, int &ste, f
     return LCQ_OK;
 }
 
+// Argument checks of lcq_gemm_packed2b (everything but the workspace); also used by the
+// allocation-free variant before it enqueues anything.
+lcq_status check_gemm_packed2b_args(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n, int d,
+                                    const float *A, const float *b, const uint16_t *Y) {
+    lcq_status s = check_common(m, n, d);
+    if (s != LCQ_OK) return s;
+    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    if ((s = check_tensor(X, N * n)) != LCQ_OK) return s;
+    if ((s = check_tensor(packed, m * n)) != LCQ_OK) return s;
+    if ((s = check_tensor(Y, N * m)) != LCQ_OK) return s;
+    if (!A || !b) return LCQ_ERR_NULL;
+    return LCQ_OK;
+}
+
 }  // namespace lcq
 
 using namespace lcq;
@@ -586,12 +600,7 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
 
 lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n, int d,
                              const float *A, const float *b, uint16_t *Y, void *ws, size_t ws_bytes, void *stream) {
-    LCQ_TRY(check_common(m, n, d));
-    if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
-    LCQ_TRY(check_tensor(X, N * n));
-    LCQ_TRY(check_tensor(packed, m * n));
-    LCQ_TRY(check_tensor(Y, N * m));
-    if (!A || !b) return LCQ_ERR_NULL;
+    LCQ_TRY(check_gemm_packed2b_args(X, N, packed, m, n, d, A, b, Y));
     LCQ_TRY(check_ws(ws, ws_bytes, lcq_workspace_size(LCQ_OP_GEMM_PACKED2B, N, m, n, d)));
     cudaStream_t st = as_stream(stream);
     if (N * m == 0) return LCQ_OK;

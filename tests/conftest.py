@@ -12,11 +12,6 @@ def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built liblcq.so")
 
 
-def pytest_collection_modifyitems(config, items):
-    # Run GPU parity files in a stable order; the no-allocation test file sorts last by name.
-    pass
-
-
 @pytest.fixture(scope="session")
 def golden_dir():
     return os.path.join(ROOT, "tests", "golden")
