@@ -271,7 +271,7 @@ lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed
  * with a hard memory budget), and for C callers with no device allocator.
  *
  * Same arguments and results as lcq_gemm_packed2b, without ws/ws_bytes: the
- * scratch lives in one static device array of about 1 MiB that every GPU
+ * scratch lives in one static device array of 1.25 MiB + 4 KiB that every GPU
  * which loads the library holds until the process exits. The call itself
  * allocates nothing (no cudaMalloc, cudaFree or allocating library routine).
  *   - Limits: N <= 16 tokens and n <= 32768; larger problems return

@@ -12,7 +12,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblcq.so")
-SOURCES = ["lcq_api.cu", "kernels_elem.cu", "gemm_tc.cu", "gemv_packed.cu", "gemv_noalloc.cu", "ldlq.cu"]
+SOURCES = ["lcq_api.cu", "kernels_elem.cu", "gemm_tc.cu", "gemv_packed.cu", "gemv_fp4.cu", "gemv_noalloc.cu", "ldlq.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I" + os.path.join(ROOT, "include")]

@@ -20,7 +20,7 @@ namespace lcq {
 // Largest problem the static scratch holds: 16 tokens, n <= 32768 (see lcq.h).
 constexpr int64_t kNoallocMaxTokens = 16;
 constexpr int64_t kNoallocMaxN = 32768;
-constexpr size_t kNoallocScratchBytes = (size_t(1) << 20) + 4096;
+constexpr size_t kNoallocScratchBytes = (size_t(5) << 18) + 4096;   // 1.25 MiB + 4 KiB
 
 static __device__ __align__(256) unsigned char g_gemv_scratch[kNoallocScratchBytes];
 

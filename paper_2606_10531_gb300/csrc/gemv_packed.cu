@@ -612,6 +612,7 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
 // Launched with programmatic dependent launch: the code stream starts while the previous kernel in
 // the stream finishes; the consumers wait for it (griddepcontrol.wait) before reading X.
 
+constexpr int kFp4MinTokens = 8;          // the tcgen05 fp4 kernel takes more tokens than this
 constexpr int kDpMaxTokens = 1;            // two tokens measured slower than the tensor-core kernel
 constexpr int kDpWarps = 16;               // consumer warps (a multiple of 8)
 constexpr int64_t kDpMaxN = 32768;         // integer row sums stay below 2^31
@@ -1129,7 +1130,9 @@ cudaError_t launch_hadamard(const void *in, bool in_bf16, int64_t rows, int64_t 
 size_t packed_gemv_workspace(int64_t N, int64_t n) {
     const size_t xp = static_cast<size_t>(N) * static_cast<size_t>(gemv_npad(n)) * 2;
     const size_t cr = static_cast<size_t>(N) * static_cast<size_t>(gemv_nprep(n)) * 4;
-    return ((xp + 255) / 256) * 256 + ((cr + 255) / 256) * 256;
+    const size_t mma_sync_path = ((xp + 255) / 256) * 256 + ((cr + 255) / 256) * 256;
+    const size_t fp4_path = packed_gemv_fp4_workspace(N, n);
+    return mma_sync_path > fp4_path ? mma_sync_path : fp4_path;
 }
 
 size_t packed_gemv_corr_offset(int64_t N, int64_t n) {
@@ -1307,6 +1310,16 @@ bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cud
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st) {
     const int64_t npad = gemv_npad(a.n), nprep = gemv_nprep(a.n);
     trace_begin(LCQ_K_GEMV, st);
+    if (a.N > kFp4MinTokens) {
+        // 9-16 tokens, n % 64 == 0: codes as fp4 tensor-core operands in tensor memory (tcgen05); at
+        // 2-8 tokens the mma.sync kernel below measured faster (18.9 against 20.2 us on the 70B gate)
+        cudaError_t e = cudaSuccess;
+        if (launch_packed_gemv_fp4(a, d, num_sms, st, e)) {
+            if (e != cudaSuccess) return e;
+            trace_end(LCQ_K_GEMV, st);
+            return cudaGetLastError();
+        }
+    }
     if (a.n % 64 == 0 && a.n <= kDpMaxN && a.m >= 16 && a.N == kDpMaxTokens) {
         bool done = false;
         const cudaError_t e = launch_packed_gemv_dp(a, d, num_sms, st, done);

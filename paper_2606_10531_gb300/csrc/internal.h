@@ -178,6 +178,11 @@ lcq_status check_gemm_packed2b_args(const uint16_t *X, int64_t N, const uint8_t 
 size_t packed_gemv_workspace(int64_t N, int64_t n);
 size_t packed_gemv_corr_offset(int64_t N, int64_t n);
 cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st);
+// The tcgen05 (kind::mxf4) product for 1-16 tokens and n % 64 == 0, with its digits and constants in
+// the workspace at a.Xp. Returns false (nothing launched) when it does not apply; err holds a launch
+// error otherwise.
+size_t packed_gemv_fp4_workspace(int64_t N, int64_t n);
+bool launch_packed_gemv_fp4(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err);
 // The rotated product with the rotation in the one-token kernel's prologue. Returns false (nothing
 // launched) when that kernel does not apply; err holds a launch error otherwise.
 bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err);

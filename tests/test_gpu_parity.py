@@ -487,3 +487,49 @@ def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)
     lcq.lcq_gemm_packed2b_hadamard(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
+
+
+# 9-16 tokens with n % 64 == 0 take the tcgen05 kernel (kind::mxf4): the codes are fp4 operands in
+# tensor memory and the activations exact integer digits, q = rint(X' 8191 / max|X'_t|) per token, so
+# its only errors are that rounding (at most 2^-14 of max|X'_t| per element) and the bf16 output
+# rounding: it is held to the tighter bound of the one-token kernel, on heavy-tailed activations.
+# The shapes cover ragged rows (not a multiple of 32 or 128), a partial last 512-column tile, ranges
+# of one to eight 32-row slices, and more rows than one wave of CTAs holds (several ranges per CTA).
+@pytest.mark.parametrize("N", [9, 12, 16])
+@pytest.mark.parametrize("m,n,d", [(1000, 4096, 8), (300, 8192, 4), (77, 576, 8), (129, 1088, 4), (2500, 512, 8),
+                                   (40000, 64, 8)])
+def test_gemm_packed2b_tcgen05_heavy_tailed(N, m, n, d):
+    rng = np.random.default_rng(11 * N + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n))
+    X[:, rng.random(n) < 0.01] *= 50.0
+    Xb = wl.bf16_bits(X.astype(np.float32))
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+    lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    assert max_rel(host_bf16(Y), ref) <= TOL_DP
+
+
+def test_gemm_packed2b_tcgen05_zero_token_and_repeat():
+    """A token of zeros (scale 0) beside others; two calls in a row give identical bytes (the
+    accumulators hold exact integer sums, so the result does not depend on the order of the sums)."""
+    torch = T()
+    rng = np.random.default_rng(5)
+    N, m, n, d = 12, 700, 2048, 8
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n)).astype(np.float32)
+    X[3] = 0.0
+    Xb = wl.bf16_bits(X)
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+    Y1, Y2 = empty_bf16(N, m), empty_bf16(N, m)
+    Xd, Pd, Ad, bd = dev_bf16(Xb), dev(oracle.pack2b(Z)), dev(A), dev(b)
+    lcq.lcq_gemm_packed2b(Xd, Pd, n, d, Ad, bd, Y1, ws)
+    lcq.lcq_gemm_packed2b(Xd, Pd, n, d, Ad, bd, Y2, ws)
+    assert torch.equal(Y1, Y2)
+    assert float(Y1[3].float().abs().max()) == 0.0
+    assert max_rel(host_bf16(Y1), ref) <= TOL_DP
