@@ -17,6 +17,7 @@ from tests.gpu_util import TOL_BF16, dev, dev_bf16, empty_bf16, host_bf16, ldlq_
 pytestmark = pytest.mark.gpu
 
 SEED = 0
+SAMPLES = 32      # tokens and weight rows recomputed one by one in fp64
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -63,22 +64,23 @@ def _check_linear(mx, index):
     X, dY = wl.bf16_to_f32(Xb).astype(np.float64), wl.bf16_to_f32(dYb).astype(np.float64)
     W_hat = oracle.decode(Z, A, b, d)
     rng = np.random.default_rng(1234 + index)
-    toks = rng.choice(N, 8, replace=False)
-    rows = rng.choice(m, 8, replace=False)
+    k = SAMPLES
+    toks = rng.choice(N, k, replace=False)
+    rows = rng.choice(m, k, replace=False)
     # sampled rows of Y = X W_hat^T and dX = dY W_hat
     Yg, dXg = host_bf16(Y), host_bf16(dX)
     assert max_rel(Yg[toks], X[toks] @ W_hat.T) <= TOL_BF16
     assert max_rel(dXg[toks], dY[toks] @ W_hat) <= TOL_BF16
     # sampled rows of dP = (dY^T X)_g A
-    dW_rows = dY[:, rows].T @ X                                    # 8 x n
-    dP_ref = (dW_rows.reshape(8, n // d, d) @ A.astype(np.float64)).reshape(8, n)
+    dW_rows = dY[:, rows].T @ X                                    # k x n
+    dP_ref = (dW_rows.reshape(k, n // d, d) @ A.astype(np.float64)).reshape(k, n)
     assert max_rel(dP.cpu().numpy()[rows], dP_ref) <= TOL_BF16
-    # db, dA through their row-sum identities (any size)
+    # db, dA through their row-sum identities (any size), in fp64
     rho = dY.sum(axis=1)
     sig = X.reshape(N, n // d, d).sum(axis=1)
     assert max_rel(db.cpu().numpy(), rho @ sig) <= TOL_BF16
-    T = (wl.bf16_to_f32(dYb) @ Z.astype(np.float32)).astype(np.float64)      # dY Z, N x n
-    dA_ref = np.einsum("tgj,tgk->jk", X.reshape(N, n // d, d), T.reshape(N, n // d, d))
+    T = dY @ Z.astype(np.float64)                                  # dY Z, N x n
+    dA_ref = X.reshape(N * (n // d), d).T @ T.reshape(N * (n // d), d)
     assert max_rel(dA.cpu().numpy(), dA_ref) <= TOL_BF16
 
 
@@ -87,9 +89,24 @@ def test_llama3_8b_gate_fwd_bwd_full_size():
     _check_linear(mats[4], 4)         # gate 14336 x 4096, d = 8, 16384 tokens
 
 
+def test_llama3_8b_down_fwd_bwd_full_size():
+    mats = wl.llama3_8b_layer()
+    _check_linear(mats[6], 6)         # down 4096 x 14336: K = 14336 in the forward, the widest dW epilogue
+
+
+def test_llama3_8b_k_fwd_bwd_full_size():
+    mats = wl.llama3_8b_layer()
+    _check_linear(mats[1], 1)         # k 1024 x 4096: eight 128-row blocks of weight rows
+
+
 def test_llama2_7b_gate_fwd_bwd_full_size_d4_outliers():
     mats = wl.llama2_7b_projections(d=4)
     _check_linear(mats[4], 4)         # gate 11008 x 4096, d = 4, 4096 tokens, 1% outlier channels x20
+
+
+def test_llama2_7b_gate_fwd_bwd_full_size_d8_outliers():
+    mats = wl.llama2_7b_projections(d=8)
+    _check_linear(mats[4], 4)         # gate 11008 x 4096, d = 8, 4096 tokens, 1% outlier channels x20
 
 
 @pytest.mark.parametrize("B", [1, 4, 16])
@@ -191,3 +208,39 @@ def test_llama3_70b_gate_ldlq_full_size():
         sq += float(np.sum((W[r0:r0 + 2048].astype(np.float64) - oracle.decode(Z[r0:r0 + 2048], A, b, d)) ** 2))
     ref_mse = sq / (m * n)
     assert abs(mse.item() - ref_mse) <= 1e-5 * ref_mse
+
+
+def test_llama3_70b_layer_bulk_encode_batch_full_size():
+    """The bulk encode that bench.py times: all seven linears of a Llama-3-70B layer (855,638,016
+    weights, d = 8, heavy-tailed) in one lcq_encode_batch call with packed codes and MSE per matrix,
+    checked against the oracle matrix by matrix in row chunks (codes bit-exact away from rounding
+    boundaries, MSE to 1e-4 relative)."""
+    import torch
+    mats = wl.llama3_70b_layer_encode()
+    items, host = [], []
+    for i, mx in enumerate(mats):
+        W = wl.draw_W(mx, SEED + 1000, i)
+        A, b = wl.draw_A(mx, SEED + 1000, i), wl.draw_b(mx, SEED + 1000, i)
+        packed = torch.empty((mx.m, mx.n // 4), dtype=torch.uint8, device="cuda")
+        mse = torch.empty(1, dtype=torch.float64, device="cuda")
+        items.append({"W": dev(W), "A": dev(A), "b": dev(b), "packed": packed, "mse": mse})
+        host.append((mx, W, A, b))
+    ws = lcq.workspace(lcq.LCQ_OP_ENCODE_BATCH, len(items), 0, 0, mats[0].d)
+    lcq.lcq_encode_batch(items, mats[0].d, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    near_total = 0
+    for (mx, W, A, b), it in zip(host, items):
+        got = it["packed"].cpu().numpy()
+        it["W"] = None
+        sq, mismatch = 0.0, 0
+        for r0 in range(0, mx.m, 2048):
+            ref = oracle.encode(W[r0:r0 + 2048], A, b, mx.d)
+            z = oracle.unpack2b(got[r0:r0 + 2048], mx.n)
+            keep = ~ref["near"]
+            mismatch += int(np.sum((z != ref["codes"]) & keep))
+            near_total += int(np.sum(ref["near"]))
+            sq += ref["mse"] * z.size
+        assert mismatch == 0, mx.name
+        ref_mse = sq / (mx.m * mx.n)
+        assert abs(it["mse"].item() - ref_mse) <= 1e-4 * ref_mse, mx.name
+    print(f"near-boundary codes excluded: {near_total} of {sum(mx.m * mx.n for mx in mats)}")
