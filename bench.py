@@ -361,6 +361,45 @@ def time_training_sets(torch, lcq, wl, seed, device, pk):
     return out
 
 
+def time_xform_8b(torch, lcq, wl, seed, device, pk):
+    """Activation transform X' = X_g A, r = sum_g X_g . b (the activation side of the reformulated
+    forward, Eq. def:forward_x) for the seven linears of the Llama-3-8B layer at 16384 tokens, timed with
+    CUDA events over 5 passes after 2 warm-up passes (inputs larger than L2). This is what a forward
+    through X' Z^T + r would add per layer step in place of the weight decode."""
+    mats = wl.llama3_8b_layer()
+    bufs = []
+    for i, mx in enumerate(mats):
+        X = wl.torch_X(torch, mx, seed + 5000, i, device)
+        bufs.append((mx, X, wl.torch_A(torch, mx, seed + 5000, i, device).contiguous(),
+                     wl.torch_b(torch, mx, seed + 5000, i, device).contiguous(), torch.empty_like(X),
+                     torch.empty(mx.N, dtype=torch.float32, device=device)))
+
+    def run():
+        for mx, X, A, b, Xp, r in bufs:
+            lcq.lcq_activation_transform(X, mx.d, A, b, Xp=Xp, r=r)
+
+    for _ in range(2):
+        run()
+    torch.cuda.synchronize()
+    lcq.lcq_trace_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(5):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    lcq.lcq_trace_enable(False)
+    calls, kms = lcq.lcq_trace_read().get("xform", (0, 0.0))
+    t = e0.elapsed_time(e1) * 1e-3 / 5
+    nbytes = sum(mx.N * mx.n * 4 + mx.N * 4 for mx, *_ in bufs)
+    k_t = kms * 1e-3 / 5 if calls else t
+    del bufs
+    torch.cuda.empty_cache()
+    return {"workload": "llama3-8b layer activations: 7 linears, 16384 tokens x n (4096 for q,k,v,o,gate,up; 14336 for "
+                        "down), d = 8; bf16 X' and fp32 r", "ms_per_layer": t * 1e3, "bytes_per_layer": nbytes,
+            "GB/s": nbytes / k_t / 1e9, "frac_hbm": nbytes / k_t / 1e9 / pk["hbm"]}
+
+
 # fp32 FMA peak of the CUDA cores (the LDLQ sweep is bound by it): 152 SMs x 128 FP32 lanes x 2 flops
 # per FMA x 2.07 GHz maximum SM clock
 FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
@@ -556,6 +595,10 @@ def main():
         line["packed_decode"] = time_gemv_70b(torch, lcq, wl, args.seed, device, pk)
         line["ldlq_init"] = time_ldlq_70b(torch, lcq, wl, args.seed, device, pk)
         line["other_training_workloads"] = time_training_sets(torch, lcq, wl, args.seed, device, pk)
+        line["activation_transform"] = time_xform_8b(torch, lcq, wl, args.seed, device, pk)
+        bd = line["breakdown"]
+        line["activation_transform"]["decode_path_ms_per_layer_step"] = (
+            bd.get("quant_decode", {}).get("ms_per_step", 0.0) + bd.get("decode", {}).get("ms_per_step", 0.0))
         torch.cuda.empty_cache()
         layer = None
 
@@ -597,6 +640,11 @@ def summary(line):
         out["ldlq_factor_ms"] = r3(ld["factor_ms"])
         out["ldlq_sweep_ms"] = r3(ld["sweep_ms"])
         out["ldlq_sweep_frac_fp32"] = r3(ld["roofline"]["frac"])
+    xf = line.get("activation_transform")
+    if xf:
+        out["xform8b_ms"] = r3(xf["ms_per_layer"])
+        out["xform8b_frac_hbm"] = r3(xf["frac_hbm"])
+        out["decode_path8b_ms"] = r3(xf["decode_path_ms_per_layer_step"])
     ot = line.get("other_training_workloads")
     if ot:
         for k, v in ot.items():

@@ -209,6 +209,19 @@ lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const 
                       float *W_hat_f32, uint16_t *W_hat_bf16, void *stream);
 
 /*
+ * lcq_activation_transform - activation side of the reformulated forward (Sec. 3.2,
+ * Eq. def:forward_x), for every token t and group g of d columns:
+ *   X'[t, g*d + k] = sum_j X[t, g*d + j] * A[j][k]     (the row vector X_g times A)
+ *   r[t]           = sum_g sum_j X[t, g*d + j] * b[j]
+ * so that X W_hat^T = X' Z^T + r 1^T for the decoded weights W_hat_g = A z_g + b.
+ * X [N][n] bf16 input; Xp [N][n] bf16 output (rounded to nearest even) or NULL;
+ * r [N] fp32 output or NULL (not both NULL unless N = 0). r is summed in a
+ * fixed order (bitwise reproducible). Needs no workspace.
+ */
+lcq_status lcq_activation_transform(const uint16_t *X, int64_t N, int64_t n, int d, const float *A, const float *b,
+                                    uint16_t *Xp, float *r, void *stream);
+
+/*
  * lcq_pack2b - storage of the 2-bit codes (Sec. 2.1: in the 2-bit setting each
  * dimension takes one of 4 values, so four codes fill a byte). Packs
  * one-code-per-byte codes [m][n] into [m][n/4] bytes in the library's bit
@@ -375,7 +388,8 @@ typedef enum lcq_kernel_kind {
     LCQ_K_GEMV = 9,          /* packed product: activation transform + main  */
     LCQ_K_LDL_FACTOR = 10,   /* LDLQ: block U D U^T factorisation (all its launches) */
     LCQ_K_LDLQ = 11,         /* LDLQ: error-feedback sweep                   */
-    LCQ_K_NUM_KINDS = 12
+    LCQ_K_XFORM = 12,        /* activation transform X' = X_g A, r = X_g . b  */
+    LCQ_K_NUM_KINDS = 13
 } lcq_kernel_kind;
 lcq_status lcq_trace_enable(int on);
 /*

@@ -16,6 +16,7 @@ inverse) with no blocking, fusion or reordering:
   * column grouping     G = n/d groups of d consecutive columns (Sec. 3.2)
   * decode              W_hat^T = [A W_{z,i}^T + B 1^T]_i       (Sec. 3.2, Eq. def:forward)
   * forward             Y = X W_hat^T (nn.Linear orientation)   (Sec. 3.2, Eq. def:forward_x)
+  * activation side     X'_g = X_g A, r = sum_g X_g . B          (Sec. 3.2, Eq. def:forward_x)
   * backward            exact gradients of the linear map, with the
                         straight-through estimator dW_z/dW_p = 1 (Sec. 3.3)
   * LDLQ initialisation column groups quantized in order, each target
@@ -146,6 +147,17 @@ def mse(W, Z, A, b, d: int) -> float:
 def linear_fwd(X, Z, A, b, d: int) -> np.ndarray:
     """Layer output Y = X W_hat^T with W_hat decoded from the integer weights (Eq. def:forward)."""
     return _f64(X) @ decode(Z, A, b, d).T
+
+
+def activation_transform(X, A, b, d: int):
+    """Activation side of the reformulated forward (Sec. 3.2, Eq. def:forward_x): per token and
+    group of d columns, the row vector X_g A, and the bias term r = sum_g X_g . B, so that
+    X W_hat^T = X' Z^T + r 1^T. Returns (X' (N x n), r (N,)) in fp64."""
+    X64 = _f64(X)
+    Xg = _grouped(X64, d)                      # (N, G, d)
+    Xp = (Xg @ _f64(A)).reshape(X64.shape)
+    r = (Xg @ _f64(b)).sum(axis=1)
+    return Xp, r
 
 
 DGE_K = 5.0          # sharpness k of the differentiable gradient estimator (Sec. 4.4)

@@ -29,9 +29,9 @@ EXPORTS = ("lcq_workspace_size", "lcq_encode", "lcq_decode", "lcq_pack2b", "lcq_
            "lcq_gemm_packed2b", "lcq_device_status", "lcq_status_string", "lcq_launch_count", "lcq_trace_enable",
            "lcq_trace_read", "lcq_gemm_packed2b_noalloc", "lcq_last_cuda_error", "lcq_selftest_wait_timeout",
            "lcq_init_codebook", "lcq_init_latent", "lcq_hadamard", "lcq_gemm_packed2b_hadamard", "lcq_encode_batch",
-           "lcq_ldl_factor", "lcq_ldlq")
+           "lcq_ldl_factor", "lcq_ldlq", "lcq_activation_transform")
 KERNEL_KINDS = ("encode", "quant_decode", "decode", "pack", "gemm_fwd", "gemm_dx", "gemm_dw", "reduce",
-                "gemv_prep", "gemv", "ldl_factor", "ldlq")
+                "gemv_prep", "gemv", "ldl_factor", "ldlq", "xform")
 
 
 class LCQError(RuntimeError):
@@ -68,6 +68,7 @@ _SIG = {
     "lcq_ldl_factor": (ctypes.c_int, [_P, _I64, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
     "lcq_ldlq": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "lcq_pack2b": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
+    "lcq_activation_transform": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P]),
     "lcq_linear_fwd": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P,
                                       ctypes.c_size_t, _P]),
     "lcq_linear_bwd": (ctypes.c_int, [_P, _P, _P, _P, _I64, _I64, _I64, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P,
@@ -185,6 +186,13 @@ def lcq_decode(packed, n: int, d: int, A, b, W_hat_f32=None, W_hat_bf16=None, st
     m = packed.shape[0]
     _check(lib().lcq_decode(_ptr(packed), m, n, d, _ptr(A), _ptr(b), _ptr(W_hat_f32), _ptr(W_hat_bf16),
                             _stream(stream)), "lcq_decode")
+
+
+def lcq_activation_transform(X, d: int, A, b, Xp=None, r=None, stream=None):
+    """X' = X_g A (bf16, into Xp) and r = sum_g X_g . b (fp32, into r) per token; either output may be None."""
+    N, n = X.shape
+    _check(lib().lcq_activation_transform(_ptr(X), N, n, d, _ptr(A), _ptr(b), _ptr(Xp), _ptr(r), _stream(stream)),
+           "lcq_activation_transform")
 
 
 def lcq_pack2b(codes, packed, stream=None):

@@ -113,6 +113,8 @@ cudaError_t launch_encode_batch(const EncodeBatchArgs &a, int d, int num_sms, cu
 cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t st);
 cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, int num_sms, cudaStream_t st);
+cudaError_t launch_xform(const uint16_t *X, int64_t N, int64_t n, int d, const float *A, const float *b, uint16_t *Xp,
+                         float *r, cudaStream_t st);
 cudaError_t launch_wait_timeout_selftest(int32_t *status, cudaStream_t st);
 cudaError_t launch_init_codebook(const float *G, int d, float *A, float *b, cudaStream_t st);
 cudaError_t launch_init_latent(const uint8_t *packed, int64_t total, float s, float t, float *P, int num_sms,

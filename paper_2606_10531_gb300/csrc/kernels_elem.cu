@@ -832,6 +832,89 @@ cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t 
     return cudaGetLastError();
 }
 
+// Activation transform (Sec. 3.2, Eq. def:forward_x): one warp per token row. A lane takes the row's
+// 8-column units lane, lane + 32, ... (one 16-byte load of bf16 each), four loads in flight before
+// their arithmetic; it forms X' = X_g A for the unit's groups and adds X_g . b into its share of r,
+// which the warp sums by a fixed butterfly.
+constexpr int kXformWarps = 8;
+
+template <int D>
+__device__ __forceinline__ void xform_unit(const uint4 v, const float (&Am)[D * D], const float (&bv)[D], uint4 &out,
+                                           float &racc) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    float x[8], y[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+#pragma unroll
+    for (int g = 0; g < 8 / D; ++g) {
+#pragma unroll
+        for (int k = 0; k < D; ++k) {
+            float acc = 0.0f;
+#pragma unroll
+            for (int j = 0; j < D; ++j) acc = fmaf(x[g * D + j], Am[j * D + k], acc);
+            y[g * D + k] = acc;
+        }
+#pragma unroll
+        for (int j = 0; j < D; ++j) racc = fmaf(x[g * D + j], bv[j], racc);
+    }
+    out = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]), pack_bf16x2(y[4], y[5]), pack_bf16x2(y[6], y[7]));
+}
+
+template <int D>
+__global__ void __launch_bounds__(32 * kXformWarps)
+xform_kernel(const uint16_t *__restrict__ X, int64_t N, int64_t n, const float *__restrict__ A,
+             const float *__restrict__ b, uint16_t *__restrict__ Xp, float *__restrict__ r) {
+    __shared__ float sA[D * D], sb[D];
+    if (threadIdx.x < D * D) sA[threadIdx.x] = __ldg(A + threadIdx.x);
+    if (threadIdx.x < D) sb[threadIdx.x] = __ldg(b + threadIdx.x);
+    __syncthreads();
+    float Am[D * D], bv[D];
+#pragma unroll
+    for (int i = 0; i < D * D; ++i) Am[i] = sA[i];
+#pragma unroll
+    for (int i = 0; i < D; ++i) bv[i] = sb[i];
+    const int lane = threadIdx.x & 31;
+    const int64_t t = static_cast<int64_t>(blockIdx.x) * kXformWarps + (threadIdx.x >> 5);
+    if (t >= N) return;
+    const uint4 *src = reinterpret_cast<const uint4 *>(X + t * n);
+    uint4 *dst = Xp ? reinterpret_cast<uint4 *>(Xp + t * n) : nullptr;
+    const int64_t units = n / 8;
+    float racc = 0.0f;
+    int64_t u = lane;
+    for (; u + 96 < units; u += 128) {
+        uint4 v[4], o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __ldg(src + u + 32 * i);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) xform_unit<D>(v[i], Am, bv, o[i], racc);
+        if (dst) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) dst[u + 32 * i] = o[i];
+        }
+    }
+    for (; u < units; u += 32) {
+        uint4 o;
+        xform_unit<D>(__ldg(src + u), Am, bv, o, racc);
+        if (dst) dst[u] = o;
+    }
+    for (int o = 16; o; o >>= 1) racc += __shfl_xor_sync(0xffffffffu, racc, o);
+    if (r && lane == 0) r[t] = racc;
+}
+
+cudaError_t launch_xform(const uint16_t *X, int64_t N, int64_t n, int d, const float *A, const float *b, uint16_t *Xp,
+                         float *r, cudaStream_t st) {
+    trace_begin(LCQ_K_XFORM, st);
+    const unsigned grid = static_cast<unsigned>((N + kXformWarps - 1) / kXformWarps);
+    if (d == 4) xform_kernel<4><<<grid, 32 * kXformWarps, 0, st>>>(X, N, n, A, b, Xp, r);
+    else xform_kernel<8><<<grid, 32 * kXformWarps, 0, st>>>(X, N, n, A, b, Xp, r);
+    trace_end(LCQ_K_XFORM, st);
+    count_launch();
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, int num_sms, cudaStream_t st) {
     const int64_t nslices = (total + 15) / 16;
     int64_t grid = (nslices + 255) / 256;

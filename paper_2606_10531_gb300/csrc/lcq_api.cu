@@ -480,6 +480,20 @@ lcq_status lcq_decode(const uint8_t *packed, int64_t m, int64_t n, int d, const 
     return cuda_status(launch_decode(a, d, num_sms_current(), as_stream(stream)));
 }
 
+lcq_status lcq_activation_transform(const uint16_t *X, int64_t N, int64_t n, int d, const float *A, const float *b,
+                                    uint16_t *Xp, float *r, void *stream) {
+    LCQ_TRY(check_common(0, n, d));
+    if (N < 0 || N > (int64_t(1) << 31) - 1) return LCQ_ERR_SHAPE;
+    if (N == 0) return LCQ_OK;
+    if (!Xp && !r) return LCQ_ERR_NULL;
+    LCQ_TRY(check_tensor(X, N * n));
+    LCQ_TRY(check_tensor(Xp, N * n, false));
+    LCQ_TRY(check_tensor(r, N, false));
+    if (!A || !b) return LCQ_ERR_NULL;
+    if (n == 0) return r ? cuda_status(cudaMemsetAsync(r, 0, sizeof(float) * N, as_stream(stream))) : LCQ_OK;
+    return cuda_status(launch_xform(X, N, n, d, A, b, Xp, r, as_stream(stream)));
+}
+
 lcq_status lcq_pack2b(const uint8_t *codes, int64_t m, int64_t n, uint8_t *packed, void *stream) {
     if (m < 0 || n < 0) return LCQ_ERR_SHAPE;
     if (n % 4 != 0) return LCQ_ERR_SHAPE;

@@ -244,3 +244,25 @@ def test_llama3_70b_layer_bulk_encode_batch_full_size():
         ref_mse = sq / (mx.m * mx.n)
         assert abs(it["mse"].item() - ref_mse) <= 1e-4 * ref_mse, mx.name
     print(f"near-boundary codes excluded: {near_total} of {sum(mx.m * mx.n for mx in mats)}")
+
+
+@pytest.mark.parametrize("index", [0, 6])
+def test_llama3_8b_activation_transform_full_size(index):
+    """The activation transform of the reformulated forward (Eq. def:forward_x) at the training shapes
+    of the Llama-3-8B layer (16384 tokens; n = 4096 for q, n = 14336 for down): sampled tokens against
+    the oracle in fp64, within the bf16 rounding of X' and the fp32 sum bound of r."""
+    import torch
+    from tests.test_gpu_parity import _xform_bounds
+    mx = wl.llama3_8b_layer()[index]
+    Xb = wl.draw_X(mx, SEED, index)
+    A, b = wl.draw_A(mx, SEED, index), wl.draw_b(mx, SEED, index)
+    Xp = empty_bf16(mx.N, mx.n)
+    r = torch.empty(mx.N, dtype=torch.float32, device="cuda")
+    lcq.lcq_activation_transform(dev_bf16(Xb), mx.d, dev(A), dev(b), Xp=Xp, r=r)
+    toks = np.random.default_rng(7 + index).choice(mx.N, SAMPLES, replace=False)
+    Xf = wl.bf16_to_f32(Xb[toks])
+    ref_p, ref_r = oracle.activation_transform(Xf, A, b, mx.d)
+    bp, br = _xform_bounds(Xf, ref_p, A, b, mx.d)
+    got_p = host_bf16(Xp[torch.as_tensor(toks, device="cuda")])
+    assert np.all(np.abs(got_p - ref_p) <= bp)
+    assert np.all(np.abs(r.cpu().numpy()[toks].astype(np.float64) - ref_r) <= br)

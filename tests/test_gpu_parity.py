@@ -533,3 +533,57 @@ def test_gemm_packed2b_tcgen05_zero_token_and_repeat():
     assert torch.equal(Y1, Y2)
     assert float(Y1[3].float().abs().max()) == 0.0
     assert max_rel(host_bf16(Y1), ref) <= TOL_DP
+
+
+# ----------------------------------------------------------------------------- activation transform
+
+def _xform_bounds(Xf, ref_p, A, b, d):
+    """Elementwise error bounds of the transform against fp64: X' is an fp32 sum of d products (error
+    at most gamma_d sum |x a|) rounded to bf16 (8 significant bits: half an ulp is at most 2^-8 of the
+    value); r is an fp32 sum of n products, bounded by gamma_n-sized multiples of sum |x b|
+    (u = 2^-24)."""
+    N, n = Xf.shape
+    u = 2.0 ** -24
+    Xg = np.abs(Xf.astype(np.float64)).reshape(N, n // d, d)
+    absxa = (Xg @ np.abs(A.astype(np.float64))).reshape(N, n)
+    absxb = (Xg @ np.abs(b.astype(np.float64))).sum(axis=1)
+    sum_err = 2 * d * u * absxa
+    return 2.0 ** -8 * (np.abs(ref_p) + sum_err) + sum_err, 2 * (n + 8) * u * absxb
+
+
+@pytest.mark.parametrize("d", [4, 8])
+@pytest.mark.parametrize("N,n", [(64, 512), (3, 200), (33, 4104), (1, 8)])
+def test_activation_transform_matches_oracle(N, n, d):
+    torch = T()
+    if n % d:
+        pytest.skip("n % d")
+    rng = np.random.default_rng(N + n + d)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n))
+    X[:, rng.random(n) < 0.01] *= 50.0
+    Xb = wl.bf16_bits(X.astype(np.float32))
+    Xf = wl.bf16_to_f32(Xb)
+    ref_p, ref_r = oracle.activation_transform(Xf, A, b, d)
+    Xp = empty_bf16(N, n)
+    r = torch.empty(N, dtype=torch.float32, device="cuda")
+    lcq.lcq_activation_transform(dev_bf16(Xb), d, dev(A), dev(b), Xp=Xp, r=r)
+    bp, br = _xform_bounds(Xf, ref_p, A, b, d)
+    assert np.all(np.abs(host_bf16(Xp) - ref_p) <= bp)
+    assert np.all(np.abs(r.cpu().numpy().astype(np.float64) - ref_r) <= br)
+
+
+def test_activation_transform_single_output_and_empty():
+    torch = T()
+    rng = np.random.default_rng(3)
+    d, N, n = 8, 5, 64
+    A, b = config_A(d, rng), config_b(d, rng)
+    Xb = wl.bf16_bits(rng.normal(0, 1, (N, n)).astype(np.float32))
+    r = torch.full((N,), 7.0, dtype=torch.float32, device="cuda")
+    lcq.lcq_activation_transform(dev_bf16(Xb), d, dev(A), dev(b), r=r)      # X' not written (NULL)
+    ref_p, ref_r = oracle.activation_transform(wl.bf16_to_f32(Xb), A, b, d)
+    np.testing.assert_allclose(r.cpu().numpy(), ref_r, rtol=1e-5, atol=1e-7)
+    Xp = empty_bf16(N, n)
+    lcq.lcq_activation_transform(dev_bf16(Xb), d, dev(A), dev(b), Xp=Xp)     # r not written (NULL)
+    assert max_rel(host_bf16(Xp), ref_p) <= 4e-3
+    E = torch.empty((0, n), dtype=torch.bfloat16, device="cuda")
+    lcq.lcq_activation_transform(E, d, dev(A), dev(b), r=torch.empty(0, device="cuda"))

@@ -203,6 +203,40 @@ def test_forward_equals_reformulated_sum(d):
     np.testing.assert_allclose(oracle.linear_fwd(X, Z, A, b, d), Y, rtol=1e-12, atol=1e-15)
 
 
+@pytest.mark.parametrize("d", [4, 8])
+def test_activation_transform_reproduces_the_decoded_product(d):
+    """X' Z^T + r 1^T equals X W_hat^T computed through decode (Eq. def:forward vs def:forward_x): a
+    transposed A, a dropped bias term or a wrong group stride breaks the identity."""
+    N, m, n = 5, 7, 4 * d
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    Z = RNG.integers(0, 4, (m, n))
+    X = RNG.normal(size=(N, n))
+    Xp, r = oracle.activation_transform(X, A, b, d)
+    np.testing.assert_allclose(Xp @ Z.T + r[:, None], oracle.linear_fwd(X, Z, A, b, d), rtol=1e-12, atol=1e-12)
+
+
+def test_activation_transform_special_cases():
+    """A = I, b = 0 leaves X unchanged with r = 0; a one-hot token e_c (c = g d + j) gives row j of A in
+    group g and r = b_j; r is X times b repeated over the groups."""
+    d, N, n = 4, 3, 12
+    X = RNG.normal(size=(N, n))
+    Xp, r = oracle.activation_transform(X, np.eye(d), np.zeros(d), d)
+    np.testing.assert_array_equal(Xp, X)
+    np.testing.assert_array_equal(r, np.zeros(N))
+    A, b = RNG.normal(size=(d, d)), RNG.normal(size=d)
+    for c in (0, 5, 11):
+        e = np.zeros((1, n))
+        e[0, c] = 1.0
+        Xp, r = oracle.activation_transform(e, A, b, d)
+        g, j = divmod(c, d)
+        expect = np.zeros(n)
+        expect[g * d:(g + 1) * d] = A[j]
+        np.testing.assert_allclose(Xp[0], expect, atol=0)
+        assert r[0] == b[j]
+    Xp, r = oracle.activation_transform(X, A, b, d)
+    np.testing.assert_allclose(r, X @ np.tile(b, n // d), rtol=1e-13)
+
+
 def test_packed_product_equals_unpacked_product():
     d, m, n = 8, 6, 32
     A, b = config_like_A(d, RNG), RNG.normal(0, 1e-3, d)
