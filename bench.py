@@ -46,11 +46,12 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the separate encode / packed-product timings")
-    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq"], default=None,
+    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq", "xform"], default=None,
                     help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
                          "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
                          "28672 x 8192, gemv = 70B gate at --tokens tokens, ldlq = LDLQ sweep of a "
-                         "9728 x 4096 slice of the 8B gate (one wave, small case)")
+                         "9728 x 4096 slice of the 8B gate (one wave, small case), xform = activation "
+                         "transform of the q projection's 16384 x 4096 activations")
     ap.add_argument("--tokens", type=int, default=None, help="tokens of the gemv profiling case (default 16)")
     return ap.parse_args()
 
@@ -765,6 +766,15 @@ def profile_case(args):
         def run():
             lcq.lcq_ldlq(W, A, b, U, d, ws, packed=pk_)
         wss = [wsf, ws]
+    elif args.case == "xform":
+        mx = wl.llama3_8b_layer()[0]
+        X = wl.torch_X(torch, mx, args.seed, 0, device)
+        A, b = wl.torch_A(torch, mx, args.seed, 0, device).contiguous(), wl.torch_b(torch, mx, args.seed, 0, device)
+        Xp, r = torch.empty_like(X), torch.empty(mx.N, dtype=torch.float32, device=device)
+
+        def run():
+            lcq.lcq_activation_transform(X, mx.d, A, b, Xp=Xp, r=r)
+        wss = []
     else:
         mx = wl.llama3_70b_gate_decode(args.tokens or GEMV_TOKENS)[0]
         packed = wl.torch_packed_codes(torch, mx, args.seed, 0, device)
