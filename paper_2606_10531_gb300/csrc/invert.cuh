@@ -1,7 +1,7 @@
 // A^{-1} of a small (d x d, d <= 8) matrix by one warp, to fp32 accuracy: register Gauss-Jordan
 // elimination in fp32, refined by Newton steps whose residual is accumulated in double-float, with
 // an fp64 elimination as the fallback for badly conditioned input. Used by the encoders (A^{-1} of
-// the codebook map) and by the block factorisation of LDLQ (inverses of its diagonal blocks).
+// the codebook map) and by the LDLQ sweep.
 //
 // The scratch type Smem must provide: float A[64] (input, row-major d x d), float Ainv[64] (output),
 // float M[64] (output: A^T A), double gj[8][16], float gjf[8][16] (work), int singular (output).
@@ -84,64 +84,6 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &err) 
     err = (a - (s - bb)) + (b - bb);
 }
 
-// One thread: X = A^{-1} of a symmetric positive definite A (row-major in smem) by Cholesky, A = L L^T,
-// X = L^{-T} L^{-1}, all in registers (fp32; the caller refines). Returns false if a pivot is not
-// (relatively) positive.
-template <int D>
-__device__ __forceinline__ bool spd_inverse_thread(const float *A, float (&X)[8][16], float amax) {
-    float L[D][D];
-#pragma unroll
-    for (int i = 0; i < D; ++i)
-#pragma unroll
-        for (int j = 0; j < D; ++j) L[i][j] = 0.0f;
-    float dinv[D];
-    bool ok = true;
-#pragma unroll
-    for (int j = 0; j < D; ++j) {
-        float dj = A[j * D + j];
-#pragma unroll
-        for (int k = 0; k < j; ++k) dj = fmaf(-L[j][k], L[j][k], dj);
-        ok = ok && (dj > 1e-12f * amax) && isfinite(dj);
-        const float ljj = sqrtf(fmaxf(dj, 1e-30f));
-        L[j][j] = ljj;
-        dinv[j] = 1.0f / ljj;
-#pragma unroll
-        for (int i = j + 1; i < D; ++i) {
-            float v = A[i * D + j];
-#pragma unroll
-            for (int k = 0; k < j; ++k) v = fmaf(-L[i][k], L[j][k], v);
-            L[i][j] = v * dinv[j];
-        }
-    }
-    // W = L^{-1} (lower triangular), column by column
-    float W[D][D];
-#pragma unroll
-    for (int j = 0; j < D; ++j) {
-#pragma unroll
-        for (int i = 0; i < D; ++i) W[i][j] = 0.0f;
-        W[j][j] = dinv[j];
-#pragma unroll
-        for (int i = j + 1; i < D; ++i) {
-            float v = 0.0f;
-#pragma unroll
-            for (int k = j; k < i; ++k) v = fmaf(L[i][k], W[k][j], v);
-            W[i][j] = -v * dinv[i];
-        }
-    }
-    // X = W^T W (symmetric)
-#pragma unroll
-    for (int i = 0; i < D; ++i)
-#pragma unroll
-        for (int j = i; j < D; ++j) {
-            float v = 0.0f;
-#pragma unroll
-            for (int k = j; k < D; ++k) v = fmaf(W[k][i], W[k][j], v);
-            X[i][j] = v;
-            X[j][i] = v;
-        }
-    return ok;
-}
-
 // One warp: A^{-1} and M = A^T A (fp32).
 //  1. Gauss-Jordan elimination with partial pivoting in fp32, in registers: lane r + D h (r < D,
 //     h < 2D/8) holds columns 8h .. 8h+7 of row r of [A | I]; pivots, row swaps and the pivot row
@@ -152,10 +94,7 @@ __device__ __forceinline__ bool spd_inverse_thread(const float *A, float (&X)[8]
 //  3. If the residual does not reach the acceptance bound within four steps (A badly conditioned, or
 //     non-finite), the fp64 elimination runs instead.
 // Sets s.singular if a pivot is (relatively) zero.
-// kSpd: A is symmetric positive definite (the diagonal blocks of LDLQ's factorisation): the first
-// approximation is lane 0's Cholesky-based inverse (spd_inverse_thread) instead of the elimination,
-// and M is not formed; the refinement and its fp64 fallback are the same.
-template <int D, typename Smem, bool kSpd = false>
+template <int D, typename Smem>
 __device__ void invert_warp(Smem &s) {
     constexpr int H = 2 * D / 8;                 // 8-column blocks of [A | I]
     const int lane = threadIdx.x & 31;
@@ -167,13 +106,11 @@ __device__ void invert_warp(Smem &s) {
         const int c = 8 * h + j;
         row[j] = !act ? 0.0f : (c < D ? s.A[r * D + c] : (c - D == r ? 1.0f : 0.0f));
     }
-    if (!kSpd) {
-        for (int e = lane; e < D * D; e += 32) {
-            const int i = e / D, j = e % D;
-            float acc = 0.0f;
-            for (int k = 0; k < D; ++k) acc = fmaf(s.A[k * D + i], s.A[k * D + j], acc);
-            s.M[e] = acc;
-        }
+    for (int e = lane; e < D * D; e += 32) {
+        const int i = e / D, j = e % D;
+        float acc = 0.0f;
+        for (int k = 0; k < D; ++k) acc = fmaf(s.A[k * D + i], s.A[k * D + j], acc);
+        s.M[e] = acc;
     }
     float amax = 0.0f;
 #pragma unroll
@@ -181,38 +118,24 @@ __device__ void invert_warp(Smem &s) {
         if (8 * h + j < D) amax = fmaxf(amax, fabsf(row[j]));
     for (int o = 16; o; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
     int singular = !(amax > 0.0f) || !isfinite(amax);
-    if (kSpd) {
-        if (!singular) {
-            int bad = 0;
-            if (lane == 0) bad = spd_inverse_thread<D>(s.A, s.gjf, amax) ? 0 : 1;
-            singular = __shfl_sync(0xffffffffu, bad, 0);
-        }
-    }
 #pragma unroll
     for (int c = 0; c < D; ++c) {
-        if (singular || kSpd) break;
-        float piv;
-        if (kSpd) {
-            // the diagonal pivot (positive for a positive definite A)
-            piv = __shfl_sync(0xffffffffu, row[c], c);
-            if (!(static_cast<double>(piv) > 1e-12 * static_cast<double>(amax)) || !isfinite(piv)) { singular = 1; break; }
-        } else {
-            // pivot: largest |a[r][c]| over rows r >= c (column c sits in block 0, lane r)
-            float v = (act && h == 0 && r >= c) ? fabsf(row[c]) : -1.0f;
-            int idx = r;
-            for (int o = 16; o; o >>= 1) {
-                const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-                if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
-            }
-            if (!(static_cast<double>(v) > 1e-12 * static_cast<double>(amax)) || !isfinite(v)) { singular = 1; break; }
-            const int prow = idx;
-            // swap rows c and prow, within each column block
-            const int src = (r == c) ? prow : (r == prow ? c : r);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src + D * h);
-            piv = __shfl_sync(0xffffffffu, row[c], c);     // a[c][c], block 0
+        if (singular) break;
+        // pivot: largest |a[r][c]| over rows r >= c (column c sits in block 0, lane r)
+        float v = (act && h == 0 && r >= c) ? fabsf(row[c]) : -1.0f;
+        int idx = r;
+        for (int o = 16; o; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+            if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
         }
+        if (!(static_cast<double>(v) > 1e-12 * static_cast<double>(amax)) || !isfinite(v)) { singular = 1; break; }
+        const int prow = idx;
+        // swap rows c and prow, within each column block
+        const int src = (r == c) ? prow : (r == prow ? c : r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src + D * h);
+        const float piv = __shfl_sync(0xffffffffu, row[c], c);     // a[c][c], block 0
         const float rinv = 1.0f / piv;
         if (r == c) {
 #pragma unroll
@@ -231,13 +154,11 @@ __device__ void invert_warp(Smem &s) {
         __syncwarp();
         return;
     }
-    // X = right half of [I | A^{-1}] (kSpd: lane 0 has written it)
-    if (!kSpd) {
+    // X = right half of [I | A^{-1}]
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int c = 8 * h + j;
-            if (act && c >= D) s.gjf[r][c - D] = row[j];
-        }
+    for (int j = 0; j < 8; ++j) {
+        const int c = 8 * h + j;
+        if (act && c >= D) s.gjf[r][c - D] = row[j];
     }
     __syncwarp();
     // Acceptance: the residual of any fp32-stored inverse has a rounding floor of about

@@ -5,11 +5,12 @@
 //     H = (U + I) D (U + I)^T,   T_k = W_k + sum_{j<k} (W_j - W_hat_j) U_{j,k},
 //     z_k = clip(round(A^{-1}(T_k - b)), 0, 3),   W_hat_k = A z_k + b.
 //
-// Factorisation (ldl_panel_kernel, ldl_gemm_nt_kernel): right-looking over 128-column panels from
-// the last to the first. A panel's diagonal block is factored by one CTA in shared memory; the
-// column block above it and the Schur-complement update of the leading matrix are fp32 SIMT GEMMs
-// (Y = S_QP M^-T, U_QP = S_QP M^-T D^-1, S_QQ -= Y U_QP^T; upper triangle only, the panel kernel
-// mirrors it).
+// Factorisation (ldl_panel_kernel, ldl_gemm_k128_kernel, ldl_syrk_kernel): H = R R^T with R upper
+// triangular (a Cholesky factorisation in reverse index order), from which D_k = R_kk R_kk^T and
+// U = R Rd^-1 - I (Rd = the block diagonal of R). Right-looking over 128-column panels from the last
+// to the first: one CTA factors a panel's diagonal block in shared memory and forms W = R_PP^-1; the
+// column block above it, Z = S_QP W^T (with U_QP = Z Rd^-1 in the same kernel), and the Schur update
+// S_QQ -= Z Z^T (upper triangle only) are fp32 SIMT GEMMs.
 //
 // Sweep (ldlq_sweep_kernel): rows are independent, so one CTA takes 64 rows through every column
 // chunk of 128 columns. For chunk c it first forms the feedback of all earlier columns as a GEMM,
@@ -32,169 +33,466 @@ namespace lcq {
 
 constexpr int kLdlPanel = 128;        // panel width (columns), a multiple of 8
 constexpr int kLdlThreads = 256;
-constexpr int kLdlLd = kLdlPanel + 1;
+constexpr int kLdlLd = kLdlPanel + 4; // rows 16-byte aligned, consecutive rows 4 banks apart
+constexpr int kLdlRinvLd = 72;        // floats between the groups of R_kk^-1 (8 banks apart)
+constexpr int kLdlBarColumns = 1;     // named barrier: the column block of R is complete
 
+// The panel's diagonal block is factored as S = R R^T with R upper triangular (a Cholesky factorisation
+// in reverse index order, group by group). The block factor follows from it without d x d inversions:
+// D_k = R_kk R_kk^T and U = R Rd^-1 - I (Rd = block diagonal of R). The panel hands W = R^-1 and the
+// R_kk^-1 to the trailing update: Z = S_QP W^T is the factor's column block above the panel,
+// U_QP = Z Rd^-1 and the Schur update is S_QQ -= Z Z^T.
 struct LdlPanelSmem {
-    float S[kLdlPanel][kLdlLd];       // Schur block of the panel (symmetrised); later M^-1
-    float Up[kLdlPanel][kLdlLd];      // U of the panel (strictly upper d x d blocks)
-    float Dinv[kLdlPanel / 4][64];    // D_k^{-1} per group
-    InvScratch inv;
+    float S[kLdlPanel][kLdlLd];       // Schur block (block-upper part current); row block k becomes W's once consumed
+    float R[kLdlPanel][kLdlLd];       // R's column blocks above the diagonal blocks, as they are formed
+    float RT[8][kLdlPanel];           // the current column block of R, transposed
+    float Rinv[kLdlPanel / 4][kLdlRinvLd];   // R_kk^-1 per group (D x D row-major, upper triangular)
 };
 
-// Factor the diagonal block S[c0:c0+P, c0:c0+P] (upper triangle read, mirrored) of the current
-// Schur complement: U and D of the panel's groups, eliminated from the last group to the first; then
-// M^-1 = (I + U_PP)^-1 by block back substitution, and D^-1 M^-1. Writes U's panel block, D (if
-// requested), Minv and Binv (P x P, leading dimension kLdlPanel).
+__device__ __forceinline__ void ldl_named_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+__device__ __forceinline__ void ldl_named_arrive(int id, int count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// One warp: S_kk = R_kk R_kk^T (upper triangle of S_kk read) and R_kk^-1. Every lane factors the block
+// in registers (pivots from the last index to the first); lane j then forms column j of R_kk^-1. A pivot
+// that is not positive relative to the block's largest entry (or a non-finite block) sets
+// LCQ_ERR_SINGULAR and leaves R_kk^-1 zero.
 template <int D>
-__global__ void __launch_bounds__(kLdlThreads)
-ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, float *__restrict__ U,
-                 float *__restrict__ Dout, float *__restrict__ Minv, float *__restrict__ Binv, int32_t *status) {
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    LdlPanelSmem &s = *reinterpret_cast<LdlPanelSmem *>(smem_raw);
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int G = P / D;
-    for (int e = tid; e < P * P; e += kLdlThreads) {
-        const int i = e / P, j = e % P;
-        const int64_t lo = i <= j ? i : j, hi = i <= j ? j : i;
-        s.S[i][j] = S[(c0 + lo) * n + c0 + hi];
-        s.Up[i][j] = 0.0f;
-    }
-    __syncthreads();
-    // D_k^{-1} of the last group; then per group k (from the last): U_{<k,k} = S_{<k,k} D_k^{-1}, the
-    // next diagonal block D_{k-1} updated first, and its inversion (warp 0) overlapped with the rest of
-    // the Schur update S_{<k,<k} -= U_{<k,k} S_{k,<k} (warps 1..). Only the block-upper triangle is
-    // kept current (S_{k,<k} is read as S_{<k,k}^T).
-    const auto invert_group = [&](int k) {
-        const int kd = k * D;
-        for (int e = tid; e < D * D; e += 32) s.inv.A[e] = s.S[kd + e / D][kd + e % D];
-        __syncwarp();
-        invert_warp<D, InvScratch, true>(s.inv);
-        for (int e = tid; e < D * D; e += 32) {
-            s.Dinv[k][e] = s.inv.Ainv[e];
-            if (Dout) Dout[(c0 / D + k) * D * D + e] = s.inv.A[e];
-        }
-        if (tid == 0 && s.inv.singular) set_status(status, LCQ_ERR_SINGULAR);
-    };
-    if (warp == 0) invert_group(G - 1);
-    __syncthreads();
-    for (int k = G - 1; k >= 1; --k) {
-        const int kd = k * D, kp = kd - D;
-        // U_{<k,k} = S_{<k,k} D_k^{-1}
-        for (int e = tid; e < kd * D; e += kLdlThreads) {
+__device__ void ldl_factor_group(LdlPanelSmem &s, int k, float *Dk, int32_t *status) {
+    const int lane = threadIdx.x & 31, kd = k * D;
+    if (Dk) {
+        for (int e = lane; e < D * D; e += 32) {
             const int i = e / D, j = e % D;
-            float acc = 0.0f;
-#pragma unroll
-            for (int q = 0; q < D; ++q) acc = fmaf(s.S[i][kd + q], s.Dinv[k][q * D + j], acc);
-            s.Up[i][kd + j] = acc;
+            Dk[e] = i <= j ? s.S[kd + i][kd + j] : s.S[kd + j][kd + i];
         }
-        __syncthreads();
-        // the next diagonal block, D_{k-1} -= U_{k-1,k} S_{k,k-1}
-        for (int e = tid; e < D * D; e += kLdlThreads) {
-            const int i = kp + e / D, j = kp + e % D;
-            float acc = s.S[i][j];
-#pragma unroll
-            for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[j][kd + q], acc);
-            s.S[i][j] = acc;
-        }
-        __syncthreads();
-        if (warp == 0) {
-            invert_group(k - 1);
-        } else {
-            // the rest of the block-upper triangle of S_{<k,<k}
-            for (int e = tid - 32; e < kd * kd; e += kLdlThreads - 32) {
-                const int i = e / kd, j = e % kd;
-                const int bi = i / D, bj = j / D;
-                if (bi > bj || (bi == k - 1 && bj == k - 1)) continue;
-                float acc = s.S[i][j];
-#pragma unroll
-                for (int q = 0; q < D; ++q) acc = fmaf(-s.Up[i][kd + q], s.S[j][kd + q], acc);
-                s.S[i][j] = acc;
-            }
-        }
-        __syncthreads();
     }
-    // U's panel block (the zero blocks stay as the caller cleared them)
-    for (int e = tid; e < P * P; e += kLdlThreads) {
-        const int i = e / P, j = e % P;
-        if (i / D < j / D) U[(c0 + i) * n + c0 + j] = s.Up[i][j];
-    }
-    // X = M^-1, M = I + Up unit block-upper triangular: X_k = E_k - sum_{j>k} Up_{k,j} X_j, block rows
-    // from the last; X is block-upper triangular too, so X_k[., col] needs the blocks up to col's only
-    for (int k = G - 1; k >= 0; --k) {
-        const int kd = k * D;
-        for (int e = tid; e < D * P; e += kLdlThreads) {
-            const int r = kd + e / P, col = e % P;
-            float acc;
-            if (col < kd + D) {
-                acc = (r == col) ? 1.0f : 0.0f;
-            } else {
-                // four partial sums (the block boundaries are multiples of D >= 4)
-                float a4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                const int cend = (col / D + 1) * D;
-                for (int c = kd + D; c < cend; c += 4)
+    float a[D][D];                                 // upper triangle
+    float amax = 0.0f;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) a4[q] = fmaf(-s.Up[r][c + q], s.S[c + q][col], a4[q]);
-                acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
-            }
-            s.S[r][col] = acc;
+    for (int i = 0; i < D; ++i)
+#pragma unroll
+        for (int j = i; j < D; ++j) {
+            a[i][j] = s.S[kd + i][kd + j];
+            amax = fmaxf(amax, fabsf(a[i][j]));
         }
-        __syncthreads();
+    bool ok = amax > 0.0f && isfinite(amax);
+    float ip[D];                                   // 1 / R_pp
+#pragma unroll
+    for (int p = D - 1; p >= 0; --p) {
+        const float piv = a[p][p];
+        ok = ok && piv > 1e-12f * amax;
+        ip[p] = rsqrtf(fmaxf(piv, 1e-30f));
+#pragma unroll
+        for (int i = 0; i <= p; ++i) a[i][p] *= ip[p];          // column p of R
+#pragma unroll
+        for (int i = 0; i < p; ++i)
+#pragma unroll
+            for (int j = i; j < p; ++j) a[i][j] = fmaf(-a[i][p], a[j][p], a[i][j]);
     }
-    for (int e = tid; e < P * P; e += kLdlThreads) {
-        const int i = e / P, j = e % P;
-        Minv[i * kLdlPanel + j] = s.S[i][j];
-        const int k = i / D, r = i % D;
+    // column `lane` of R_kk^-1 by back substitution
+    float x[D];
+#pragma unroll
+    for (int q = 0; q < D; ++q) x[q] = q == lane ? ip[q] : 0.0f;
+#pragma unroll
+    for (int r = D - 2; r >= 0; --r) {
         float acc = 0.0f;
 #pragma unroll
-        for (int q = 0; q < D; ++q) acc = fmaf(s.Dinv[k][r * D + q], s.S[k * D + q][j], acc);
-        Binv[i * kLdlPanel + j] = acc;
+        for (int l = r + 1; l < D; ++l) acc = fmaf(a[r][l], x[l], acc);
+        if (r < lane) x[r] = -acc * ip[r];
+    }
+    if (lane < D) {
+#pragma unroll
+        for (int r = 0; r < D; ++r) s.Rinv[k][r * D + lane] = ok ? x[r] : 0.0f;
+    }
+    if (lane == 0 && !ok) set_status(status, LCQ_ERR_SINGULAR);
+    __syncwarp();
+}
+
+// Row i of the column block k of R: R_{i,k} = S_{i,k} R_kk^-T, outputs 4h .. 4h+3 (into R and RT).
+template <int D>
+__device__ __forceinline__ void ldl_column_quad(LdlPanelSmem &s, int k, int i, int h) {
+    const int kd = k * D;
+    float sv[D];
+#pragma unroll
+    for (int q = 0; q < D; q += 4) {
+        const float4 v = *reinterpret_cast<const float4 *>(&s.S[i][kd + q]);
+        sv[q] = v.x; sv[q + 1] = v.y; sv[q + 2] = v.z; sv[q + 3] = v.w;
+    }
+    float o[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        const float *rr = &s.Rinv[k][(4 * h + t) * D];     // row 4h+t of R_kk^-1 (zero below the diagonal)
+        float acc = 0.0f;
+#pragma unroll
+        for (int q = 0; q < D; q += 4) {
+            const float4 r4 = *reinterpret_cast<const float4 *>(rr + q);
+            acc = fmaf(sv[q], r4.x, acc);
+            acc = fmaf(sv[q + 1], r4.y, acc);
+            acc = fmaf(sv[q + 2], r4.z, acc);
+            acc = fmaf(sv[q + 3], r4.w, acc);
+        }
+        o[t] = acc;
+    }
+    *reinterpret_cast<float4 *>(&s.R[i][kd + 4 * h]) = make_float4(o[0], o[1], o[2], o[3]);
+#pragma unroll
+    for (int t = 0; t < 4; ++t) s.RT[4 * h + t][i] = o[t];
+}
+
+// Row block k of W = R^-1 (into S's row block k, whose Schur entries are consumed): W_kk = R_kk^-1 and
+// W_{k,j} = -R_kk^-1 sum_{k<l<=j} R_{k,l} W_{l,j}; needs W's row blocks after k. Threads t < nthr in
+// pairs: a pair takes one column, each summing every other 4-row chunk of it.
+template <int D>
+__device__ __forceinline__ void ldl_w_row_block(LdlPanelSmem &s, int k, int P, int t, int nthr) {
+    const int kd = k * D;
+    for (int e = t; e < D * D; e += nthr) s.S[kd + e / D][kd + e % D] = s.Rinv[k][e];
+    const int items = 2 * (P - kd - D);
+    for (int base = 0; base < items; base += nthr) {           // uniform trip count: the pair exchange below
+        const int e = base + t;
+        const int half = e & 1, col = kd + D + (e >> 1);
+        const int cend = e < items ? (col / D + 1) * D : kd + D;
+        float T[D];
+#pragma unroll
+        for (int q = 0; q < D; ++q) T[q] = 0.0f;
+        for (int cs = kd + D + 4 * half; cs < cend; cs += 8) {
+            const float w0 = s.S[cs][col], w1 = s.S[cs + 1][col], w2 = s.S[cs + 2][col], w3 = s.S[cs + 3][col];
+#pragma unroll
+            for (int q = 0; q < D; ++q) {
+                const float4 rv = *reinterpret_cast<const float4 *>(&s.R[kd + q][cs]);
+                T[q] = fmaf(rv.x, w0, fmaf(rv.y, w1, fmaf(rv.z, w2, fmaf(rv.w, w3, T[q]))));
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < D; ++q) T[q] += __shfl_xor_sync(0xffffffffu, T[q], 1);
+        if (e < items) {
+#pragma unroll
+            for (int rr = 0; rr < D / 2; ++rr) {
+                const int r = half * (D / 2) + rr;
+                float acc = 0.0f;
+#pragma unroll
+                for (int q = 0; q < D; ++q) acc = fmaf(s.Rinv[k][r * D + q], T[q], acc);
+                s.S[kd + r][col] = -acc;
+            }
+        }
     }
 }
 
-// C[i][j] = beta C[i][j] + alpha sum_k A[i][k] B[j][k] for i < M, j < N (K a multiple of 16; rows
-// of A and B 16-byte aligned). upper: skip the 64 x 64 tiles that lie wholly below the diagonal.
-constexpr int kGemmTile = 64, kGemmK = 16, kGemmPad = 68;
-
-__global__ void __launch_bounds__(256)
-ldl_gemm_nt_kernel(const float *__restrict__ Am, int64_t lda, const float *__restrict__ Bm, int64_t ldb,
-                   float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int K, float alpha, float beta,
-                   int upper) {
-    const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kGemmTile, j0 = static_cast<int64_t>(blockIdx.x) * kGemmTile;
-    if (upper && i0 > j0 + kGemmTile - 1) return;
-    __shared__ __align__(16) float As[kGemmK][kGemmPad];
-    __shared__ __align__(16) float Bs[kGemmK][kGemmPad];
-    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
-    const int lr = tid >> 2, lk = (tid & 3) * 4;
-    float acc[4][4] = {};
-    for (int k0 = 0; k0 < K; k0 += kGemmK) {
-        float4 va = make_float4(0.f, 0.f, 0.f, 0.f), vb = va;
-        if (i0 + lr < M) va = *reinterpret_cast<const float4 *>(Am + (i0 + lr) * lda + k0 + lk);
-        if (j0 + lr < N) vb = *reinterpret_cast<const float4 *>(Bm + (j0 + lr) * ldb + k0 + lk);
-        As[lk + 0][lr] = va.x; As[lk + 1][lr] = va.y; As[lk + 2][lr] = va.z; As[lk + 3][lr] = va.w;
-        Bs[lk + 0][lr] = vb.x; Bs[lk + 1][lr] = vb.y; Bs[lk + 2][lr] = vb.z; Bs[lk + 3][lr] = vb.w;
-        __syncthreads();
+// Factor the diagonal block S[c0:c0+P, c0:c0+P] (upper triangle read) of the current Schur complement.
+// Writes U's panel block, D (if requested), W = R^-1 (P x P, leading dimension kLdlPanel, zero below
+// the diagonal) and the R_kk^-1 (P/D blocks of D x D).
+// Iteration k (from G down to 1; G = P / D): with the column block R_{<k,k} = S_{<k,k} R_kk^-T formed,
+// warp 0 updates the next diagonal block S_{k-1,k-1} -= R_{k-1,k} R_{k-1,k}^T and factors it, while
+// warps 1.. apply the rest of the Schur update S_{<k,<k} -= R_{<k,k} R_{<k,k}^T (block-upper part, one
+// D x D block per thread), write U_{<k,k} = R_{<k,k} R_kk^-1 and form W's row block k.
+template <int D>
+__global__ void __launch_bounds__(kLdlThreads)
+ldl_panel_kernel(const float *__restrict__ S, int64_t n, int64_t c0, int P, float *__restrict__ U,
+                 float *__restrict__ Dout, float *__restrict__ Wout, float *__restrict__ RinvOut, int32_t *status) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    LdlPanelSmem &s = *reinterpret_cast<LdlPanelSmem *>(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = P / D, P4 = P / 4;
+    constexpr int NQ = D / 4;                      // output quads per row of a column block
+    constexpr int kWork = kLdlThreads - 32;        // threads of warps 1..
+    // the block-upper part of S in 16-byte chunks, eight loads in flight per thread
+    {
+        constexpr int kBatch = 8;
+        const int total = P * P4;
+        for (int e0 = tid; e0 < total; e0 += kLdlThreads * kBatch) {
+            float4 v[kBatch];
 #pragma unroll
-        for (int kk = 0; kk < kGemmK; ++kk) {
-            const float4 a = *reinterpret_cast<const float4 *>(&As[kk][ty * 4]);
-            const float4 b = *reinterpret_cast<const float4 *>(&Bs[kk][tx * 4]);
-            const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+            for (int u = 0; u < kBatch; ++u) {
+                const int e = e0 + u * kLdlThreads;
+                const int i = e / P4, j = (e % P4) * 4;
+                v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (e < total && j / D >= i / D)
+                    v[u] = __ldg(reinterpret_cast<const float4 *>(S + (c0 + i) * n + c0 + j));
+            }
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+            for (int u = 0; u < kBatch; ++u) {
+                const int e = e0 + u * kLdlThreads;
+                const int i = e / P4, j = (e % P4) * 4;
+                if (e < total && j / D >= i / D) *reinterpret_cast<float4 *>(&s.S[i][j]) = v[u];
+            }
+        }
+    }
+    __syncthreads();
+    for (int k = G; k >= 1; --k) {
+        const int kd = k * D, kp = kd - D;
+        const bool cols = k < G;                   // the column block k exists (R_kk known)
+        if (warp == 0) {
+            if (cols) {
+                if (lane < D * NQ) ldl_column_quad<D>(s, k, kp + lane / NQ, lane % NQ);
+                __syncwarp();
+                ldl_named_arrive(kLdlBarColumns, kLdlThreads);
+                for (int e = lane; e < D * D; e += 32) {
+                    const int r = e / D, c = e % D;
+                    float acc = s.S[kp + r][kp + c];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                    for (int q = 0; q < D; ++q) acc = fmaf(-s.RT[q][kp + r], s.RT[q][kp + c], acc);
+                    s.S[kp + r][kp + c] = acc;
+                }
+                __syncwarp();
+            }
+            ldl_factor_group<D>(s, k - 1, Dout ? Dout + (c0 / D + k - 1) * D * D : nullptr, status);
+        } else if (cols) {
+            const int t = tid - 32;
+            for (int e = t; e < kp * NQ; e += kWork) ldl_column_quad<D>(s, k, e / NQ, e % NQ);
+            ldl_named_sync(kLdlBarColumns, kLdlThreads);
+            // Schur update: blocks (gi, gj), gi <= gj < k, in row-major order, all but the last, (k-1, k-1)
+            const int nblk = k * (k + 1) / 2 - 1;
+            for (int e = t; e < nblk; e += kWork) {
+                int gi = 0, rem = e;
+                while (rem >= k - gi) { rem -= k - gi; ++gi; }
+                const int gj = gi + rem;
+                float c[D][D];
+#pragma unroll
+                for (int r = 0; r < D; ++r)
+#pragma unroll
+                    for (int q = 0; q < D; q += 4) {
+                        const float4 v = *reinterpret_cast<const float4 *>(&s.S[gi * D + r][gj * D + q]);
+                        c[r][q] = v.x; c[r][q + 1] = v.y; c[r][q + 2] = v.z; c[r][q + 3] = v.w;
+                    }
+#pragma unroll
+                for (int q = 0; q < D; ++q) {
+                    float av[D], bv[D];
+#pragma unroll
+                    for (int u = 0; u < D; u += 4) {
+                        const float4 a4 = *reinterpret_cast<const float4 *>(&s.RT[q][gi * D + u]);
+                        const float4 b4 = *reinterpret_cast<const float4 *>(&s.RT[q][gj * D + u]);
+                        av[u] = a4.x; av[u + 1] = a4.y; av[u + 2] = a4.z; av[u + 3] = a4.w;
+                        bv[u] = b4.x; bv[u + 1] = b4.y; bv[u + 2] = b4.z; bv[u + 3] = b4.w;
+                    }
+#pragma unroll
+                    for (int r = 0; r < D; ++r)
+#pragma unroll
+                        for (int cc = 0; cc < D; ++cc) c[r][cc] = fmaf(-av[r], bv[cc], c[r][cc]);
+                }
+#pragma unroll
+                for (int r = 0; r < D; ++r)
+#pragma unroll
+                    for (int q = 0; q < D; q += 4)
+                        *reinterpret_cast<float4 *>(&s.S[gi * D + r][gj * D + q]) =
+                            make_float4(c[r][q], c[r][q + 1], c[r][q + 2], c[r][q + 3]);
+            }
+            // U_{<k,k} = R_{<k,k} R_kk^-1, one row per thread
+            for (int i = t; i < kd; i += kWork) {
+                float rv[D];
+#pragma unroll
+                for (int q = 0; q < D; q += 4) {
+                    const float4 v = *reinterpret_cast<const float4 *>(&s.R[i][kd + q]);
+                    rv[q] = v.x; rv[q + 1] = v.y; rv[q + 2] = v.z; rv[q + 3] = v.w;
+                }
+                float o[D];
+#pragma unroll
+                for (int jj = 0; jj < D; ++jj) {
+                    float acc = 0.0f;
+#pragma unroll
+                    for (int q = 0; q <= jj; ++q) acc = fmaf(rv[q], s.Rinv[k][q * D + jj], acc);
+                    o[jj] = acc;
+                }
+                float *dst = U + (c0 + i) * n + c0 + kd;
+#pragma unroll
+                for (int q = 0; q < D; q += 4)
+                    *reinterpret_cast<float4 *>(dst + q) = make_float4(o[q], o[q + 1], o[q + 2], o[q + 3]);
+            }
+            ldl_w_row_block<D>(s, k, P, t, kWork);
         }
         __syncthreads();
     }
+    ldl_w_row_block<D>(s, 0, P, tid, kLdlThreads);
+    __syncthreads();
+    // W (zero below the block diagonal and below the diagonal of W_kk, which S holds as zeros) and R_kk^-1
+    for (int e = tid; e < P * P4; e += kLdlThreads) {
+        const int i = e / P4, j = (e % P4) * 4;
+        const float4 v = j / D >= i / D ? *reinterpret_cast<const float4 *>(&s.S[i][j]) : make_float4(0.f, 0.f, 0.f, 0.f);
+        *reinterpret_cast<float4 *>(Wout + i * kLdlPanel + j) = v;
+    }
+    for (int e = tid; e < G * D * D; e += kLdlThreads) RinvOut[e] = s.Rinv[e / (D * D)][e % (D * D)];
+}
+
+// The trailing update's GEMMs. All have K = kLdlPanel = 128 (the panel width; only the first panel can
+// be narrower, and no update follows it) and both operands K-contiguous (C += A B^T form).
+//
+// ldl_gemm_k128_kernel: C[i][j] = beta C[i][j] + alpha sum_k A[i][k] B[j][k] on a 64 x 64 tile, the
+// whole K of both operands copied to shared memory up front by cp.async (one load latency per tile:
+// these run on the critical path between two panels). Thread (ty, tx) computes rows ty + 16 i and
+// columns tx + 16 j (i, j < 4), reading its operand rows 16 bytes of K at a time. EPI_D > 0 (alpha = 1,
+// beta = 0, N a multiple of EPI_D): also U2 = C blockdiag(Rinv) with the EPI_D x EPI_D blocks Rinv[g]
+// (U2[i][j] = sum_q C[i][gD + q] Rinv[g][q][j - gD], g = j / EPI_D).
+constexpr int kGemmTile = 64, kGemmKAll = kLdlPanel, kGemmLd = kGemmKAll + 4;
+
+struct GemmK128Smem {
+    float As[kGemmTile][kGemmLd];     // A tile, row-major (rows 16-byte aligned, 4 banks apart)
+    float Bs[kGemmTile][kGemmLd];
+};
+static_assert(kGemmTile * (kGemmTile + 4) <= kGemmTile * kGemmLd, "the C tile reuses As");
+
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gsrc, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(smem_dst)), "l"(gsrc),
+                 "r"(valid ? 16 : 0)
+                 : "memory");
+}
+
+template <int EPI_D>
+__global__ void __launch_bounds__(256)
+ldl_gemm_k128_kernel(const float *__restrict__ Am, int64_t lda, const float *__restrict__ Bm, int64_t ldb,
+                     float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, float alpha, float beta,
+                     const float *__restrict__ Rinv, float *__restrict__ U2, int64_t ldu2) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    GemmK128Smem &s = *reinterpret_cast<GemmK128Smem *>(smem_raw);
+    const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kGemmTile, j0 = static_cast<int64_t>(blockIdx.x) * kGemmTile;
+    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+    // 64 rows x 32 16-byte chunks per operand: rows (tid >> 3) + 32 v, chunks (tid & 7) + 8 u; rows past
+    // the matrix are zero-filled (the source address stays the operand's first row)
+#pragma unroll
+    for (int v = 0; v < 2; ++v)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int r = (tid >> 3) + 32 * v, q = (tid & 7) + 8 * u;
+            const bool va = i0 + r < M, vb = j0 + r < N;
+            cp_async16(&s.As[r][4 * q], Am + (va ? (i0 + r) * lda : 0) + 4 * q, va);
+            cp_async16(&s.Bs[r][4 * q], Bm + (vb ? (j0 + r) * ldb : 0) + 4 * q, vb);
+        }
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    float acc[4][4] = {};
+#pragma unroll 4
+    for (int k = 0; k < kGemmKAll; k += 4) {
+        float4 a[4], b[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            a[i] = *reinterpret_cast<const float4 *>(&s.As[ty + 16 * i][k]);
+            b[i] = *reinterpret_cast<const float4 *>(&s.Bs[tx + 16 * i][k]);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                acc[i][j] = fmaf(a[i].x, b[j].x, acc[i][j]);
+                acc[i][j] = fmaf(a[i].y, b[j].y, acc[i][j]);
+                acc[i][j] = fmaf(a[i].z, b[j].z, acc[i][j]);
+                acc[i][j] = fmaf(a[i].w, b[j].w, acc[i][j]);
+            }
+    }
+    if constexpr (EPI_D > 0) {
+        // the C tile through shared memory: a group of EPI_D columns spans several threads
+        __syncthreads();
+        float(*Cs)[kGemmTile + 4] = reinterpret_cast<float(*)[kGemmTile + 4]>(&s.As[0][0]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) Cs[ty + 16 * i][tx + 16 * j] = acc[i][j];
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int lc = tx + 16 * j;
+            const int64_t c = j0 + lc;
+            if (c >= N) continue;
+            const int jj = static_cast<int>(c % EPI_D), lg = lc - jj;
+            const float *Rg = Rinv + (c / EPI_D) * EPI_D * EPI_D + jj;
+            float rq[EPI_D];
+#pragma unroll
+            for (int q = 0; q < EPI_D; ++q) rq[q] = __ldg(Rg + q * EPI_D);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int64_t r = i0 + ty + 16 * i;
+                if (r >= M) continue;
+                float u = 0.0f;
+#pragma unroll
+                for (int q = 0; q < EPI_D; ++q) u = fmaf(Cs[ty + 16 * i][lg + q], rq[q], u);
+                U2[r * ldu2 + c] = u;
+            }
+        }
+    }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int64_t r = i0 + ty * 4 + i;
+        const int64_t r = i0 + ty + 16 * i;
         if (r >= M) continue;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const int64_t c = j0 + tx * 4 + j;
+            const int64_t c = j0 + tx + 16 * j;
             if (c >= N) continue;
             float *p = C + r * ldc + c;
             *p = beta == 0.0f ? alpha * acc[i][j] : fmaf(alpha, acc[i][j], beta * *p);
+        }
+    }
+}
+
+// ldl_syrk_kernel: the leading square of the Schur update, C -= Z Z^T on the tiles (ti <= tj) of a
+// 128 x 128 tiling of the m x m upper triangle (m a multiple of 4; one CTA per tile, blockIdx.x the
+// tile's index in row-major order). 8 x 8 outputs per thread (rows ty*4 + {0..3, 64..67}, likewise the
+// columns), K in steps of 16 through two shared-memory stages, the next step's loads in registers
+// while the current one is multiplied.
+constexpr int kSyrkTile = 128, kSyrkK = 16, kSyrkLd = kSyrkTile + 4;
+
+__global__ void __launch_bounds__(256, 2)
+ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C, int64_t ldc, int64_t m, int nt) {
+    __shared__ __align__(16) float As[2][kSyrkK][kSyrkLd];
+    __shared__ __align__(16) float Bs[2][kSyrkK][kSyrkLd];
+    int ti = 0, rem = static_cast<int>(blockIdx.x);
+    while (rem >= nt - ti) { rem -= nt - ti; ++ti; }
+    const int tj = ti + rem;
+    const int64_t i0 = static_cast<int64_t>(ti) * kSyrkTile, j0 = static_cast<int64_t>(tj) * kSyrkTile;
+    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+    // loads: rows (tid >> 2) + 64 v of each operand, 16-byte chunk (tid & 3) of the K step
+    const int lr = tid >> 2, lq = tid & 3;
+    float4 pa[2], pb[2];
+    const auto load = [&](int k0) {
+#pragma unroll
+        for (int v = 0; v < 2; ++v) {
+            const int64_t ra = i0 + lr + 64 * v, rb = j0 + lr + 64 * v;
+            pa[v] = ra < m ? __ldg(reinterpret_cast<const float4 *>(Zm + ra * ldz + k0 + 4 * lq)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            pb[v] = rb < m ? __ldg(reinterpret_cast<const float4 *>(Zm + rb * ldz + k0 + 4 * lq)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    };
+    const auto store = [&](int st) {
+#pragma unroll
+        for (int v = 0; v < 2; ++v) {
+            const int r = lr + 64 * v, k = 4 * lq;
+            As[st][k][r] = pa[v].x; As[st][k + 1][r] = pa[v].y; As[st][k + 2][r] = pa[v].z; As[st][k + 3][r] = pa[v].w;
+            Bs[st][k][r] = pb[v].x; Bs[st][k + 1][r] = pb[v].y; Bs[st][k + 2][r] = pb[v].z; Bs[st][k + 3][r] = pb[v].w;
+        }
+    };
+    float acc[8][8] = {};
+    load(0);
+    store(0);
+    __syncthreads();
+    constexpr int kSteps = kLdlPanel / kSyrkK;
+#pragma unroll 1
+    for (int step = 0; step < kSteps; ++step) {
+        const int st = step & 1;
+        if (step + 1 < kSteps) load((step + 1) * kSyrkK);
+#pragma unroll
+        for (int kk = 0; kk < kSyrkK; ++kk) {
+            const float4 a0 = *reinterpret_cast<const float4 *>(&As[st][kk][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4 *>(&As[st][kk][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4 *>(&Bs[st][kk][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4 *>(&Bs[st][kk][64 + tx * 4]);
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+        if (step + 1 < kSteps) store(st ^ 1);
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int64_t r = i0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4);
+        if (r >= m) continue;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int64_t c = j0 + h * 64 + tx * 4;
+            if (c >= m) continue;                  // m % 4 == 0: a 4-column group is all in or all out
+            float4 *p = reinterpret_cast<float4 *>(C + r * ldc + c);
+            float4 v = *p;
+            v.x -= acc[i][4 * h]; v.y -= acc[i][4 * h + 1]; v.z -= acc[i][4 * h + 2]; v.w -= acc[i][4 * h + 3];
+            *p = v;
         }
     }
 }
@@ -205,11 +503,27 @@ size_t ldl_factor_scratch_bytes(int64_t n) {
     return al(nn * nn * 4) + al(nn * kLdlPanel * 4) + 2 * al(size_t(kLdlPanel) * kLdlPanel * 4);
 }
 
-static cudaError_t gemm_nt(const float *A, int64_t lda, const float *B, int64_t ldb, float *C, int64_t ldc, int64_t M,
-                           int64_t N, int K, float alpha, float beta, bool upper, cudaStream_t st) {
+static cudaError_t gemm_k128(const float *A, int64_t lda, const float *B, int64_t ldb, float *C, int64_t ldc,
+                             int64_t M, int64_t N, float alpha, float beta, const float *Rinv, float *U2, int64_t ldu2,
+                             int epi_d, cudaStream_t st) {
     if (M <= 0 || N <= 0) return cudaSuccess;
+    void (*fn)(const float *, int64_t, const float *, int64_t, float *, int64_t, int64_t, int64_t, float, float,
+               const float *, float *, int64_t) =
+        epi_d == 8 ? ldl_gemm_k128_kernel<8> : epi_d == 4 ? ldl_gemm_k128_kernel<4> : ldl_gemm_k128_kernel<0>;
+    const int smem = static_cast<int>(sizeof(GemmK128Smem));
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(fn), smem);
+    if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>((N + kGemmTile - 1) / kGemmTile), static_cast<unsigned>((M + kGemmTile - 1) / kGemmTile));
-    ldl_gemm_nt_kernel<<<grid, 256, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, alpha, beta, upper ? 1 : 0);
+    fn<<<grid, 256, smem, st>>>(A, lda, B, ldb, C, ldc, M, N, alpha, beta, Rinv, U2, ldu2);
+    count_launch();
+    return cudaGetLastError();
+}
+
+// C[0:m, 0:m] -= Z Z^T on the upper tiles (Z: m x kLdlPanel, leading dimension ldz).
+static cudaError_t syrk_upper(const float *Z, int64_t ldz, float *C, int64_t ldc, int64_t m, cudaStream_t st) {
+    if (m <= 0) return cudaSuccess;
+    const int nt = static_cast<int>((m + kSyrkTile - 1) / kSyrkTile);
+    ldl_syrk_kernel<<<static_cast<unsigned>(nt * (nt + 1) / 2), 256, 0, st>>>(Z, ldz, C, ldc, m, nt);
     count_launch();
     return cudaGetLastError();
 }
@@ -249,9 +563,9 @@ cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
     const size_t nn = static_cast<size_t>(n);
     const auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
     float *S = a.scratch;
-    float *Y = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(S) + al(nn * nn * 4));
-    float *Minv = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(Y) + al(nn * kLdlPanel * 4));
-    float *Binv = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(Minv) + al(size_t(kLdlPanel) * kLdlPanel * 4));
+    float *Z = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(S) + al(nn * nn * 4));
+    float *W = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(Z) + al(nn * kLdlPanel * 4));
+    float *Rinv = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(W) + al(size_t(kLdlPanel) * kLdlPanel * 4));
     void (*panel)(const float *, int64_t, int64_t, int, float *, float *, float *, float *, int32_t *) =
         a.d == 4 ? ldl_panel_kernel<4> : ldl_panel_kernel<8>;
     const int smem = static_cast<int>(sizeof(LdlPanelSmem));
@@ -267,7 +581,7 @@ cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
     if ((e = cudaMemsetAsync(a.U, 0, nn * nn * 4, st)) != cudaSuccess) return e;
     int64_t c1 = n;
     int64_t c0 = c1 > kLdlPanel ? c1 - kLdlPanel : 0;
-    panel<<<1, kLdlThreads, smem, st>>>(S, n, c0, static_cast<int>(c1 - c0), a.U, a.D, Minv, Binv, a.status);
+    panel<<<1, kLdlThreads, smem, st>>>(S, n, c0, static_cast<int>(c1 - c0), a.U, a.D, W, Rinv, a.status);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     bool side_pending = false;
@@ -276,22 +590,24 @@ cudaError_t launch_ldl_factor(const LdlFactorArgs &a, cudaStream_t st) {
         const int64_t p0 = c0 > kLdlPanel ? c0 - kLdlPanel : 0;
         const int Pn = static_cast<int>(c0 - p0);
         if (side_pending && (e = cudaStreamWaitEvent(st, ev.join, 0)) != cudaSuccess) return e;
-        // Y = S_QP M^-T, U_QP = S_QP (D^-1 M^-1)^T (P = kLdlPanel here)
-        if ((e = gemm_nt(S + c0, n, Minv, kLdlPanel, Y, kLdlPanel, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
-        if ((e = gemm_nt(S + c0, n, Binv, kLdlPanel, a.U + c0, n, c0, P, P, 1.0f, 0.0f, false, st)) != cudaSuccess) return e;
-        // the next panel's columns of S_QQ -= Y U_QP^T (rows 0 .. c0, columns p0 .. c0)
-        if ((e = gemm_nt(Y, kLdlPanel, a.U + p0 * n + c0, n, S + p0, n, c0, Pn, P, -1.0f, 1.0f, false, st)) != cudaSuccess)
+        // the factor's column block above the panel, Z = S_QP W^T, and U_QP = Z Rd^-1 (P = kLdlPanel here)
+        if ((e = gemm_k128(S + c0, n, W, kLdlPanel, Z, kLdlPanel, c0, P, 1.0f, 0.0f, Rinv, a.U + c0, n, a.d, st)) !=
+            cudaSuccess)
             return e;
-        // the next panel on the side stream, after all of the above (it overwrites M^-1, D^-1 M^-1)
+        // the next panel's columns of S_QQ -= Z Z^T (rows 0 .. c0, columns p0 .. c0)
+        if ((e = gemm_k128(Z, kLdlPanel, Z + p0 * kLdlPanel, kLdlPanel, S + p0, n, c0, Pn, -1.0f, 1.0f, nullptr, nullptr,
+                           0, 0, st)) != cudaSuccess)
+            return e;
+        // the next panel on the side stream, after all of the above (it overwrites W and the R_kk^-1)
         if ((e = cudaEventRecord(ev.fork, st)) != cudaSuccess) return e;
         if ((e = cudaStreamWaitEvent(side, ev.fork, 0)) != cudaSuccess) return e;
-        panel<<<1, kLdlThreads, smem, side>>>(S, n, p0, Pn, a.U, a.D, Minv, Binv, a.status);
+        panel<<<1, kLdlThreads, smem, side>>>(S, n, p0, Pn, a.U, a.D, W, Rinv, a.status);
         count_launch();
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         if ((e = cudaEventRecord(ev.join, side)) != cudaSuccess) return e;
         side_pending = true;
         // the rest of the update, the leading p0 x p0 square (upper tiles), meanwhile
-        if ((e = gemm_nt(Y, kLdlPanel, a.U + c0, n, S, n, p0, p0, P, -1.0f, 1.0f, true, st)) != cudaSuccess) return e;
+        if ((e = syrk_upper(Z, kLdlPanel, S, n, p0, st)) != cudaSuccess) return e;
         c1 = c0;
         c0 = p0;
     }
