@@ -787,7 +787,7 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
         }
         sweep_bar();
         if (ok && !mbar_wait(&s.wfull, c & 1, p.status)) ok = false;
-        uint32_t bits[2][2] = {{0u, 0u}, {0u, 0u}};
+        uint64_t bits[2] = {0ull, 0ull};             // this thread's 32 codes of rows lane, lane + 32
         float csq = 0.0f;
         // the chunk's slices in order: slice s (its 32 rows of U's diagonal block in one or two ring
         // stages) is rounded by warp s in place in T (target - weight -> error); its errors then reach
@@ -836,8 +836,7 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                             tb[rr][4 * hh + 3] = (wv.w + fv.w) - bb[4 * hh + 3];
                         }
                     }
-                    // u = A^{-1} (t - b) and z = clip(round(u), 0, 3)
-                    float u[2][D];
+                    // u = A^{-1} (t - b) (written out as it is formed) and z = clip(round(u), 0, 3)
                     uint32_t z[2][D];
 #pragma unroll
                     for (int i = 0; i < D; ++i) {
@@ -852,8 +851,9 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                             float v = 0.0f;
 #pragma unroll
                             for (int jj = 0; jj < D; ++jj) v = fmaf(ar[jj], tb[rr][jj], v);
-                            u[rr][i] = v;
                             z[rr][i] = round_clamp3(v);
+                            const int64_t grow = tile * kSwR + lane + 32 * rr;
+                            if (p.latent && grow < p.m) p.latent[grow * n + col0 + j * D + i] = v;
                         }
                     }
                     // e = w - (A z + b)
@@ -877,14 +877,10 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
 #pragma unroll
                     for (int rr = 0; rr < 2; ++rr) {
                         const int64_t grow = tile * kSwR + lane + 32 * rr;
-                        if (p.latent && grow < p.m) {
-#pragma unroll
-                            for (int i = 0; i < D; ++i) p.latent[grow * n + col0 + j * D + i] = u[rr][i];
-                        }
                         uint32_t zb = 0;
 #pragma unroll
                         for (int i = 0; i < D; ++i) zb |= z[rr][i] << (2 * i);
-                        bits[rr][(j * D) >> 4] |= zb << (2 * ((j * D) & 15));
+                        bits[rr] |= static_cast<uint64_t>(zb) << (2 * j * D);
                         if (grow < p.m) {
 #pragma unroll
                             for (int i = 0; i < D; ++i) csq = fmaf(e[rr][i], e[rr][i], csq);
@@ -911,45 +907,50 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
             }
             if (sl < kSwSlices - 1 && q >= sl) slice_bar(sl);
             if (q > sl) {
-                // T[r][this slice] += e_slice U[slice rows][this thread's columns], both rows per U load
-                float2 acc2[2][kSwS / 2];
-#pragma unroll
-                for (int rr = 0; rr < 2; ++rr) {
-                    const float4 *own = reinterpret_cast<const float4 *>(&s.T[lane + 32 * rr][kSwS * q]);
-#pragma unroll
-                    for (int c4 = 0; c4 < kSwS / 4; ++c4) {
-                        const float4 v = own[c4];
-                        acc2[rr][2 * c4] = make_float2(v.x, v.y);
-                        acc2[rr][2 * c4 + 1] = make_float2(v.z, v.w);
-                    }
-                }
+                // T[r][this slice] += e_slice U[slice rows][this thread's columns], both rows per U load, the
+                // slice's 32 columns in two halves of 16
 #pragma unroll 1
-                for (int i4 = 0; i4 < span / 4; ++i4) {
-                    const float4 e0 = reinterpret_cast<const float4 *>(&s.T[lane][kSwS * sl])[i4];
-                    const float4 e1 = reinterpret_cast<const float4 *>(&s.T[lane + 32][kSwS * sl])[i4];
-                    const float ev0[4] = {e0.x, e0.y, e0.z, e0.w}, ev1[4] = {e1.x, e1.y, e1.z, e1.w};
+                for (int hc = 0; hc < 2; ++hc) {
+                    float2 acc2[2][kSwS / 4];
 #pragma unroll
-                    for (int ii = 0; ii < 4; ++ii) {
-                        const float4 *ur = reinterpret_cast<const float4 *>(urow(4 * i4 + ii) + kSwS * q);
-                        const float2 x0 = make_float2(ev0[ii], ev0[ii]), x1 = make_float2(ev1[ii], ev1[ii]);
+                    for (int rr = 0; rr < 2; ++rr) {
+                        const float4 *own = reinterpret_cast<const float4 *>(&s.T[lane + 32 * rr][kSwS * q + 16 * hc]);
 #pragma unroll
-                        for (int c4 = 0; c4 < kSwS / 4; ++c4) {
-                            const float4 uv = ur[c4];
-                            const float2 ua = make_float2(uv.x, uv.y), ub = make_float2(uv.z, uv.w);
-                            acc2[0][2 * c4] = __ffma2_rn(x0, ua, acc2[0][2 * c4]);
-                            acc2[0][2 * c4 + 1] = __ffma2_rn(x0, ub, acc2[0][2 * c4 + 1]);
-                            acc2[1][2 * c4] = __ffma2_rn(x1, ua, acc2[1][2 * c4]);
-                            acc2[1][2 * c4 + 1] = __ffma2_rn(x1, ub, acc2[1][2 * c4 + 1]);
+                        for (int c4 = 0; c4 < kSwS / 8; ++c4) {
+                            const float4 v = own[c4];
+                            acc2[rr][2 * c4] = make_float2(v.x, v.y);
+                            acc2[rr][2 * c4 + 1] = make_float2(v.z, v.w);
                         }
-                        asm volatile("" ::: "memory");
                     }
-                }
+#pragma unroll 1
+                    for (int i4 = 0; i4 < span / 4; ++i4) {
+                        const float4 e0 = reinterpret_cast<const float4 *>(&s.T[lane][kSwS * sl])[i4];
+                        const float4 e1 = reinterpret_cast<const float4 *>(&s.T[lane + 32][kSwS * sl])[i4];
+                        const float ev0[4] = {e0.x, e0.y, e0.z, e0.w}, ev1[4] = {e1.x, e1.y, e1.z, e1.w};
 #pragma unroll
-                for (int rr = 0; rr < 2; ++rr) {
-                    float4 *ownw = reinterpret_cast<float4 *>(&s.T[lane + 32 * rr][kSwS * q]);
+                        for (int ii = 0; ii < 4; ++ii) {
+                            const float4 *ur = reinterpret_cast<const float4 *>(urow(4 * i4 + ii) + kSwS * q + 16 * hc);
+                            const float2 x0 = make_float2(ev0[ii], ev0[ii]), x1 = make_float2(ev1[ii], ev1[ii]);
 #pragma unroll
-                    for (int c4 = 0; c4 < kSwS / 4; ++c4)
-                        ownw[c4] = make_float4(acc2[rr][2 * c4].x, acc2[rr][2 * c4].y, acc2[rr][2 * c4 + 1].x, acc2[rr][2 * c4 + 1].y);
+                            for (int c4 = 0; c4 < kSwS / 8; ++c4) {
+                                const float4 uv = ur[c4];
+                                const float2 ua = make_float2(uv.x, uv.y), ub = make_float2(uv.z, uv.w);
+                                acc2[0][2 * c4] = __ffma2_rn(x0, ua, acc2[0][2 * c4]);
+                                acc2[0][2 * c4 + 1] = __ffma2_rn(x0, ub, acc2[0][2 * c4 + 1]);
+                                acc2[1][2 * c4] = __ffma2_rn(x1, ua, acc2[1][2 * c4]);
+                                acc2[1][2 * c4 + 1] = __ffma2_rn(x1, ub, acc2[1][2 * c4 + 1]);
+                            }
+                            asm volatile("" ::: "memory");
+                        }
+                    }
+#pragma unroll
+                    for (int rr = 0; rr < 2; ++rr) {
+                        float4 *ownw = reinterpret_cast<float4 *>(&s.T[lane + 32 * rr][kSwS * q + 16 * hc]);
+#pragma unroll
+                        for (int c4 = 0; c4 < kSwS / 8; ++c4)
+                            ownw[c4] = make_float4(acc2[rr][2 * c4].x, acc2[rr][2 * c4].y, acc2[rr][2 * c4 + 1].x,
+                                                   acc2[rr][2 * c4 + 1].y);
+                    }
                 }
             }
             __syncwarp();
@@ -978,16 +979,17 @@ ldlq_sweep_kernel(const __grid_constant__ CUtensorMap tmU, const __grid_constant
                 if (grow < p.m && p.packed) {
                     uint8_t *pk = p.packed + grow * (n / 4) + col0 / 4;
                     if (col0 + kSwS <= n && (reinterpret_cast<uintptr_t>(pk) & 7u) == 0) {
-                        *reinterpret_cast<uint2 *>(pk) = make_uint2(bits[rr][0], bits[rr][1]);
+                        *reinterpret_cast<uint2 *>(pk) =
+                            make_uint2(static_cast<uint32_t>(bits[rr]), static_cast<uint32_t>(bits[rr] >> 32));
                     } else {
                         for (int i = 0; i < kSwS && col0 + i < n; i += 4)
-                            pk[i / 4] = static_cast<uint8_t>((bits[rr][i >> 4] >> (2 * (i & 15))) & 0xFFu);
+                            pk[i / 4] = static_cast<uint8_t>((bits[rr] >> (2 * i)) & 0xFFu);
                     }
                 }
                 if (grow < p.m && p.codes) {
                     uint8_t *cd = p.codes + grow * n + col0;
                     for (int i = 0; i < kSwS && col0 + i < n; ++i)
-                        cd[i] = static_cast<uint8_t>((bits[rr][i >> 4] >> (2 * (i & 15))) & 3u);
+                        cd[i] = static_cast<uint8_t>((bits[rr] >> (2 * i)) & 3u);
                 }
             }
         }

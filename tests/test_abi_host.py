@@ -156,12 +156,8 @@ def test_product_package_never_reaches_the_oracle():
                 assert not re.search(r"^\s*(import|from)\s+oracle\b|oracle/|brute\.c|lcvq", text, flags=re.M), f
 
 
-# the one known spill: 8 bytes in the d = 8 LDLQ sweep (its feedback tile holds 8 x 8 outputs per thread)
-SPILL_ALLOWED = {"ldlq_sweep_kernel": 8}
-
-
 def test_no_kernel_spills_registers(L):
-    """ptxas resource reports of the build: no entry function spills (one known exception)."""
+    """ptxas resource reports of the build: no entry function spills registers (no exemptions)."""
     import re as _re
     if not all(os.path.exists(lcq_build.ptxas_report(s)) for s in lcq_build.SOURCES):
         lcq_build.build(force=True)
@@ -176,6 +172,5 @@ def test_no_kernel_spills_registers(L):
                 continue
             m = _re.search(r"(\d+) bytes spill stores, (\d+) bytes spill loads", line)
             if m and cur:
-                allowed = max([v for k, v in SPILL_ALLOWED.items() if k in cur], default=0)
-                assert int(m.group(1)) <= allowed and int(m.group(2)) <= allowed, (src, cur, line.strip())
+                assert m.group(1) == m.group(2) == "0", (src, cur, line.strip())
     assert entries > 20
