@@ -109,7 +109,7 @@ def test_llama2_7b_gate_fwd_bwd_full_size_d8_outliers():
     _check_linear(mats[4], 4)         # gate 11008 x 4096, d = 8, 4096 tokens, 1% outlier channels x20
 
 
-@pytest.mark.parametrize("B", [1, 4, 16])
+@pytest.mark.parametrize("B", [1, 2, 4, 16])
 def test_llama3_70b_gate_packed_product_full_size(B):
     mx = wl.llama3_70b_gate_decode(B)[0]
     packed = wl.draw_packed_codes(mx, SEED, 0)

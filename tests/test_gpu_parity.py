@@ -383,6 +383,33 @@ def test_gemm_packed2b_one_token_zero_activations():
             assert max_rel(got, ref) <= TOL_DP
 
 
+def test_gemm_packed2b_two_tokens_independent_scales():
+    # two tokens, one all zero (outputs exactly 0), then one 1e4 x larger than the other: each token is
+    # scaled on its own, so neither loses precision to the other
+    rng = np.random.default_rng(11)
+    m, n, d = 500, 4096, 8
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    for case in ("zero", "scaled"):
+        X = rng.normal(0, 1, (2, n))
+        if case == "zero":
+            X[1, :] = 0.0
+        else:
+            X[1, :] *= 1e4
+        Xb = wl.bf16_bits(X.astype(np.float32))
+        ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+        Y = empty_bf16(2, m)
+        ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, 2, m, n, d)
+        lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+        assert lcq.lcq_device_status(ws) == 0
+        got = host_bf16(Y)
+        assert max_rel(got[0], ref[0]) <= TOL_BF16
+        if case == "zero":
+            assert np.all(got[1] == 0.0)
+        else:
+            assert max_rel(got[1], ref[1]) <= TOL_BF16
+
+
 # ----------------------------------------------------------------------------- failure detection
 
 def test_bounded_wait_reports_timeout_and_context_stays_usable():
