@@ -46,12 +46,15 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the separate encode / packed-product timings")
-    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq", "xform"], default=None,
+    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq", "ldlq70", "ldl_factor", "xform"],
+                    default=None,
                     help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
                          "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
                          "28672 x 8192, gemv = 70B gate at --tokens tokens, ldlq = LDLQ sweep of a "
-                         "9728 x 4096 slice of the 8B gate (one wave, small case), xform = activation "
-                         "transform of the q projection's 16384 x 4096 activations")
+                         "9728 x 4096 slice of the 8B gate (one wave, small case), ldlq70 = LDLQ sweep of "
+                         "the 70B gate 28672 x 8192, ldl_factor = factorisation of its 8192 x 8192 proxy "
+                         "Hessian, xform = activation transform of the q projection's 16384 x 4096 "
+                         "activations")
     ap.add_argument("--tokens", type=int, default=None, help="tokens of the gemv profiling case (default 16)")
     return ap.parse_args()
 
@@ -766,6 +769,29 @@ def profile_case(args):
         def run():
             lcq.lcq_ldlq(W, A, b, U, d, ws, packed=pk_)
         wss = [wsf, ws]
+    elif args.case in ("ldlq70", "ldl_factor"):
+        # the bench's LDLQ workload: the 70B gate and its proxy Hessian (same seeds as time_ldlq_70b)
+        mx = wl.llama3_70b_gate_ldlq()[0]
+        m, n, d = mx.m, mx.n, mx.d
+        H = wl.torch_hessian(torch, n, args.seed + 4000, 0, device)
+        U = torch.empty((n, n), dtype=torch.float32, device=device)
+        wsf = lcq.workspace(lcq.LCQ_OP_LDL_FACTOR, 0, 0, n, d, device)
+        lcq.lcq_ldl_factor(H, d, U, wsf)
+        wss = [wsf]
+        if args.case == "ldl_factor":
+            def run():
+                lcq.lcq_ldl_factor(H, d, U, wsf)
+        else:
+            W = wl.torch_W(torch, mx, args.seed + 4000, 0, device)
+            A = wl.torch_A(torch, mx, args.seed + 4000, 0, device).contiguous()
+            b = wl.torch_b(torch, mx, args.seed + 4000, 0, device).contiguous()
+            pk_ = torch.empty((m, n // 4), dtype=torch.uint8, device=device)
+            mse = torch.empty(1, dtype=torch.float64, device=device)
+            ws = lcq.workspace(lcq.LCQ_OP_LDLQ, 0, m, n, d, device)
+            wss.append(ws)
+
+            def run():
+                lcq.lcq_ldlq(W, A, b, U, d, ws, packed=pk_, mse=mse)
     elif args.case == "xform":
         mx = wl.llama3_8b_layer()[0]
         X = wl.torch_X(torch, mx, args.seed, 0, device)
