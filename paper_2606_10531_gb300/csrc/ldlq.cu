@@ -423,54 +423,74 @@ ldl_gemm_k128_kernel(const float *__restrict__ Am, int64_t lda, const float *__r
 
 // ldl_syrk_kernel: the leading square of the Schur update, C -= Z Z^T on the tiles (ti <= tj) of a
 // 128 x 128 tiling of the m x m upper triangle (m a multiple of 4; one CTA per tile, blockIdx.x the
-// tile's index in row-major order). 8 x 8 outputs per thread (rows ty*4 + {0..3, 64..67}, likewise the
-// columns), K in steps of 16 through two shared-memory stages, the next step's loads in registers
-// while the current one is multiplied.
-constexpr int kSyrkTile = 128, kSyrkK = 16, kSyrkLd = kSyrkTile + 4;
+// tile's index in row-major order). K = 128 in steps of 16: cp.async copies the steps' rows of both
+// operands into a 4-stage raw ring three steps ahead; each step is transposed in shared memory
+// (As[k][row]) for conflict-free 16-byte operand reads; 8 x 8 outputs per thread (rows ty*4 + {0..3,
+// 64..67}, likewise the columns). The epilogue passes the tile through shared memory so that all of a
+// thread's C loads are in flight at once.
+constexpr int kSyrkTile = 128, kSyrkK = 16, kSyrkLd = kSyrkTile + 4, kSyrkRaw = 4;
+constexpr int kSyrkSteps = kLdlPanel / kSyrkK;
+
+struct SyrkSmem {
+    float raw[kSyrkRaw][2][kSyrkTile][kSyrkK];   // [stage][operand][row][k], as copied
+    float T[2][2][kSyrkK][kSyrkLd];              // [buffer][operand][k][row]
+};
+static_assert(sizeof(float) * kSyrkTile * kSyrkTile <= sizeof(float) * kSyrkRaw * 2 * kSyrkTile * kSyrkK,
+              "the epilogue's C tile reuses the raw ring");
 
 __global__ void __launch_bounds__(256, 2)
 ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C, int64_t ldc, int64_t m, int nt) {
-    __shared__ __align__(16) float As[2][kSyrkK][kSyrkLd];
-    __shared__ __align__(16) float Bs[2][kSyrkK][kSyrkLd];
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    SyrkSmem &s = *reinterpret_cast<SyrkSmem *>(smem_raw);
     int ti = 0, rem = static_cast<int>(blockIdx.x);
     while (rem >= nt - ti) { rem -= nt - ti; ++ti; }
     const int tj = ti + rem;
     const int64_t i0 = static_cast<int64_t>(ti) * kSyrkTile, j0 = static_cast<int64_t>(tj) * kSyrkTile;
     const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
-    // loads: rows (tid >> 2) + 64 v of each operand, 16-byte chunk (tid & 3) of the K step
+    // copies: rows (tid >> 2) + 64 v of each operand, 16-byte chunk (tid & 3) of the step's 16 columns;
+    // rows past m are zero-filled (the source address stays the operand's first row)
     const int lr = tid >> 2, lq = tid & 3;
-    float4 pa[2], pb[2];
-    const auto load = [&](int k0) {
+    const auto issue = [&](int step) {
+        if (step < kSyrkSteps) {
+            const int k0 = step * kSyrkK, st = step % kSyrkRaw;
 #pragma unroll
-        for (int v = 0; v < 2; ++v) {
-            const int64_t ra = i0 + lr + 64 * v, rb = j0 + lr + 64 * v;
-            pa[v] = ra < m ? __ldg(reinterpret_cast<const float4 *>(Zm + ra * ldz + k0 + 4 * lq)) : make_float4(0.f, 0.f, 0.f, 0.f);
-            pb[v] = rb < m ? __ldg(reinterpret_cast<const float4 *>(Zm + rb * ldz + k0 + 4 * lq)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int v = 0; v < 2; ++v) {
+                const int r = lr + 64 * v;
+                const bool va = i0 + r < m, vb = j0 + r < m;
+                cp_async16(&s.raw[st][0][r][4 * lq], Zm + (va ? (i0 + r) * ldz : 0) + k0 + 4 * lq, va);
+                cp_async16(&s.raw[st][1][r][4 * lq], Zm + (vb ? (j0 + r) * ldz : 0) + k0 + 4 * lq, vb);
+            }
         }
+        asm volatile("cp.async.commit_group;" ::: "memory");
     };
-    const auto store = [&](int st) {
-#pragma unroll
-        for (int v = 0; v < 2; ++v) {
-            const int r = lr + 64 * v, k = 4 * lq;
-            As[st][k][r] = pa[v].x; As[st][k + 1][r] = pa[v].y; As[st][k + 2][r] = pa[v].z; As[st][k + 3][r] = pa[v].w;
-            Bs[st][k][r] = pb[v].x; Bs[st][k + 1][r] = pb[v].y; Bs[st][k + 2][r] = pb[v].z; Bs[st][k + 3][r] = pb[v].w;
-        }
-    };
+    issue(0);
+    issue(1);
+    issue(2);
     float acc[8][8] = {};
-    load(0);
-    store(0);
-    __syncthreads();
-    constexpr int kSteps = kLdlPanel / kSyrkK;
 #pragma unroll 1
-    for (int step = 0; step < kSteps; ++step) {
-        const int st = step & 1;
-        if (step + 1 < kSteps) load((step + 1) * kSyrkK);
+    for (int step = 0; step < kSyrkSteps; ++step) {
+        asm volatile("cp.async.wait_group 2;" ::: "memory");   // this step's copies have landed
+        __syncthreads();                                      // ... for every thread; step - 1 is consumed
+        issue(step + 3);                                      // into the raw stage step - 1 used
+        const int st = step % kSyrkRaw, tb = step & 1;
+#pragma unroll
+        for (int o = 0; o < 2; ++o)
+#pragma unroll
+            for (int v = 0; v < 2; ++v) {
+                const int r = lr + 64 * v;
+                const float4 x = *reinterpret_cast<const float4 *>(&s.raw[st][o][r][4 * lq]);
+                s.T[tb][o][4 * lq][r] = x.x;
+                s.T[tb][o][4 * lq + 1][r] = x.y;
+                s.T[tb][o][4 * lq + 2][r] = x.z;
+                s.T[tb][o][4 * lq + 3][r] = x.w;
+            }
+        __syncthreads();
 #pragma unroll
         for (int kk = 0; kk < kSyrkK; ++kk) {
-            const float4 a0 = *reinterpret_cast<const float4 *>(&As[st][kk][ty * 4]);
-            const float4 a1 = *reinterpret_cast<const float4 *>(&As[st][kk][64 + ty * 4]);
-            const float4 b0 = *reinterpret_cast<const float4 *>(&Bs[st][kk][tx * 4]);
-            const float4 b1 = *reinterpret_cast<const float4 *>(&Bs[st][kk][64 + tx * 4]);
+            const float4 a0 = *reinterpret_cast<const float4 *>(&s.T[tb][0][kk][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4 *>(&s.T[tb][0][kk][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4 *>(&s.T[tb][1][kk][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4 *>(&s.T[tb][1][kk][64 + tx * 4]);
             const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
             const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
@@ -478,21 +498,35 @@ ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C
 #pragma unroll
                 for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
         }
-        if (step + 1 < kSteps) store(st ^ 1);
-        __syncthreads();
     }
+    // the tile through shared memory (the raw ring is free: every copy has been consumed)
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    float(*Cs)[kSyrkTile] = reinterpret_cast<float(*)[kSyrkTile]>(&s.raw[0][0][0][0]);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        const int64_t r = i0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4);
-        if (r >= m) continue;
+        const int r = i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4;
+        *reinterpret_cast<float4 *>(&Cs[r][tx * 4]) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+        *reinterpret_cast<float4 *>(&Cs[r][64 + tx * 4]) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+    }
+    __syncthreads();
+    // 16-byte chunk e = tid + 256 u of the tile: row e / 32, columns 4 (e % 32) .. + 3
+    constexpr int kChunks = kSyrkTile * kSyrkTile / 4 / 256;
+    float4 cv[kChunks];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int64_t c = j0 + h * 64 + tx * 4;
-            if (c >= m) continue;                  // m % 4 == 0: a 4-column group is all in or all out
-            float4 *p = reinterpret_cast<float4 *>(C + r * ldc + c);
-            float4 v = *p;
-            v.x -= acc[i][4 * h]; v.y -= acc[i][4 * h + 1]; v.z -= acc[i][4 * h + 2]; v.w -= acc[i][4 * h + 3];
-            *p = v;
+    for (int u = 0; u < kChunks; ++u) {
+        const int e = tid + 256 * u, r = e >> 5, c = 4 * (e & 31);
+        cv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i0 + r < m && j0 + c < m) cv[u] = *reinterpret_cast<const float4 *>(C + (i0 + r) * ldc + j0 + c);
+    }
+#pragma unroll
+    for (int u = 0; u < kChunks; ++u) {
+        const int e = tid + 256 * u, r = e >> 5, c = 4 * (e & 31);
+        if (i0 + r < m && j0 + c < m) {     // m % 4 == 0: a 4-column chunk is all in or all out
+            const float4 z = *reinterpret_cast<const float4 *>(&Cs[r][c]);
+            float4 v = cv[u];
+            v.x -= z.x; v.y -= z.y; v.z -= z.z; v.w -= z.w;
+            *reinterpret_cast<float4 *>(C + (i0 + r) * ldc + j0 + c) = v;
         }
     }
 }
@@ -523,7 +557,10 @@ static cudaError_t gemm_k128(const float *A, int64_t lda, const float *B, int64_
 static cudaError_t syrk_upper(const float *Z, int64_t ldz, float *C, int64_t ldc, int64_t m, cudaStream_t st) {
     if (m <= 0) return cudaSuccess;
     const int nt = static_cast<int>((m + kSyrkTile - 1) / kSyrkTile);
-    ldl_syrk_kernel<<<static_cast<unsigned>(nt * (nt + 1) / 2), 256, 0, st>>>(Z, ldz, C, ldc, m, nt);
+    const int smem = static_cast<int>(sizeof(SyrkSmem));
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(ldl_syrk_kernel), smem);
+    if (e != cudaSuccess) return e;
+    ldl_syrk_kernel<<<static_cast<unsigned>(nt * (nt + 1) / 2), 256, smem, st>>>(Z, ldz, C, ldc, m, nt);
     count_launch();
     return cudaGetLastError();
 }
