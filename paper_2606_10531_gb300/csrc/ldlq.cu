@@ -426,8 +426,8 @@ ldl_gemm_k128_kernel(const float *__restrict__ Am, int64_t lda, const float *__r
 // tile's index in row-major order). K = 128 in steps of 16: cp.async copies the steps' rows of both
 // operands into a 4-stage raw ring three steps ahead; each step is transposed in shared memory
 // (As[k][row]) for conflict-free 16-byte operand reads; 8 x 8 outputs per thread (rows ty*4 + {0..3,
-// 64..67}, likewise the columns). The epilogue passes the tile through shared memory so that all of a
-// thread's C loads are in flight at once.
+// 64..67}, likewise the columns), accumulated with packed fp32x2 FMAs. The epilogue passes the tile
+// through shared memory so that all of a thread's C loads are in flight at once.
 constexpr int kSyrkTile = 128, kSyrkK = 16, kSyrkLd = kSyrkTile + 4, kSyrkRaw = 4;
 constexpr int kSyrkSteps = kLdlPanel / kSyrkK;
 
@@ -466,7 +466,11 @@ ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C
     issue(0);
     issue(1);
     issue(2);
-    float acc[8][8] = {};
+    float2 acc[8][4];                                  // acc[i][j] holds columns 2j, 2j + 1 (packed FMAs)
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = make_float2(0.0f, 0.0f);
 #pragma unroll 1
     for (int step = 0; step < kSyrkSteps; ++step) {
         asm volatile("cp.async.wait_group 2;" ::: "memory");   // this step's copies have landed
@@ -492,11 +496,14 @@ ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C
             const float4 b0 = *reinterpret_cast<const float4 *>(&s.T[tb][1][kk][tx * 4]);
             const float4 b1 = *reinterpret_cast<const float4 *>(&s.T[tb][1][kk][64 + tx * 4]);
             const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+            const float2 bv[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
+                                  make_float2(b1.z, b1.w)};
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < 8; ++i) {
+                const float2 ai = make_float2(av[i], av[i]);
 #pragma unroll
-                for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+                for (int j = 0; j < 4; ++j) acc[i][j] = __ffma2_rn(ai, bv[j], acc[i][j]);
+            }
         }
     }
     // the tile through shared memory (the raw ring is free: every copy has been consumed)
@@ -506,8 +513,8 @@ ldl_syrk_kernel(const float *__restrict__ Zm, int64_t ldz, float *__restrict__ C
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const int r = i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4;
-        *reinterpret_cast<float4 *>(&Cs[r][tx * 4]) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-        *reinterpret_cast<float4 *>(&Cs[r][64 + tx * 4]) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+        *reinterpret_cast<float4 *>(&Cs[r][tx * 4]) = make_float4(acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y);
+        *reinterpret_cast<float4 *>(&Cs[r][64 + tx * 4]) = make_float4(acc[i][2].x, acc[i][2].y, acc[i][3].x, acc[i][3].y);
     }
     __syncthreads();
     // 16-byte chunk e = tid + 256 u of the tile: row e / 32, columns 4 (e % 32) .. + 3
