@@ -161,12 +161,15 @@ lcq_status lcq_encode_batch(const lcq_encode_item *items, int count, int d, void
  *     H = (U + I) D (U + I)^T
  *
  * U is strictly upper block-triangular in d x d blocks (zero on and below the block diagonal), D is
- * block diagonal. The blocks are eliminated from the last to the first in 128-column panels, in fp32.
+ * block diagonal. Computed in fp32 through the Cholesky factorisation H = R R^T in reverse index order
+ * (R upper triangular; 128-column panels from the last to the first): with Rd the block diagonal of R,
+ * U + I = R Rd^-1 and D_k = R_kk R_kk^T. D_k is written as the Schur-complement block it factors.
+ * If a pivot of D_k is not positive (H not positive definite), the status word becomes
+ * LCQ_ERR_SINGULAR and that block's contributions are zero.
  *
  * H  [n][n] fp32, symmetric positive definite; only its upper triangle (i <= j) is read.
  * U  [n][n] fp32 output; every element is written.
  * D  [n/d][d][d] fp32 output (block k is D_k), or NULL.
- * If a block D_k is singular (H not positive definite) the status word becomes LCQ_ERR_SINGULAR.
  * Needs lcq_workspace_size(LCQ_OP_LDL_FACTOR, 0, 0, n, d) bytes of ws (a copy of H, about 4 n^2 bytes).
  * Streams: each panel's factorisation runs on a library-owned high-priority stream (one per device),
  * forked from and joined back to `stream` by events, so work enqueued on `stream` after the call sees
