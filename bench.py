@@ -662,7 +662,10 @@ def e2e_arm(torch, lcq, wl, args, device, world, rank):
     every step copies W, X, dY host->device and reads every result of the step back device->host
     (Y, dX, dP, dA, db, the MSE and the packed-product output). Copies run on two copy streams: a
     linear's inputs arrive while the previous linear computes, and its results leave while the next
-    one computes."""
+    one computes. Steps are ordered by events only (a linear's inputs are overwritten after its
+    previous compute, its results after their previous copy out), so one step's readback overlaps the
+    next step's input copies; the timed region ends with a device synchronisation after the last
+    step's readback."""
     layer = [Linear(torch, lcq, wl, mx, args.seed + 7919 * rank, i, device)
              for i, mx in enumerate(wl.llama3_8b_layer())]
     outs = ("Y", "dX", "dP", "dA", "db", "mse", "Yg")
@@ -706,8 +709,6 @@ def e2e_arm(torch, lcq, wl, args, device, world, rank):
                 for k in outs:
                     h[k].copy_(getattr(L, k), non_blocking=True)
                 out.record(cout)
-        main.synchronize()
-        cout.synchronize()
 
     from paper_2606_10531_gb300 import dist as lcq_dist
     for _ in range(max(args.warmup, 3)):
