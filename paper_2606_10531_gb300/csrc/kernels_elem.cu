@@ -522,63 +522,72 @@ quant_decode_kernel(QuantDecodeArgs a) {
 
 // ------------------------------------------------------------------ decode
 
+// One group of d weights per lane, so that a warp's store of its 32 groups is one contiguous run
+// (512 bytes of bf16 at d = 8): W_hat = A z + b with packed fp32x2 FMAs (rows 2jp, 2jp + 1 of A per
+// pair, k in order from b: the plain sum's rounding); a code becomes an exact float as (2^23 + z) - 2^23,
+// its bits OR-ed into 2^23's mantissa. Each lane keeps kDecGroups groups' codes in flight.
+constexpr int kDecGroups = 8;
+
+template <int D>
+__device__ __forceinline__ void decode_group(uint32_t codes, const float2 (&A2)[D / 2][D], const float2 (&b2)[D / 2],
+                                             float (&wh)[D]) {
+    float z[D];
+#pragma unroll
+    for (int k = 0; k < D; ++k) z[k] = __uint_as_float(0x4B000000u | ((codes >> (2 * k)) & 3u)) - 8388608.0f;
+#pragma unroll
+    for (int jp = 0; jp < D / 2; ++jp) {
+        float2 acc = b2[jp];
+#pragma unroll
+        for (int k = 0; k < D; ++k) acc = __ffma2_rn(A2[jp][k], make_float2(z[k], z[k]), acc);
+        wh[2 * jp] = acc.x;
+        wh[2 * jp + 1] = acc.y;
+    }
+}
+
 template <int D>
 __global__ void __launch_bounds__(256)
 decode_kernel(DecodeArgs a) {
-    float Am[D * D], bv[D];
+    float2 A2[D / 2][D], b2[D / 2];
 #pragma unroll
-    for (int i = 0; i < D * D; ++i) Am[i] = __ldg(a.A + i);
+    for (int jp = 0; jp < D / 2; ++jp) {
 #pragma unroll
-    for (int i = 0; i < D; ++i) bv[i] = __ldg(a.b + i);
-    const int64_t total = a.m * a.n;
-    const int64_t nslices = (total + 15) / 16;
-    for (int64_t sl = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; sl < nslices;
-         sl += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t gidx = sl * 16;
-        const int valid = static_cast<int>((total - gidx) < 16 ? (total - gidx) : 16);
-        uint32_t p;
-        if (valid == 16) {
-            p = __ldg(reinterpret_cast<const uint32_t *>(a.packed + gidx / 4));
-        } else {
-            p = 0;
+        for (int k = 0; k < D; ++k) A2[jp][k] = make_float2(__ldg(a.A + (2 * jp) * D + k), __ldg(a.A + (2 * jp + 1) * D + k));
+        b2[jp] = make_float2(__ldg(a.b + 2 * jp), __ldg(a.b + 2 * jp + 1));
+    }
+    const int64_t ngroups = a.m * a.n / D;            // n % d == 0: whole groups
+    const int lane = threadIdx.x & 31;
+    const int64_t warp0 = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
+    const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    constexpr int64_t kSpan = 32 * kDecGroups;         // groups a warp takes per iteration
+    for (int64_t g0 = warp0 * kSpan; g0 < ngroups; g0 += nwarps * kSpan) {
+        uint32_t cw[kDecGroups];
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-                if (k < valid / 4) p |= static_cast<uint32_t>(a.packed[gidx / 4 + k]) << (8 * k);
-        }
-        float wh[16];
-#pragma unroll
-        for (int g = 0; g < 16 / D; ++g) {
-#pragma unroll
-            for (int j = 0; j < D; ++j) {
-                float acc = bv[j];
-#pragma unroll
-                for (int k = 0; k < D; ++k)
-                    acc = fmaf(Am[j * D + k], static_cast<float>((p >> (2 * (g * D + k))) & 3u), acc);
-                wh[g * D + j] = acc;
+        for (int i = 0; i < kDecGroups; ++i) {
+            const int64_t g = g0 + i * 32 + lane;
+            cw[i] = 0;
+            if (g < ngroups) {
+                if (D == 8) cw[i] = __ldg(reinterpret_cast<const uint16_t *>(a.packed) + g);
+                else cw[i] = __ldg(a.packed + g);
             }
         }
-        if (valid == 16) {
-            if (a.W_f32) {
-                float4 *dst = reinterpret_cast<float4 *>(a.W_f32 + gidx);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) dst[q] = make_float4(wh[4 * q], wh[4 * q + 1], wh[4 * q + 2], wh[4 * q + 3]);
+        for (int i = 0; i < kDecGroups; ++i) {
+            const int64_t g = g0 + i * 32 + lane;
+            if (g >= ngroups) continue;
+            float wh[D];
+            decode_group<D>(cw[i], A2, b2, wh);
+            if (a.W_f32) {
+                float4 *dst = reinterpret_cast<float4 *>(a.W_f32 + g * D);
+#pragma unroll
+                for (int q = 0; q < D / 4; ++q) dst[q] = make_float4(wh[4 * q], wh[4 * q + 1], wh[4 * q + 2], wh[4 * q + 3]);
             }
             if (a.W_bf16) {
-                uint4 *dst = reinterpret_cast<uint4 *>(a.W_bf16 + gidx);
-                dst[0] = make_uint4(pack_bf16x2(wh[0], wh[1]), pack_bf16x2(wh[2], wh[3]), pack_bf16x2(wh[4], wh[5]),
-                                    pack_bf16x2(wh[6], wh[7]));
-                dst[1] = make_uint4(pack_bf16x2(wh[8], wh[9]), pack_bf16x2(wh[10], wh[11]),
-                                    pack_bf16x2(wh[12], wh[13]), pack_bf16x2(wh[14], wh[15]));
-            }
-        } else {
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                if (k < valid) {
-                    if (a.W_f32) a.W_f32[gidx + k] = wh[k];
-                    if (a.W_bf16) {
-                        const __nv_bfloat16 h = __float2bfloat16_rn(wh[k]);
-                        a.W_bf16[gidx + k] = *reinterpret_cast<const uint16_t *>(&h);
-                    }
+                if (D == 8) {
+                    *reinterpret_cast<uint4 *>(a.W_bf16 + g * D) =
+                        make_uint4(pack_bf16x2(wh[0], wh[1]), pack_bf16x2(wh[2], wh[3]), pack_bf16x2(wh[4], wh[5]),
+                                   pack_bf16x2(wh[6], wh[7]));
+                } else {
+                    *reinterpret_cast<uint2 *>(a.W_bf16 + g * D) = make_uint2(pack_bf16x2(wh[0], wh[1]), pack_bf16x2(wh[2], wh[3]));
                 }
             }
         }
@@ -820,8 +829,8 @@ cudaError_t launch_quant_decode(const QuantDecodeArgs &a, int d, int num_sms, cu
 }
 
 cudaError_t launch_decode(const DecodeArgs &a, int d, int num_sms, cudaStream_t st) {
-    const int64_t nslices = (a.m * a.n + 15) / 16;
-    int64_t grid = (nslices + 255) / 256;
+    const int64_t nspans = (a.m * a.n / d + 32 * kDecGroups - 1) / (32 * kDecGroups);   // one warp each
+    int64_t grid = (nspans + 7) / 8;
     if (grid > 8LL * num_sms) grid = 8LL * num_sms;
     if (grid < 1) grid = 1;
     trace_begin(LCQ_K_DECODE, st);
