@@ -621,11 +621,18 @@ pack2b_kernel(const uint8_t *__restrict__ codes, int64_t total, uint8_t *__restr
 
 // ------------------------------------------------------------------ dA / db final reduction
 
-__global__ void reduce_partials_kernel(const float *__restrict__ partials, int nparts, int d, float *dA, float *db) {
+// One warp per value: lane l sums partials l, l + 32, ... in order, then a fixed butterfly adds the
+// lanes, so the result is the same on every run (no atomics) and all of a lane's loads are in flight.
+__global__ void __launch_bounds__(256)
+reduce_partials_kernel(const float *__restrict__ partials, int nparts, int d, float *dA, float *db) {
     const int nvals = d * d + d;
-    for (int i = threadIdx.x; i < nvals; i += blockDim.x) {
-        float acc = 0.0f;
-        for (int p = 0; p < nparts; ++p) acc += partials[static_cast<int64_t>(p) * nvals + i];
+    const int i = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (i >= nvals) return;                   // whole warps: i is uniform across the warp
+    float acc = 0.0f;
+#pragma unroll 8
+    for (int p = lane; p < nparts; p += 32) acc += __ldg(partials + static_cast<int64_t>(p) * nvals + i);
+    for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) {
         if (i < d * d) dA[i] = acc;
         else db[i - d * d] = acc;
     }
@@ -938,7 +945,8 @@ cudaError_t launch_pack2b(const uint8_t *codes, int64_t total, uint8_t *packed, 
 
 cudaError_t launch_reduce_partials(const float *partials, int nparts, int d, float *dA, float *db, cudaStream_t st) {
     trace_begin(LCQ_K_REDUCE, st);
-    reduce_partials_kernel<<<1, 128, 0, st>>>(partials, nparts, d, dA, db);
+    const int nvals = d * d + d;
+    reduce_partials_kernel<<<(nvals * 32 + 255) / 256, 256, 0, st>>>(partials, nparts, d, dA, db);
     trace_end(LCQ_K_REDUCE, st);
     count_launch();
     return cudaGetLastError();
