@@ -271,8 +271,14 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
  * reformulated forward (Sec. 3.2 Eq. def:forward_x):
  *   Y = sum_g (X_g A) Z_g^T + sum_g (X_g b) 1^T  ( = X W_hat^T )
  * X [N][n] bf16 activations (any N; built for N <= 16 tokens), packed
- * [m][n/4] uint8 codes, Y [N][m] bf16 output. X_g A is rounded to bf16
- * before the tensor-core product; accumulation is fp32.
+ * [m][n/4] uint8 codes, Y [N][m] bf16 output. How X_g A is rounded before
+ * the product depends on the shape:
+ *   - n % 64 == 0 and n <= 32768, one token: to int16 with one scale per
+ *     token, exact integer sums;
+ *   - the same n, 2-16 tokens: to q = rint(X' 8191 / max|X'_t|) per token
+ *     (five base-8 digits, the tensor cores' fp4 operands), exact integer
+ *     sums;
+ *   - any other shape: to bf16, fp32 accumulation.
  * Needs lcq_workspace_size(LCQ_OP_GEMM_PACKED2B, N, m, n, d).
  */
 lcq_status lcq_gemm_packed2b(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,

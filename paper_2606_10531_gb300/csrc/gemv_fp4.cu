@@ -26,11 +26,13 @@
 //               K = 64), A (codes) from tensor memory, B (digits) from the digit ring, every block
 //               scale 1. It never touches shared memory while MMAs are queued (such an access waits for
 //               them): the converters hand each tile over through a named barrier.
-//   warps 2-9   converters: warp (128-row block, lane quarter) expands the 512 codes of each of its
-//               rows in the tile from the code ring into an fp4 A slot in tensor memory (two slots),
+//   warps 2-9   converters, two teams of four (warps 2-5 and 6-9) taking alternate tiles, so that the
+//               per-tile chain of one team (code loads, mbarrier checks, stores, barrier) overlaps the
+//               other's: a warp expands the 512 codes of its TMEM lane quarter's rows of both 128-row
+//               blocks from the code ring into the tile's fp4 A slot in tensor memory (slot = team),
 //               waits for the tile's digits, then joins the named barrier of that slot. They also run
-//               the epilogue of a range: tcgen05.ld of the accumulator, the digit sum and scales,
-//               bf16 stores.
+//               the epilogue of a range (warp of team t: block t): tcgen05.ld of the accumulator, the
+//               digit sum and scales, bf16 stores.
 // Every wait on an mbarrier gives up after kWaitLimitNs (status LCQ_ERR_TIMEOUT); every warp still
 // reaches every named barrier of every tile, so no warp waits forever on one.
 #include "common.cuh"
@@ -46,13 +48,13 @@ constexpr int kF4MaxTokens = 16;
 constexpr int kF4TileCols = 512;           // codes per row and ring stage (128 bytes)
 constexpr int kF4SliceRows = 32;           // rows per code box
 constexpr int kF4MaxSlices = 8;            // rows per range <= 256: two 128-row MMA blocks
-constexpr int kF4ConvWarps = 8;            // one per (128-row block, TMEM lane quarter)
-constexpr int kF4Halves = 16 / kF4ConvWarps;   // K halves of a tile per converter warp
+constexpr int kF4ConvWarps = 8;            // two teams of one warp per TMEM lane quarter
 constexpr int kF4Conv0 = 2;                // first converter warp
 constexpr int kF4DigitWarp = kF4Conv0 + kF4ConvWarps;
 constexpr int kF4Threads = 32 * (kF4DigitWarp + 1);
 constexpr int kF4CodeStagesMax = 8;
 constexpr int kF4DigitStagesMax = 4;
+constexpr int kF4MinCodeStages = 5;       // code stages kept before digit stages are given up
 constexpr int kF4PreStages = 2;           // code stages loaded before the prep kernel has completed
 constexpr uint32_t kF4TmemCols = 512;
 // Tensor memory columns: accumulators of the two row blocks, block scales of A and B, the A ring
@@ -60,7 +62,8 @@ constexpr uint32_t kF4TmemCols = 512;
 constexpr uint32_t kF4ColD1 = 128, kF4ColSFA = 224, kF4ColSFB = 240, kF4ColA = 256;
 // Named barriers (0 is __syncthreads): A slot s full = 1 + s; accumulator read = 3.
 constexpr int kF4BarAFull = 1, kF4BarDFree = 3;
-constexpr int kF4BarAFullCount = 32 * (kF4ConvWarps + 1);
+constexpr int kF4TeamWarps = kF4ConvWarps / 2;   // converter warps per tile (two teams)
+constexpr int kF4BarAFullCount = 32 * (kF4TeamWarps + 1);
 constexpr int kF4BarDFreeCount = 32 * (8 + 1);   // the eight epilogue warps and the issuer
 constexpr size_t kF4SmemLimit = 227 * 1024;
 constexpr size_t kF4SmemMin = 120 * 1024;
@@ -149,6 +152,32 @@ __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, bool o
     if (ok && (threadIdx.x & 31) == 0) r = mbar_wait(bar, parity, status) ? 1u : 0u;
     r = __shfl_sync(0xffffffffu, r, 0);
     return r != 0;
+}
+
+// A warp waits on up to three mbarrier phases at once, one lane per barrier (a barrier pointer of
+// nullptr is skipped): an mbarrier check costs ~220 cycles even on a completed phase, so the three
+// checks share one latency. Returns the warp-uniform outcome; skips the waits once ok == false.
+__device__ __forceinline__ bool warp_wait3(uint64_t *b0, uint32_t p0, uint64_t *b1, uint32_t p1, uint64_t *b2,
+                                           uint32_t p2, bool ok, int32_t *status) {
+    if (!ok) return false;
+    const int lane = threadIdx.x & 31;
+    uint64_t *bar = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : nullptr;
+    const uint32_t par = lane == 0 ? p0 : lane == 1 ? p1 : p2;
+    bool done = bar == nullptr || mbar_test_wait(bar, par);
+    if (__all_sync(0xffffffffu, done)) return true;
+    uint64_t t0 = 0;
+    if (lane == 0) t0 = globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (!done) done = mbar_try_wait(bar, par);
+        if (__all_sync(0xffffffffu, done)) return true;
+        if ((it & 63u) == 0) {
+            int late = lane == 0 && globaltimer() - t0 > kWaitLimitNs;
+            if (__shfl_sync(0xffffffffu, late, 0)) {
+                if (lane == 0) set_status(status, LCQ_ERR_TIMEOUT);
+                return false;
+            }
+        }
+    }
 }
 
 // One lane of the (converged) warp returns true: warp-uniform issue of tcgen05 instructions.
@@ -337,7 +366,7 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
     uint8_t *cring = align_smem_1024(smem_raw);                                     // [cstages][code_bytes]
     uint8_t *dring = cring + static_cast<size_t>(p.cstages) * p.code_bytes;          // [dstages][act_bytes]
     uint64_t *cfull = reinterpret_cast<uint64_t *>(dring + static_cast<size_t>(p.dstages) * p.act_bytes);
-    uint64_t *cempty = cfull + kF4CodeStagesMax;   // 16 converter-warp arrivals: the codes were read
+    uint64_t *cempty = cfull + kF4CodeStagesMax;   // one arrival per warp of the tile's team: codes read
     uint64_t *dfull = cempty + kF4CodeStagesMax;
     uint64_t *dempty = dfull + kF4DigitStagesMax;  // the MMAs reading the digits completed
     uint64_t *aempty = dempty + kF4DigitStagesMax; // [2] the MMAs of the tile in A slot s completed
@@ -355,7 +384,7 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
         prefetch_tensormap(&tmB);
         for (int i = 0; i < p.cstages; ++i) {
             mbar_init(&cfull[i], 1);
-            mbar_init(&cempty[i], kF4ConvWarps);
+            mbar_init(&cempty[i], kF4TeamWarps);
         }
         for (int i = 0; i < p.dstages; ++i) {
             mbar_init(&dfull[i], 1);
@@ -485,62 +514,75 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
         __syncwarp();
     } else {
         // ---------------------------------------------------------------- converters and epilogue
+        // Two teams of four warps take alternate tiles (team = T mod 2 = the A slot), so that one team
+        // converts while the other's tile waits on its barrier; a warp converts its TMEM lane quarter's
+        // rows of both 128-row blocks. In the epilogue, team t reads block t.
         const int ci = warp - kF4Conv0;
         const int q = warp & 3;                       // TMEM lane quarter this warp may access
-        const int rb = (ci >> 2) & 1, kh0 = (ci >> 3) * kF4Halves;   // 128-row block, first K half
-        const int lrow = rb * 128 + q * 32 + lane;    // row within the range
+        const int team = ci >> 2;
         const uint32_t lane_base = tb + (static_cast<uint32_t>(32 * q) << 16);
-        const uint32_t a_base = lane_base + kF4ColA + static_cast<uint32_t>(rb * 64 + kh0 * 32);
+        const uint32_t a_base = lane_base + kF4ColA;
         bool ok = true;                               // false after a failed wait: no more waits
-        int T = 0, cs = 0, ds = 0, slot = 0;
-        // stage phases; aempty parity for tiles T >= 2 is ((T >> 1) + 1) & 1: 0 for T = 2, 3, then
-        // flipping after every second tile (aph flips after each use of slot 1)
-        uint32_t cph = 0, dph = 0, aph = 1;
-        const uint8_t *crow = cring + lrow * 128;
-        const int sw = lrow & 7;
+        int T = 0, cs = 0, ds = 0;
+        uint32_t cph = 0, dph = 0;
+        const int lrow0 = q * 32 + lane;              // row of block 0 within the range; block 1: + 128
+        const uint8_t *crow = cring + lrow0 * 128;
+        const int sw = lane & 7;                      // 128-byte swizzle phase of both rows
         for (int ri = 0; ri < my_ranges; ++ri) {
             int s0, s1;
             f4_range(static_cast<int>(blockIdx.x) + ri * static_cast<int>(gridDim.x), p.slices, p.ranges, s0, s1);
-            const bool live = (rb * 4 + q) < (s1 - s0);   // this warp's 32 rows belong to the range
+            // this warp's 32 rows of block rb belong to the range
+            const bool live0 = q < (s1 - s0), live1 = (4 + q) < (s1 - s0);
             for (int k = 0; k < p.tiles; ++k, ++T) {
-                ok = warp_wait(&cfull[cs], cph, ok, p.status);
-                uint32_t f[kF4Halves][32];
-                if (ok && live) {
+                if ((T & 1) == team) {
+                    const int slot = T & 1;
+                    ok = warp_wait(&cfull[cs], cph, ok, p.status);
+                    uint4 v[2][8];
+                    if (ok) {
 #pragma unroll
-                    for (int h = 0; h < kF4Halves; ++h)
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            const int chunk = 4 * (kh0 + h) + c;
-                            const uint4 v = *reinterpret_cast<const uint4 *>(crow + ((chunk ^ sw) << 4));
-                            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                            for (int u = 0; u < 4; ++u) {
-                                f[h][8 * c + 2 * u] = w[u] & 0x33333333u;
-                                f[h][8 * c + 2 * u + 1] = (w[u] >> 2) & 0x33333333u;
-                            }
+                        for (int c = 0; c < 8; ++c) {
+                            if (live0) v[0][c] = *reinterpret_cast<const uint4 *>(crow + ((c ^ sw) << 4));
+                            if (live1) v[1][c] = *reinterpret_cast<const uint4 *>(crow + 128 * 128 + ((c ^ sw) << 4));
                         }
-                }
-                // the code stage is free once every converter warp has read its part
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&cempty[cs]);
-                if (T >= 2) ok = warp_wait(&aempty[slot], aph, ok, p.status);
-                tc_fence_after();
-                if (ok && live) {
+                    }
+                    // the code stage is free once every converter warp of the team has read its part
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&cempty[cs]);
+                    // the slot is free once the MMAs of tile T - 2 completed (aempty phase (T / 2 + 1) mod 2),
+                    // and the issuer reads the digits once the converters have seen them land
+                    ok = warp_wait3(T >= 2 ? &aempty[slot] : nullptr, static_cast<uint32_t>(((T >> 1) + 1) & 1),
+                                    &dfull[ds], dph, nullptr, 0u, ok, p.status);
+                    tc_fence_after();
 #pragma unroll
-                    for (int h = 0; h < kF4Halves; ++h) tmem_st32(a_base + static_cast<uint32_t>(slot * 128 + h * 32), f[h]);
-                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    for (int rb = 0; rb < 2; ++rb) {
+                        if (ok && (rb ? live1 : live0)) {
+                            uint32_t f[2][32];
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                const uint32_t w[4] = {v[rb][c].x, v[rb][c].y, v[rb][c].z, v[rb][c].w};
+#pragma unroll
+                                for (int u = 0; u < 4; ++u) {
+                                    f[c >> 2][8 * (c & 3) + 2 * u] = w[u] & 0x33333333u;
+                                    f[c >> 2][8 * (c & 3) + 2 * u + 1] = (w[u] >> 2) & 0x33333333u;
+                                }
+                            }
+#pragma unroll
+                            for (int h = 0; h < 2; ++h)
+                                tmem_st32(a_base + static_cast<uint32_t>(slot * 128 + rb * 64 + h * 32), f[h]);
+                        }
+                    }
+                    if (ok && (live0 || live1)) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    tc_fence_before();
+                    named_sync(kF4BarAFull + slot, kF4BarAFullCount);
                 }
-                // the issuer reads the digits once the converters have seen them land
-                ok = warp_wait(&dfull[ds], dph, ok, p.status);
-                tc_fence_before();
-                named_sync(kF4BarAFull + slot, kF4BarAFullCount);
-                if (slot) aph ^= 1;
-                slot ^= 1;
-                if (++cs == p.cstages) { cs = 0; cph ^= 1; crow = cring + lrow * 128; } else { crow += p.code_bytes; }
+                if (++cs == p.cstages) { cs = 0; cph ^= 1; crow = cring + lrow0 * 128; } else { crow += p.code_bytes; }
                 if (++ds == p.dstages) { ds = 0; dph ^= 1; }
             }
-            if (kh0 == 0) {
+            {
                 // ------------------------------------------------------------ epilogue of the range
+                const int rb = team;
+                const bool live = rb ? live1 : live0;
+                const int lrow = rb * 128 + lrow0;
                 if (ri == 0) asm volatile("griddepcontrol.wait;" ::: "memory");   // scale and corr of the prep kernel
                 ok = warp_wait(accfull, ri & 1, ok, p.status);
                 tc_fence_after();
@@ -616,8 +658,8 @@ bool f4_plan(int64_t N, int64_t m, int64_t n, int num_sms, F4Plan &pl) {
     const int max_slices = (pl.slices + pl.ranges - 1) / pl.ranges;
     pl.code_bytes = static_cast<uint32_t>(max_slices) * 4096u;
     pl.act_bytes = static_cast<uint32_t>(pl.NB) * 256u;
-    // as many code stages as fit next to up to four digit stages (at least 6 code stages while there
-    // are more than two digit stages)
+    // as many code stages as fit next to up to four digit stages (at least kF4MinCodeStages code
+    // stages while there are more than two digit stages)
     const size_t fixed = 1024 + 1024;   // barriers and the TMEM slot; alignment slack
     auto code_stages = [&](int d) {
         const size_t rest = kF4SmemLimit - fixed - static_cast<size_t>(d) * pl.act_bytes;
@@ -626,7 +668,7 @@ bool f4_plan(int64_t N, int64_t m, int64_t n, int num_sms, F4Plan &pl) {
     };
     pl.dstages = kF4DigitStagesMax;
     pl.cstages = code_stages(pl.dstages);
-    while (pl.cstages < 6 && pl.dstages > 2) pl.cstages = code_stages(--pl.dstages);
+    while (pl.cstages < kF4MinCodeStages && pl.dstages > 2) pl.cstages = code_stages(--pl.dstages);
     if (pl.cstages < 2) return false;
     pl.smem = static_cast<size_t>(pl.cstages) * pl.code_bytes + static_cast<size_t>(pl.dstages) * pl.act_bytes + fixed;
     // at least half the shared memory, so one CTA per SM owns all 512 tensor-memory columns

@@ -4,6 +4,8 @@
 //   Y[t][r] = sum_c X'[t][c] z[r][c] + sum_g X_g[t] . b,     X'_g = X_g A  (per group of d columns)
 //
 // so the integer codes themselves are the weight operand and A acts on the few activation rows.
+// With n % 64 == 0 and n <= 32768, one token takes the dp2a kernel below and 2-16 tokens the tcgen05
+// kernel (gemv_fp4.cu); the mma.sync kernels below take every other shape.
 //
 // prep kernel  (256 16-column blocks per CTA): X' in bf16, written in the column order and scale
 //              the main kernel's register fragments expect (tile-major for the tma variant), and
@@ -612,7 +614,7 @@ packed_gemv_tma_kernel(const __grid_constant__ CUtensorMap tmC, const GemvTmaPar
 // Launched with programmatic dependent launch: the code stream starts while the previous kernel in
 // the stream finishes; the consumers wait for it (griddepcontrol.wait) before reading X.
 
-constexpr int kFp4MinTokens = 8;          // the tcgen05 fp4 kernel takes more tokens than this
+constexpr int kFp4MinTokens = 1;          // the tcgen05 fp4 kernel takes more tokens than this
 constexpr int kDpMaxTokens = 1;            // two tokens measured slower than the tensor-core kernel
 constexpr int kDpWarps = 16;               // consumer warps (a multiple of 8)
 constexpr int64_t kDpMaxN = 32768;         // integer row sums stay below 2^31
@@ -1311,8 +1313,9 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
     const int64_t npad = gemv_npad(a.n), nprep = gemv_nprep(a.n);
     trace_begin(LCQ_K_GEMV, st);
     if (a.N > kFp4MinTokens) {
-        // 9-16 tokens, n % 64 == 0: codes as fp4 tensor-core operands in tensor memory (tcgen05); at
-        // 2-8 tokens the mma.sync kernel below measured faster (18.9 against 20.2 us on the 70B gate)
+        // 2-16 tokens, n % 64 == 0, n <= 32768: codes as fp4 tensor-core operands in tensor memory
+        // (tcgen05); faster than the mma.sync kernel below at every token count from 2 (70B gate:
+        // 17.2-18.0 against 18.4-18.6 us at 2-8 tokens), which keeps the other shapes
         cudaError_t e = cudaSuccess;
         if (launch_packed_gemv_fp4(a, d, num_sms, st, e)) {
             if (e != cudaSuccess) return e;

@@ -2,6 +2,7 @@
 exact same bits, reading results back, and the comparison rules of the parity bar."""
 import numpy as np
 
+import oracle
 from paper_2606_10531_gb300 import workloads as wl
 
 
@@ -41,6 +42,26 @@ def max_rel(x, ref):
         return 0.0
     den = np.max(np.abs(ref))
     return float(np.max(np.abs(x - ref)) / (den if den > 0 else 1.0))
+
+
+def digit_product_bound(Xf, Z, A, b, d, ref, levels=8191, sigmas=7.0):
+    """Elementwise error bound of the packed product on its integer-digit path (2-16 tokens): each
+    element of X' = X_g A is rounded per token to a multiple of D_t = max|X'_t| / levels, off by at
+    most D_t / 2 and independently of the others, so output (t, r) is off by the code-weighted sum of
+    these roundings (standard deviation D_t sqrt(sum_c z_rc^2 / 12)), bounded here at `sigmas`
+    standard deviations, plus the bf16 rounding of the output (at most 2^-9 of it, doubled for the
+    fp32 sums) and a floor of 1e-7 max|ref| for outputs near zero."""
+    Xp, _ = oracle.activation_transform(Xf, A, b, d)
+    D = np.abs(Xp).max(axis=1) / levels
+    spread = np.sqrt((np.asarray(Z, np.float64) ** 2).sum(axis=1) / 12.0)
+    ref = np.asarray(ref, np.float64)
+    return sigmas * D[:, None] * spread[None, :] + 2.0 ** -8 * np.abs(ref) + 1e-7 * np.abs(ref).max()
+
+
+def within(x, ref, bound):
+    """Largest |x - ref| / bound over the elements (the check passes at <= 1)."""
+    x = np.asarray(x, np.float64)
+    return float(np.max(np.abs(x - np.asarray(ref, np.float64)) / bound))
 
 
 def config_A(d, rng):

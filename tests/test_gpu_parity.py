@@ -10,8 +10,8 @@ import pytest
 import oracle
 import paper_2606_10531_gb300 as lcq
 from paper_2606_10531_gb300 import workloads as wl
-from tests.gpu_util import (TOL_BF16, TOL_DECODE_F32, config_A, config_b, dev, dev_bf16, empty_bf16, host_bf16,
-                            max_rel)
+from tests.gpu_util import (TOL_BF16, TOL_DECODE_F32, config_A, config_b, dev, dev_bf16, digit_product_bound, empty_bf16,
+                            host_bf16, max_rel, within)
 
 pytestmark = pytest.mark.gpu
 
@@ -333,12 +333,13 @@ def test_gemm_packed2b_matches_oracle(N, m, n, d):
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
 
 
-# One token with n % 64 == 0 takes the integer (dp2a) kernel: activations as int16 with one scale
-# per token (a bound on max|X'|), exact int32 sums. Its only errors are the int16 rounding (at most
-# 2^-16 of the bound per element) and the bf16 output rounding (2^-9 relative), so it is held to a
-# tighter bound than the bf16 parity bar, on heavy-tailed activations (1% of the columns x50); two to
-# four tokens (tensor-core kernel) keep the bf16 bar. (300, 28672) puts 56 activation tiles in
-# shared memory next to the code ring.
+# With n % 64 == 0 (n <= 32768), one token takes the integer (dp2a) kernel: activations as int16 with
+# one scale per token (a bound on max|X'|), exact int32 sums. Its only errors are the int16 rounding
+# (at most 2^-16 of the bound per element) and the bf16 output rounding (2^-9 relative), so it is held
+# to a tighter bound than the bf16 parity bar, on heavy-tailed activations (1% of the columns x50).
+# Two to four tokens take the tcgen05 kernel (exact integer digits, below), held to the elementwise
+# bound of its rounding (digit_product_bound). (300, 28672) puts 56 activation tiles in shared memory
+# next to the code ring.
 TOL_DP = 4e-3
 
 
@@ -356,8 +357,27 @@ def test_gemm_packed2b_few_tokens_heavy_tailed(N, m, n, d):
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
     lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert lcq.lcq_device_status(ws) == 0
-    tol = TOL_DP if N == 1 else TOL_BF16
-    assert max_rel(host_bf16(Y), ref) <= tol
+    if N == 1:
+        assert max_rel(host_bf16(Y), ref) <= TOL_DP
+    else:
+        assert within(host_bf16(Y), ref, digit_product_bound(wl.bf16_to_f32(Xb), Z, A, b, d, ref)) <= 1.0
+
+
+# Shapes the integer kernels do not take (n % 64 != 0, or n > 32768) run the mma.sync kernel: X' in
+# bf16, fp32 accumulation, the bf16 parity bar. n = 32832 streams its codes through the TMA ring.
+@pytest.mark.parametrize("N", [2, 5, 8])
+@pytest.mark.parametrize("m,n,d", [(300, 200, 4), (129, 1000, 8), (64, 32832, 8)])
+def test_gemm_packed2b_mma_sync_shapes(N, m, n, d):
+    rng = np.random.default_rng(13 * N + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    Xb = wl.bf16_bits(rng.normal(0, 1, (N, n)).astype(np.float32))
+    ref = oracle.gemm_packed2b(wl.bf16_to_f32(Xb), oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
+    lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_device_status(ws) == 0
+    assert max_rel(host_bf16(Y), ref) <= TOL_BF16
 
 
 def test_gemm_packed2b_one_token_zero_activations():
@@ -403,11 +423,12 @@ def test_gemm_packed2b_two_tokens_independent_scales():
         lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
         assert lcq.lcq_device_status(ws) == 0
         got = host_bf16(Y)
-        assert max_rel(got[0], ref[0]) <= TOL_BF16
+        bound = digit_product_bound(wl.bf16_to_f32(Xb), Z, A, b, d, ref)
+        assert within(got[0], ref[0], bound[0]) <= 1.0
         if case == "zero":
             assert np.all(got[1] == 0.0)
         else:
-            assert max_rel(got[1], ref[1]) <= TOL_BF16
+            assert within(got[1], ref[1], bound[1]) <= 1.0
 
 
 # ----------------------------------------------------------------------------- failure detection
@@ -516,13 +537,14 @@ def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
 
 
-# 9-16 tokens with n % 64 == 0 take the tcgen05 kernel (kind::mxf4): the codes are fp4 operands in
+# 2-16 tokens with n % 64 == 0 take the tcgen05 kernel (kind::mxf4): the codes are fp4 operands in
 # tensor memory and the activations exact integer digits, q = rint(X' 8191 / max|X'_t|) per token, so
 # its only errors are that rounding (at most 2^-14 of max|X'_t| per element) and the bf16 output
-# rounding: it is held to the tighter bound of the one-token kernel, on heavy-tailed activations.
+# rounding: each output is held to the bound those two give (digit_product_bound), on heavy-tailed
+# activations.
 # The shapes cover ragged rows (not a multiple of 32 or 128), a partial last 512-column tile, ranges
 # of one to eight 32-row slices, and more rows than one wave of CTAs holds (several ranges per CTA).
-@pytest.mark.parametrize("N", [9, 12, 16])
+@pytest.mark.parametrize("N", [2, 5, 8, 9, 12, 16])
 @pytest.mark.parametrize("m,n,d", [(1000, 4096, 8), (300, 8192, 4), (77, 576, 8), (129, 1088, 4), (2500, 512, 8),
                                    (40000, 64, 8)])
 def test_gemm_packed2b_tcgen05_heavy_tailed(N, m, n, d):
@@ -537,7 +559,7 @@ def test_gemm_packed2b_tcgen05_heavy_tailed(N, m, n, d):
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, N, m, n, d)
     lcq.lcq_gemm_packed2b(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert lcq.lcq_device_status(ws) == 0
-    assert max_rel(host_bf16(Y), ref) <= TOL_DP
+    assert within(host_bf16(Y), ref, digit_product_bound(wl.bf16_to_f32(Xb), Z, A, b, d, ref)) <= 1.0
 
 
 def test_gemm_packed2b_tcgen05_zero_token_and_repeat():
@@ -559,7 +581,7 @@ def test_gemm_packed2b_tcgen05_zero_token_and_repeat():
     lcq.lcq_gemm_packed2b(Xd, Pd, n, d, Ad, bd, Y2, ws)
     assert torch.equal(Y1, Y2)
     assert float(Y1[3].float().abs().max()) == 0.0
-    assert max_rel(host_bf16(Y1), ref) <= TOL_DP
+    assert within(host_bf16(Y1), ref, digit_product_bound(wl.bf16_to_f32(Xb), Z, A, b, d, ref)) <= 1.0
 
 
 # ----------------------------------------------------------------------------- activation transform
