@@ -44,6 +44,7 @@ namespace {
 
 constexpr int kF4Digits = 5;               // balanced base-8 digits per activation
 constexpr float kF4QMax = 8191.0f;         // |q| bound; 5 digits in [-4, 3] cover [-18724, 14043]
+constexpr int kF4DigitBias = 18724;        // 4 (1 + 8 + 64 + 512 + 4096): q + bias has octal digits d_j + 4
 constexpr int kF4MaxTokens = 16;
 constexpr int kF4TileCols = 512;           // codes per row and ring stage (128 bytes)
 constexpr int kF4SliceRows = 32;           // rows per code box
@@ -55,7 +56,7 @@ constexpr int kF4Threads = 32 * (kF4DigitWarp + 1);
 constexpr int kF4CodeStagesMax = 8;
 constexpr int kF4DigitStagesMax = 4;
 constexpr int kF4MinCodeStages = 5;       // code stages kept before digit stages are given up
-constexpr int kF4PreStages = 2;           // code stages loaded before the prep kernel has completed
+constexpr int kF4PreStages = 4;           // code stages loaded before the prep kernel has completed
 constexpr uint32_t kF4TmemCols = 512;
 // Tensor memory columns: accumulators of the two row blocks, block scales of A and B, the A ring
 // (slot s, block rb at kF4ColA + 128 s + 64 rb: 8 columns per K step of 64 fp4 elements).
@@ -321,11 +322,13 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
     for (int gg = 0; gg < kF4PrepGroups; ++gg) {
         const int64_t gi = threadIdx.x + static_cast<int64_t>(gg) * kF4PrepThreads;
         if (gi >= ngroups) continue;
-        int q[16];
+        // q + 4 (1 + 8 + 64 + 512 + 4096) lies in [10533, 26915]: its five octal digits, each minus 4,
+        // are the balanced digits of q (the representation is unique), so digit j is octal field j
+        uint32_t u[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const float v = fminf(fmaxf(xv[gg][i] * inv, -kF4QMax), kF4QMax);   // NaN -> one of the bounds
-            q[i] = __float2int_rn(v);
+            u[i] = static_cast<uint32_t>(__float2int_rn(v) + kF4DigitBias);
         }
         const int64_t tile = gi / (kF4TileCols / 16);
         const int slot = static_cast<int>(gi % (kF4TileCols / 16));
@@ -334,9 +337,8 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
             uint32_t lo = 0, hi = 0;   // K positions 0..7 and 8..15 of the group
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-                const int dj = ((q[i] + 4) & 7) - 4;          // balanced digit in [-4, 3]
-                q[i] = (q[i] - dj) >> 3;                      // exact: q - d is a multiple of 8
-                const uint32_t nib = (kE2m1Digits >> (4 * (dj + 4))) & 0xFu;
+                // e2m1 pattern of digit field - 4, from the table indexed by the field
+                const uint32_t nib = (kE2m1Digits >> (((u[i] >> (3 * j)) & 7u) << 2)) & 0xFu;
                 // column i = 2 u + p sits at K position 8 p + u
                 const int pos = 8 * (i & 1) + (i >> 1);
                 if (pos < 8) lo |= nib << (4 * pos);
@@ -432,9 +434,10 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
                 // one box of code_bytes / 128 rows from the range's first row (rows past the range or
                 // past m come along unused: zero-filled past m)
                 for (int k = 0; k < p.tiles; ++k, ++T) {
-                    // only the first stages go out before the prep kernel completes: a full ring of
-                    // code copies from every SM would queue the prep kernel's own memory traffic
-                    // behind it (measured: its results arrived 2-4 us later)
+                    // only the first stages go out before the prep kernel completes: code copies
+                    // from every SM queue the prep kernel's own memory traffic behind them (with eight
+                    // stages its results arrived 2-4 us later; of two to five stages, four measured
+                    // fastest, 0.7 us ahead of two)
                     if (T == kF4PreStages) asm volatile("griddepcontrol.wait;" ::: "memory");
                     if (T >= p.cstages && !mbar_wait_backoff(&cempty[cs], cph ^ 1, p.status)) { ok = false; break; }
                     mbar_arrive_expect_tx(&cfull[cs], p.code_bytes);
@@ -584,6 +587,13 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
                 const bool live = rb ? live1 : live0;
                 const int lrow = rb * 128 + lrow0;
                 if (ri == 0) asm volatile("griddepcontrol.wait;" ::: "memory");   // scale and corr of the prep kernel
+                // the token scales and bias terms are read while the range's last MMAs run
+                float sc[kF4MaxTokens], co[kF4MaxTokens];
+#pragma unroll
+                for (int t = 0; t < kF4MaxTokens; ++t) {
+                    sc[t] = t < p.ntok ? __ldg(p.scale + t) : 0.0f;
+                    co[t] = t < p.ntok ? __ldg(p.corr + t) : 0.0f;
+                }
                 ok = warp_wait(accfull, ri & 1, ok, p.status);
                 tc_fence_after();
                 // column c of the accumulator is digit c % 5 of token c / 5: sum_j 8^j acc_j per token,
@@ -615,7 +625,7 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
 #pragma unroll
                     for (int t = 0; t < kF4MaxTokens; ++t) {
                         if (t < p.ntok) {
-                            const float yt = fmaf(y[t], __ldg(p.scale + t), __ldg(p.corr + t));
+                            const float yt = fmaf(y[t], sc[t], co[t]);
                             const __nv_bfloat16 h = __float2bfloat16_rn(yt);
                             p.Y[static_cast<int64_t>(t) * p.m + grow] = *reinterpret_cast<const uint16_t *>(&h);
                         }
