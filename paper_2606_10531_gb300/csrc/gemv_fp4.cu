@@ -266,15 +266,18 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
     const int64_t t = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t ngroups = static_cast<int64_t>(tiles) * (kF4TileCols / 16);
-    // this thread's activations first (they are the long wait), then A and b through shared memory
+    // A and b are weights like the codes: read before the wait. This kernel is itself launched as a
+    // programmatic dependent of the previous kernel in the stream (it may become resident while that
+    // one runs): X, and the workspace this kernel writes, are touched only after that kernel completed.
+    if (threadIdx.x < D * D) sA[threadIdx.x] = __ldg(A + threadIdx.x);
+    if (threadIdx.x < D) sb[threadIdx.x] = __ldg(b + threadIdx.x);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     float xv[kF4PrepGroups][16];
 #pragma unroll
     for (int gg = 0; gg < kF4PrepGroups; ++gg) {
         const int64_t gi = threadIdx.x + static_cast<int64_t>(gg) * kF4PrepThreads;
         if (gi < ngroups) f4_load16<D, F32IN>(Xv, n, t, gi * 16, xv[gg]);
     }
-    if (threadIdx.x < D * D) sA[threadIdx.x] = __ldg(A + threadIdx.x);
-    if (threadIdx.x < D) sb[threadIdx.x] = __ldg(b + threadIdx.x);
     __syncthreads();
 
     float amax = 0.0f, r = 0.0f;
@@ -418,6 +421,9 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // the next kernel in the stream may start launching (the next call's prep waits for this kernel's
+    // completion before it reads or writes anything)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     // Tiles are numbered T = 0, 1, .. over this CTA's ranges in order; each role keeps its ring
     // stages, phases and A slot (T mod 2) as running counters, and computes the rows of a range once
@@ -735,12 +741,25 @@ bool launch_packed_gemv_fp4(const PackedGemvArgs &a, int d, int num_sms, cudaStr
                             float *);
     PrepFn prep = a.Xf ? (d == 4 ? fp4_prep_kernel<4, true> : fp4_prep_kernel<8, true>)
                        : (d == 4 ? fp4_prep_kernel<4, false> : fp4_prep_kernel<8, false>);
-    prep<<<static_cast<unsigned>(a.N), kF4PrepThreads, 0, st>>>(
-        a.Xf ? static_cast<const void *>(a.Xf) : static_cast<const void *>(a.X), a.n, pl.tiles,
-        static_cast<int>(a.N), pl.NB, a.A, a.b, dig, scale, corr);
-    count_launch();
-    err = cudaGetLastError();
-    if (err != cudaSuccess) return true;
+    {
+        // a programmatic dependent of the previous kernel in the stream: it may become resident on the
+        // SMs this kernel's grid leaves free while that kernel still runs, and waits for it on the device
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(a.N));
+        cfg.blockDim = dim3(kF4PrepThreads);
+        cfg.dynamicSmemBytes = 0;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        err = cudaLaunchKernelEx(&cfg, prep, a.Xf ? static_cast<const void *>(a.Xf) : static_cast<const void *>(a.X),
+                                 a.n, pl.tiles, static_cast<int>(a.N), pl.NB, a.A, a.b, dig, scale, corr);
+        count_launch();
+        if (err == cudaSuccess) err = cudaGetLastError();
+        if (err != cudaSuccess) return true;
+    }
 
     F4Params p;
     p.m = a.m;
