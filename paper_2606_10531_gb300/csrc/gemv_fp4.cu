@@ -56,7 +56,7 @@ constexpr int kF4Threads = 32 * (kF4DigitWarp + 1);
 constexpr int kF4CodeStagesMax = 8;
 constexpr int kF4DigitStagesMax = 4;
 constexpr int kF4MinCodeStages = 5;       // code stages kept before digit stages are given up
-constexpr int kF4PreStages = 4;           // code stages loaded before the prep kernel has completed
+constexpr int kF4PreStages = 8;           // code tiles requested before the prep kernel has completed
 constexpr uint32_t kF4TmemCols = 512;
 // Tensor memory columns: accumulators of the two row blocks, block scales of A and B, the A ring
 // (slot s, block rb at kF4ColA + 128 s + 64 rb: 8 columns per K step of 64 fp4 elements).
@@ -153,32 +153,6 @@ __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, bool o
     if (ok && (threadIdx.x & 31) == 0) r = mbar_wait(bar, parity, status) ? 1u : 0u;
     r = __shfl_sync(0xffffffffu, r, 0);
     return r != 0;
-}
-
-// A warp waits on up to three mbarrier phases at once, one lane per barrier (a barrier pointer of
-// nullptr is skipped): an mbarrier check costs ~220 cycles even on a completed phase, so the three
-// checks share one latency. Returns the warp-uniform outcome; skips the waits once ok == false.
-__device__ __forceinline__ bool warp_wait3(uint64_t *b0, uint32_t p0, uint64_t *b1, uint32_t p1, uint64_t *b2,
-                                           uint32_t p2, bool ok, int32_t *status) {
-    if (!ok) return false;
-    const int lane = threadIdx.x & 31;
-    uint64_t *bar = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : nullptr;
-    const uint32_t par = lane == 0 ? p0 : lane == 1 ? p1 : p2;
-    bool done = bar == nullptr || mbar_test_wait(bar, par);
-    if (__all_sync(0xffffffffu, done)) return true;
-    uint64_t t0 = 0;
-    if (lane == 0) t0 = globaltimer();
-    for (uint32_t it = 1;; ++it) {
-        if (!done) done = mbar_try_wait(bar, par);
-        if (__all_sync(0xffffffffu, done)) return true;
-        if ((it & 63u) == 0) {
-            int late = lane == 0 && globaltimer() - t0 > kWaitLimitNs;
-            if (__shfl_sync(0xffffffffu, late, 0)) {
-                if (lane == 0) set_status(status, LCQ_ERR_TIMEOUT);
-                return false;
-            }
-        }
-    }
 }
 
 // One lane of the (converged) warp returns true: warp-uniform issue of tcgen05 instructions.
@@ -440,10 +414,11 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
                 // one box of code_bytes / 128 rows from the range's first row (rows past the range or
                 // past m come along unused: zero-filled past m)
                 for (int k = 0; k < p.tiles; ++k, ++T) {
-                    // only the first stages go out before the prep kernel completes: code copies
-                    // from every SM queue the prep kernel's own memory traffic behind them (with eight
-                    // stages its results arrived 2-4 us later; of two to five stages, four measured
-                    // fastest, 0.7 us ahead of two)
+                    // only the first tiles go out before the prep kernel completes: code copies from
+                    // every SM queue the prep kernel's own memory traffic behind them. With the prep
+                    // resident early (it overlaps the previous kernel) and the first two tiles stored
+                    // before their digits are checked, eight tiles measured fastest (seven to ten alike,
+                    // 0.9 us ahead of four)
                     if (T == kF4PreStages) asm volatile("griddepcontrol.wait;" ::: "memory");
                     if (T >= p.cstages && !mbar_wait_backoff(&cempty[cs], cph ^ 1, p.status)) { ok = false; break; }
                     mbar_arrive_expect_tx(&cfull[cs], p.code_bytes);
@@ -557,10 +532,10 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
                     // the code stage is free once every converter warp of the team has read its part
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&cempty[cs]);
-                    // the slot is free once the MMAs of tile T - 2 completed (aempty phase (T / 2 + 1) mod 2),
-                    // and the issuer reads the digits once the converters have seen them land
-                    ok = warp_wait3(T >= 2 ? &aempty[slot] : nullptr, static_cast<uint32_t>(((T >> 1) + 1) & 1),
-                                    &dfull[ds], dph, nullptr, 0u, ok, p.status);
+                    // the slot is free once the MMAs of tile T - 2 completed (aempty phase (T / 2 + 1) mod 2);
+                    // the digits are checked only before the barrier, so the first two tiles leave the
+                    // code ring while the prep kernel still runs
+                    if (T >= 2) ok = warp_wait(&aempty[slot], static_cast<uint32_t>(((T >> 1) + 1) & 1), ok, p.status);
                     tc_fence_after();
 #pragma unroll
                     for (int rb = 0; rb < 2; ++rb) {
@@ -581,6 +556,8 @@ packed_gemv_fp4_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_con
                         }
                     }
                     if (ok && (live0 || live1)) asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    // the issuer reads the digits once the converters have seen them land
+                    ok = warp_wait(&dfull[ds], dph, ok, p.status);
                     tc_fence_before();
                     named_sync(kF4BarAFull + slot, kF4BarAFullCount);
                 }
