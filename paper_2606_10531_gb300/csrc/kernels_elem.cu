@@ -19,14 +19,15 @@ namespace lcq {
 constexpr int kComputeWarps = 11;                                // + 1 producer = 12 warps, 3 per SM sub-partition
 constexpr int kPerThread = 16;                                   // weights per compute thread per stage
 constexpr int kChunk = 32 * kComputeWarps * kPerThread;          // fp32 weights per stage (22 KB)
-constexpr int kStages = 6;                                       // 132 KB ring
+constexpr int kStreamStages = 8;                                 // 176 KB ring (single-matrix kernels)
+constexpr int kBatchStages = 6;                                  // 132 KB ring (batched encode)
 constexpr int kStreamThreads = 32 * (1 + kComputeWarps);
 constexpr float kRoundMagic = 12582912.0f;                       // 1.5 * 2^23
 
 struct StreamSmem {
-    float buf[kStages][kChunk];
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
+    float buf[kStreamStages][kChunk];
+    uint64_t full[kStreamStages];
+    uint64_t empty[kStreamStages];
     float Ainv[64];
     float A[64];
     float M[64];        // A^T A (encode MSE)
@@ -46,8 +47,8 @@ __device__ void stream_producer(StreamSmem &s, const float *src, int64_t total, 
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
     int i = 0;
     for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++i) {
-        const int st = i % kStages;
-        const uint32_t ph = (i / kStages) & 1;
+        const int st = i % kStreamStages;
+        const uint32_t ph = (i / kStreamStages) & 1;
         if (!mbar_wait(&s.empty[st], ph ^ 1, status)) return;
         const int64_t base = c * kChunk;
         const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
@@ -262,7 +263,7 @@ encode_kernel(EncodeArgs a) {
     const int64_t total = a.m * a.n;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
+        for (int i = 0; i < kStreamStages; ++i) {
             mbar_init(&s.full[i], 1);
             mbar_init(&s.empty[i], kComputeWarps);
         }
@@ -293,8 +294,8 @@ encode_kernel(EncodeArgs a) {
     float sq = 0.0f;
     int i = 0;
     for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++i) {
-        const int st = i % kStages;
-        if (!mbar_wait(&s.full[st], (i / kStages) & 1, a.status)) break;
+        const int st = i % kStreamStages;
+        if (!mbar_wait(&s.full[st], (i / kStreamStages) & 1, a.status)) break;
         const int64_t base = c * kChunk;
         const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
         encode_chunk<D, kMse>(s.buf[st], base, cnt, t, hswap, Ai2, qc, c2, a.packed, a.codes,
@@ -324,9 +325,9 @@ struct InvSlot {
 };
 
 struct EncBatchSmem {
-    float buf[kStages][kChunk];
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
+    float buf[kBatchStages][kChunk];
+    uint64_t full[kBatchStages];
+    uint64_t empty[kBatchStages];
     InvSlot inv[kEncodeBatchMax];
 };
 
@@ -357,8 +358,8 @@ __device__ __noinline__ void encode_batch_matrix(EncBatchSmem &s, const EncodeBa
         uint8_t *const codes = a.item[j].codes;
         float *const latent = kLatent ? a.item[j].latent : nullptr;
         for (int64_t c = first; c < chunk1 && ok; c += G, ++it) {
-            const int st = it % kStages;
-            if (!mbar_wait(&s.full[st], (it / kStages) & 1, a.status)) { ok = false; break; }
+            const int st = it % kBatchStages;
+            if (!mbar_wait(&s.full[st], (it / kBatchStages) & 1, a.status)) { ok = false; break; }
             const int64_t base = (c - chunk0) * kChunk;
             const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
             encode_chunk<D, false>(s.buf[st], base, cnt, t, hswap, Ai2, qc, c2, packed, codes, latent, sq);
@@ -376,7 +377,7 @@ encode_batch_kernel(const __grid_constant__ EncodeBatchArgs a) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
+        for (int i = 0; i < kBatchStages; ++i) {
             mbar_init(&s.full[i], 1);
             mbar_init(&s.empty[i], kComputeWarps);
         }
@@ -402,8 +403,8 @@ encode_batch_kernel(const __grid_constant__ EncodeBatchArgs a) {
                     W = a.item[j].W;
                     next0 = j + 1 < a.count ? a.item[j + 1].chunk0 : a.total_chunks;
                 }
-                const int st = it % kStages;
-                if (!mbar_wait(&s.empty[st], ((it / kStages) & 1) ^ 1, a.status)) return;
+                const int st = it % kBatchStages;
+                if (!mbar_wait(&s.empty[st], ((it / kBatchStages) & 1) ^ 1, a.status)) return;
                 const int64_t base = (c - chunk0) * kChunk;
                 const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
                 const uint32_t bytes = static_cast<uint32_t>(cnt * 4);
@@ -436,7 +437,7 @@ quant_decode_kernel(QuantDecodeArgs a) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t total = a.m * a.n;
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
+        for (int i = 0; i < kStreamStages; ++i) {
             mbar_init(&s.full[i], 1);
             mbar_init(&s.empty[i], kComputeWarps);
         }
@@ -458,8 +459,8 @@ quant_decode_kernel(QuantDecodeArgs a) {
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
     int i = 0;
     for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++i) {
-        const int st = i % kStages;
-        if (!mbar_wait(&s.full[st], (i / kStages) & 1, a.status)) break;
+        const int st = i % kStreamStages;
+        if (!mbar_wait(&s.full[st], (i / kStreamStages) & 1, a.status)) break;
         const int64_t base = c * kChunk;
         const int64_t cnt = (total - base < kChunk) ? (total - base) : kChunk;
         const int64_t off = static_cast<int64_t>(t) * kPerThread;
@@ -721,7 +722,7 @@ cudaError_t launch_wait_timeout_selftest(int32_t *status, cudaStream_t st) {
 
 static int stream_grid(int64_t total, int num_sms) {
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
-    int64_t g = num_sms;   // persistent: one CTA (a 144 KB ring) per SM
+    int64_t g = num_sms;   // persistent: one CTA (a 176 KB ring) per SM
     if (nchunks < g) g = nchunks;
     return static_cast<int>(g < 1 ? 1 : g);
 }
