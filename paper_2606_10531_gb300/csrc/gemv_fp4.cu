@@ -173,9 +173,10 @@ __device__ __forceinline__ void named_arrive(int id, int count) {
     asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
-// e2m1 bit pattern of a balanced base-8 digit d in [-4, 3], indexed by d + 4:
-// -4 -> 0xE, -3 -> 0xD, -2 -> 0xC, -1 -> 0xA, 0 -> 0x0, 1 -> 0x2, 2 -> 0x4, 3 -> 0x5
-constexpr uint32_t kE2m1Digits = 0x5420ACDEu;
+// e2m1 bit pattern of a balanced base-8 digit d in [-4, 3], one per byte, byte d + 4 of {lo, hi}
+// (a byte-permute table): -4 -> 0xE, -3 -> 0xD, -2 -> 0xC, -1 -> 0xA, 0 -> 0x0, 1 -> 0x2, 2 -> 0x4,
+// 3 -> 0x5
+constexpr uint32_t kE2m1BytesLo = 0x0A0C0D0Eu, kE2m1BytesHi = 0x05040200u;
 
 // Rows [s0, s1) of 32-row slices form range r of `ranges` (balanced split of `slices`).
 __host__ __device__ inline void f4_range(int r, int slices, int ranges, int &s0, int &s1) {
@@ -262,12 +263,18 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
         float xp[16];
 #pragma unroll
         for (int g = 0; g < 16 / D; ++g) {
+            // outputs in pairs (k, k + 1) by packed fp32x2 FMAs: each lane's FMA sequence over j is
+            // the scalar one
 #pragma unroll
-            for (int k = 0; k < D; ++k) {
-                float acc = 0.0f;
+            for (int k = 0; k < D; k += 2) {
+                float2 acc = make_float2(0.0f, 0.0f);
 #pragma unroll
-                for (int j = 0; j < D; ++j) acc = fmaf(xv[gg][g * D + j], sA[j * D + k], acc);
-                xp[k + g * D] = acc;
+                for (int j = 0; j < D; ++j) {
+                    const float xj = xv[gg][g * D + j];
+                    acc = __ffma2_rn(make_float2(xj, xj), make_float2(sA[j * D + k], sA[j * D + k + 1]), acc);
+                }
+                xp[k + g * D] = acc.x;
+                xp[k + 1 + g * D] = acc.y;
             }
 #pragma unroll
             for (int j = 0; j < D; ++j) r = fmaf(xv[gg][g * D + j], sb[j], r);
@@ -314,12 +321,15 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
             uint32_t lo = 0, hi = 0;   // K positions 0..7 and 8..15 of the group
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-                // e2m1 pattern of digit field - 4, from the table indexed by the field
-                const uint32_t nib = (kE2m1Digits >> (((u[i] >> (3 * j)) & 7u) << 2)) & 0xFu;
-                // column i = 2 u + p sits at K position 8 p + u
+                // field j of u (bit-field extract), its e2m1 pattern from the byte table (byte
+                // permute; the field selects byte f of kE2m1Bytes), inserted at the column's K position
+                // (bit-field insert of the low 4 bits): column i = 2 u + p sits at K position 8 p + u
+                uint32_t f, nib;
+                asm("bfe.u32 %0, %1, %2, 3;" : "=r"(f) : "r"(u[i]), "r"(3 * j));
+                asm("prmt.b32 %0, %1, %2, %3;" : "=r"(nib) : "r"(kE2m1BytesLo), "r"(kE2m1BytesHi), "r"(f));
                 const int pos = 8 * (i & 1) + (i >> 1);
-                if (pos < 8) lo |= nib << (4 * pos);
-                else hi |= nib << (4 * (pos - 8));
+                if (pos < 8) asm("bfi.b32 %0, %1, %2, %3, 4;" : "=r"(lo) : "r"(nib), "r"(lo), "r"(4 * pos));
+                else asm("bfi.b32 %0, %1, %2, %3, 4;" : "=r"(hi) : "r"(nib), "r"(hi), "r"(4 * (pos - 8)));
             }
             uint8_t *dst = dig + (tile * NB + t * kF4Digits + j) * 256 + slot * 8;
             *reinterpret_cast<uint2 *>(dst) = make_uint2(lo, hi);
