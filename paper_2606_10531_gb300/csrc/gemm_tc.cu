@@ -47,14 +47,17 @@ struct GemmParams {
     int32_t *status;
 };
 
-__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int &tm, int &tn) {
-    const int span = kGroupM * num_n;
+__device__ __forceinline__ void tile_coords_group(int tile, int num_m, int num_n, int group_m, int &tm, int &tn) {
+    const int span = group_m * num_n;
     const int g = tile / span;
-    const int first_m = g * kGroupM;
-    const int gsize = min(num_m - first_m, kGroupM);
+    const int first_m = g * group_m;
+    const int gsize = min(num_m - first_m, group_m);
     const int r = tile - g * span;
     tm = first_m + r % gsize;
     tn = r / gsize;
+}
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int &tm, int &tn) {
+    tile_coords_group(tile, num_m, num_n, kGroupM, tm, tn);
 }
 
 template <bool MN>
@@ -76,6 +79,117 @@ __device__ __forceinline__ void load_operand(uint8_t *dst, const CUtensorMap *ma
         for (int c = 0; c < ROWS / 64; ++c) tma_load_2d(dst + c * 8192, map, row0 + c * 64, k0, bar);
     } else {
         tma_load_2d(dst, map, k0, row0, bar);
+    }
+}
+
+// Epilogue of one 32-column chunk of an accumulator row: bf16 store, or the weight-gradient epilogue
+// (EPI_DW) with its per-thread dA, db sums.
+template <int EPI, int D>
+__device__ __forceinline__ void epilogue_chunk(const GemmParams &p, const float (&v)[32], int row, int col0,
+                                               const float (&Am)[EPI == EPI_DW ? D * D : 1],
+                                               float (&dA)[EPI == EPI_DW ? D * D : 1],
+                                               float (&db)[EPI == EPI_DW ? D : 1]) {
+    if (row >= p.M || col0 >= p.N) return;
+    if (EPI == EPI_STORE_BF16) {
+        uint16_t *dst = p.C + static_cast<int64_t>(row) * p.ldc + col0;
+        if (col0 + 32 <= p.N) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                reinterpret_cast<uint4 *>(dst)[u] =
+                    make_uint4(pack_bf16x2(v[8 * u + 0], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
+                               pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                if (col0 + e < p.N) {
+                    const __nv_bfloat16 h = __float2bfloat16_rn(v[e]);
+                    dst[e] = *reinterpret_cast<const uint16_t *>(&h);
+                }
+            }
+        }
+    } else {
+        // weight-gradient epilogue: this thread holds dW_hat[row][col0 .. col0+31]
+        const int64_t nq = p.N / 4;   // packed bytes per row
+        const uint8_t *zrow = p.dw.packed + static_cast<int64_t>(row) * nq + col0 / 4;
+        uint32_t zw[2];
+        const bool full32 = col0 + 32 <= p.N;
+        if (full32 && (nq % 8) == 0) {
+            const uint2 t2 = *reinterpret_cast<const uint2 *>(zrow);
+            zw[0] = t2.x; zw[1] = t2.y;
+        } else {
+            zw[0] = zw[1] = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                if (col0 + 4 * e < p.N) zw[e >> 2] |= static_cast<uint32_t>(zrow[e]) << (8 * (e & 3));
+        }
+        float *dprow = p.dw.dP + static_cast<int64_t>(row) * p.N + col0;
+        const float *prow = p.dw.P ? p.dw.P + static_cast<int64_t>(row) * p.N + col0 : nullptr;
+#pragma unroll
+        for (int g = 0; g < 32 / D; ++g) {
+            if (col0 + g * D >= p.N) break;
+            float z[D], out[D];
+#pragma unroll
+            for (int k = 0; k < D; ++k) {
+                const int e = g * D + k;
+                z[k] = static_cast<float>((zw[e >> 4] >> (2 * (e & 15))) & 3u);
+            }
+#pragma unroll
+            for (int k = 0; k < D; ++k) {
+                float t = 0.0f;
+#pragma unroll
+                for (int j = 0; j < D; ++j) t = fmaf(v[g * D + j], Am[j * D + k], t);
+                out[k] = t * p.dw.inv_s;
+            }
+            if (p.dw.ste_mode == LCQ_STE_CLIPPED) {
+#pragma unroll
+                for (int k = 0; k < D; ++k) {
+                    const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
+                    if (!(u >= -0.5f && u <= 3.5f)) out[k] = 0.0f;
+                }
+            } else if (p.dw.ste_mode == LCQ_STE_DGE) {
+                // slope of the differentiable gradient estimator (Eq. dge) at v, delta = 1
+#pragma unroll
+                for (int k = 0; k < D; ++k) {
+                    const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
+                    const float x = u - floorf(u);
+                    const float y = fabsf(2.0f * x - 1.0f);
+                    float gs = fminf(p.dw.dge_cap, p.dw.dge_inv_k * exp2f(p.dw.dge_exp * log2f(y)));
+                    if (!(u >= 0.0f && u < 3.0f)) gs = 0.0f;
+                    out[k] *= gs;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < D; k += 4)
+                *reinterpret_cast<float4 *>(dprow + g * D + k) = make_float4(out[k], out[k + 1], out[k + 2], out[k + 3]);
+#pragma unroll
+            for (int j = 0; j < D; ++j) {
+                db[j] += v[g * D + j];
+#pragma unroll
+                for (int k = 0; k < D; ++k) dA[j * D + k] = fmaf(v[g * D + j], z[k], dA[j * D + k]);
+            }
+        }
+    }
+}
+
+// End of a CTA's weight-gradient epilogue: fixed-order reduction of the per-thread dA, db (lanes by a
+// butterfly, then the four warps in order) into this CTA's partials.
+template <int D>
+__device__ __forceinline__ void epilogue_dw_reduce(const float (&dA)[D * D], const float (&db)[D], float (*red)[72], int q,
+                                                   int warp, int lane, float *partials) {
+    constexpr int NV = D * D + D;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        float x = i < D * D ? dA[i] : db[i - D * D];
+        for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (lane == 0) red[q][i] = x;
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (warp == 2) {
+        for (int i = lane; i < NV; i += 32) {
+            const float x = ((red[0][i] + red[1][i]) + red[2][i]) + red[3][i];
+            partials[static_cast<int64_t>(blockIdx.x) * NV + i] = x;
+        }
     }
 }
 
@@ -181,110 +295,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 float v[32];
                 __syncwarp();   // tcgen05.ld is warp-collective: reconverge after the bounds checks
                 tmem_ld32(taddr + c * 32, v);
-                const int col0 = tn * BN + c * 32;
-                if (row >= p.M || col0 >= p.N) continue;
-                if (EPI == EPI_STORE_BF16) {
-                    uint16_t *dst = p.C + static_cast<int64_t>(row) * p.ldc + col0;
-                    if (col0 + 32 <= p.N) {
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            reinterpret_cast<uint4 *>(dst)[u] =
-                                make_uint4(pack_bf16x2(v[8 * u + 0], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
-                                           pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
-                        }
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 32; ++e) {
-                            if (col0 + e < p.N) {
-                                const __nv_bfloat16 h = __float2bfloat16_rn(v[e]);
-                                dst[e] = *reinterpret_cast<const uint16_t *>(&h);
-                            }
-                        }
-                    }
-                } else {
-                    // weight-gradient epilogue: this thread holds dW_hat[row][col0 .. col0+31]
-                    const int64_t nq = p.N / 4;   // packed bytes per row
-                    const uint8_t *zrow = p.dw.packed + static_cast<int64_t>(row) * nq + col0 / 4;
-                    uint32_t zw[2];
-                    const bool full32 = col0 + 32 <= p.N;
-                    if (full32 && (nq % 8) == 0) {
-                        const uint2 t2 = *reinterpret_cast<const uint2 *>(zrow);
-                        zw[0] = t2.x; zw[1] = t2.y;
-                    } else {
-                        zw[0] = zw[1] = 0;
-#pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            if (col0 + 4 * e < p.N) zw[e >> 2] |= static_cast<uint32_t>(zrow[e]) << (8 * (e & 3));
-                    }
-                    float *dprow = p.dw.dP + static_cast<int64_t>(row) * p.N + col0;
-                    const float *prow = p.dw.P ? p.dw.P + static_cast<int64_t>(row) * p.N + col0 : nullptr;
-#pragma unroll
-                    for (int g = 0; g < 32 / D; ++g) {
-                        if (col0 + g * D >= p.N) break;
-                        float z[D], out[D];
-#pragma unroll
-                        for (int k = 0; k < D; ++k) {
-                            const int e = g * D + k;
-                            z[k] = static_cast<float>((zw[e >> 4] >> (2 * (e & 15))) & 3u);
-                        }
-#pragma unroll
-                        for (int k = 0; k < D; ++k) {
-                            float t = 0.0f;
-#pragma unroll
-                            for (int j = 0; j < D; ++j) t = fmaf(v[g * D + j], Am[j * D + k], t);
-                            out[k] = t * p.dw.inv_s;
-                        }
-                        if (p.dw.ste_mode == LCQ_STE_CLIPPED) {
-#pragma unroll
-                            for (int k = 0; k < D; ++k) {
-                                const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
-                                if (!(u >= -0.5f && u <= 3.5f)) out[k] = 0.0f;
-                            }
-                        } else if (p.dw.ste_mode == LCQ_STE_DGE) {
-                            // slope of the differentiable gradient estimator (Eq. dge) at v, delta = 1
-#pragma unroll
-                            for (int k = 0; k < D; ++k) {
-                                const float u = __fadd_rn(__fmul_rn(prow[g * D + k], p.dw.inv_s), p.dw.t);
-                                const float x = u - floorf(u);
-                                const float y = fabsf(2.0f * x - 1.0f);
-                                float gs = fminf(p.dw.dge_cap, p.dw.dge_inv_k * exp2f(p.dw.dge_exp * log2f(y)));
-                                if (!(u >= 0.0f && u < 3.0f)) gs = 0.0f;
-                                out[k] *= gs;
-                            }
-                        }
-#pragma unroll
-                        for (int k = 0; k < D; k += 4)
-                            *reinterpret_cast<float4 *>(dprow + g * D + k) = make_float4(out[k], out[k + 1], out[k + 2], out[k + 3]);
-#pragma unroll
-                        for (int j = 0; j < D; ++j) {
-                            db[j] += v[g * D + j];
-#pragma unroll
-                            for (int k = 0; k < D; ++k) dA[j * D + k] = fmaf(v[g * D + j], z[k], dA[j * D + k]);
-                        }
-                    }
-                }
+                epilogue_chunk<EPI, D>(p, v, row, tn * BN + c * 32, Am, dA, db);
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.tempty[acc]);
         }
-        if (EPI == EPI_DW) {
-            // fixed-order reduction: lanes (butterfly), then the 4 warps in order
-            constexpr int NV = D * D + D;
-#pragma unroll
-            for (int i = 0; i < NV; ++i) {
-                float x = i < D * D ? dA[i] : db[i - D * D];
-                for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-                if (lane == 0) s.red[q][i] = x;
-            }
-            asm volatile("bar.sync 1, 128;" ::: "memory");
-            if (warp == 2) {
-                for (int i = lane; i < NV; i += 32) {
-                    const float x = ((s.red[0][i] + s.red[1][i]) + s.red[2][i]) + s.red[3][i];
-                    p.dw.partials[static_cast<int64_t>(blockIdx.x) * NV + i] = x;
-                }
-            }
-        }
+        if (EPI == EPI_DW) epilogue_dw_reduce<D>(dA, db, s.red, q, warp, lane, p.dw.partials);
     }
 
     tc_fence_before();
@@ -292,6 +309,215 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ------------------------------------------------------------------ paired kernel (cta_group::2)
+//
+// The same GEMM on 256 x 256 tiles per pair of CTAs (a cluster of two). CTA r of the pair holds rows
+// r*128.. of the tile's A and rows r*128.. of its B in its own shared memory (32 KB per stage, so six
+// stages fit where the single-CTA kernel holds four 48 KB ones); the leader's tcgen05.mma.cta_group::2
+// (M = 256, N = 256) reads both CTAs' halves and writes each CTA's 128 accumulator rows into that
+// CTA's tensor memory. Both CTAs' TMA copies complete on the leader's full barrier (the copies'
+// .cta_group::2 form, the barrier addressed through mapa), the leader's MMA commits arrive on both
+// CTAs' empty and accumulator-full barriers (multicast), and both CTAs' epilogue warps arrive on the
+// leader's accumulator-empty barrier. Each CTA's epilogue handles its own 128 rows x 256 columns.
+
+constexpr int PM = 256, PN = 256, PH = 128;   // pair tile; rows of A and of B per CTA
+constexpr int PSTAGES = 6;
+constexpr int P_HALF = PH * BK * 2;            // 16 KB: one CTA's A (or B) rows of a stage
+constexpr int kPairGroupM = 8;                 // pair-tile raster: groups of 8 M pair-tiles (2048 rows)
+
+struct PairSmem {
+    uint8_t a[PSTAGES][P_HALF];
+    uint8_t b[PSTAGES][P_HALF];
+    uint64_t full[PSTAGES];    // leader's: both CTAs' copies of the stage landed
+    uint64_t empty[PSTAGES];   // each CTA's: the MMAs reading the stage completed
+    uint64_t tfull[2];         // each CTA's: the accumulator is complete
+    uint64_t tempty[2];        // leader's: both CTAs' epilogues have read the accumulator
+    uint32_t tmem_base;
+    float Am[64];
+    float red[4][72];
+};
+
+__device__ __forceinline__ uint32_t pair_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void pair_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared variable in the leader CTA (rank 0) of the pair.
+__device__ __forceinline__ uint32_t leader_smem(const void *p) {
+    uint32_t m;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(m) : "r"(smem_u32(p)));
+    return m;
+}
+// 2-D TMA copy into this CTA's shared memory, completing on the leader's mbarrier.
+__device__ __forceinline__ void tma_load_2d_to_leader(void *dst, const CUtensorMap *map, int32_t c0, int32_t c1,
+                                                      uint32_t leader_bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%2, "
+        "%3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(leader_bar)
+        : "memory");
+}
+template <bool MN>
+__device__ __forceinline__ void load_half(uint8_t *dst, const CUtensorMap *map, int row0, int k0, uint32_t leader_bar) {
+    if (MN) {
+#pragma unroll
+        for (int c = 0; c < PH / 64; ++c) tma_load_2d_to_leader(dst + c * 8192, map, row0 + c * 64, k0, leader_bar);
+    } else {
+        tma_load_2d_to_leader(dst, map, k0, row0, leader_bar);
+    }
+}
+__device__ __forceinline__ void umma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive on the mbarrier at this shared address in both CTAs of the pair once the MMAs issued so far
+// have completed.
+__device__ __forceinline__ void umma_commit_both(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"(static_cast<uint16_t>(3))
+        : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+template <int EPI, int D, bool A_MN, bool B_MN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    PairSmem &s = *reinterpret_cast<PairSmem *>(align_smem_1024(smem_raw));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = pair_rank();
+    const int cid = static_cast<int>(blockIdx.x) >> 1, nclusters = static_cast<int>(gridDim.x) >> 1;
+    const int num_m = (p.M + PM - 1) / PM, num_n = (p.N + PN - 1) / PN;
+    const int num_tiles = num_m * num_n;
+    const int num_kb = (p.K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        prefetch_tensormap(&tmA);
+        prefetch_tensormap(&tmB);
+        for (int i = 0; i < PSTAGES; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s.tfull[i], 1);
+            mbar_init(&s.tempty[i], 8);   // the four epilogue warps of each CTA
+        }
+        fence_barrier_init();
+    }
+    if (EPI == EPI_DW && threadIdx.x < D * D) s.Am[threadIdx.x] = p.dw.A[threadIdx.x];
+    if (warp == 1) {
+        // the pair allocates together: both CTAs receive the same columns
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s.tmem_base)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    pair_sync();   // both CTAs' barriers are initialised before any copy or arrival reaches them
+    tc_fence_after();
+    const uint32_t tmem = s.tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------------------ TMA producer (both CTAs)
+            int it = 0;
+            bool ok = true;
+            for (int tile = cid; tile < num_tiles && ok; tile += nclusters) {
+                int tm, tn;
+                tile_coords_group(tile, num_m, num_n, kPairGroupM, tm, tn);
+                for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                    const int st = it % PSTAGES;
+                    if (!mbar_wait(&s.empty[st], ((it / PSTAGES) & 1) ^ 1, p.status)) { ok = false; break; }
+                    if (rank == 0) mbar_arrive_expect_tx(&s.full[st], 4 * P_HALF);   // both CTAs' A and B halves
+                    const uint32_t fb = leader_smem(&s.full[st]);
+                    load_half<A_MN>(s.a[st], &tmA, tm * PM + static_cast<int>(rank) * PH, kb * BK, fb);
+                    load_half<B_MN>(s.b[st], &tmB, tn * PN + static_cast<int>(rank) * PH, kb * BK, fb);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            // ------------------------------------------------------------ MMA issuer (leader)
+            constexpr uint32_t idesc = idesc_bf16(PM, PN, A_MN, B_MN);
+            int it = 0, tcount = 0;
+            bool ok = true;
+            for (int tile = cid; tile < num_tiles && ok; tile += nclusters, ++tcount) {
+                const int acc = tcount & 1;
+                if (!mbar_wait(&s.tempty[acc], ((tcount >> 1) & 1) ^ 1, p.status)) break;
+                tc_fence_after();
+                const uint32_t dtm = tmem + acc * PN;
+                for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                    const int st = it % PSTAGES;
+                    if (!mbar_wait(&s.full[st], (it / PSTAGES) & 1, p.status)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t abase = smem_u32(s.a[st]), bbase = smem_u32(s.b[st]);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k) {
+                        umma_bf16_pair(dtm, operand_desc<A_MN>(abase, k), operand_desc<B_MN>(bbase, k), idesc,
+                                       (kb | k) != 0);
+                    }
+                    umma_commit_both(&s.empty[st]);
+                }
+                umma_commit_both(&s.tfull[acc]);
+            }
+        }
+    } else {
+        // ---------------------------------------------------------------- epilogue (warps 2..5, both CTAs)
+        const int q = warp & 3;   // TMEM lane quarter this warp may access
+        float dA[EPI == EPI_DW ? D * D : 1], db[EPI == EPI_DW ? D : 1];
+        float Am[EPI == EPI_DW ? D * D : 1];
+        if (EPI == EPI_DW) {
+#pragma unroll
+            for (int i = 0; i < D * D; ++i) { dA[i] = 0.0f; Am[i] = s.Am[i]; }
+#pragma unroll
+            for (int i = 0; i < D; ++i) db[i] = 0.0f;
+        }
+        const uint32_t tempty_leader0 = leader_smem(&s.tempty[0]), tempty_leader1 = leader_smem(&s.tempty[1]);
+        int tcount = 0;
+        for (int tile = cid; tile < num_tiles; tile += nclusters, ++tcount) {
+            int tm, tn;
+            tile_coords_group(tile, num_m, num_n, kPairGroupM, tm, tn);
+            const int acc = tcount & 1;
+            if (!mbar_wait(&s.tfull[acc], (tcount >> 1) & 1, p.status)) break;
+            tc_fence_after();
+            const int row = tm * PM + static_cast<int>(rank) * PH + q * 32 + lane;
+            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * PN;
+#pragma unroll 1
+            for (int c = 0; c < PN / 32; ++c) {
+                float v[32];
+                __syncwarp();   // tcgen05.ld is warp-collective: reconverge after the bounds checks
+                tmem_ld32(taddr + c * 32, v);
+                epilogue_chunk<EPI, D>(p, v, row, tn * PN + c * 32, Am, dA, db);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
+        }
+        if (EPI == EPI_DW) epilogue_dw_reduce<D>(dA, db, s.red, q, warp, lane, p.dw.partials);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    pair_sync();   // no copy, commit or arrival of either CTA is still headed for the other
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -325,20 +551,23 @@ static bool make_map(CUtensorMap *map, const GemmOperand &op, int64_t rows, int6
     return r == CUDA_SUCCESS;
 }
 
+// Pairs of CTAs (clusters of two) run the paired kernel; the grid is two CTAs per pair tile, at most
+// one per SM.
 int gemm_grid(int64_t M, int64_t N, int num_sms) {
-    const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-    return static_cast<int>(tiles < num_sms ? (tiles < 1 ? 1 : tiles) : num_sms);
+    const int64_t tiles = ((M + PM - 1) / PM) * ((N + PN - 1) / PN);
+    const int64_t pairs = num_sms / 2 > 0 ? num_sms / 2 : 1;
+    return static_cast<int>(2 * (tiles < pairs ? (tiles < 1 ? 1 : tiles) : pairs));
 }
 
 template <int EPI, int D, bool A_MN, bool B_MN>
 static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, const GemmParams &gp, int grid,
                               int trace_kind, cudaStream_t st) {
-    auto k = gemm_kernel<EPI, D, A_MN, B_MN>;
-    const int smem = static_cast<int>(sizeof(GemmSmem) + 1024);
+    auto k = gemm_pair_kernel<EPI, D, A_MN, B_MN>;
+    const int smem = static_cast<int>(sizeof(PairSmem) + 1024);
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), smem);
     if (e != cudaSuccess) return e;
     trace_begin(trace_kind, st);
-    k<<<grid, kGemmThreads, smem, st>>>(ma, mb, gp);
+    k<<<grid, kGemmThreads, smem, st>>>(ma, mb, gp);   // cluster dimensions (2, 1, 1) from the kernel
     trace_end(trace_kind, st);
     count_launch();
     return cudaGetLastError();
@@ -346,7 +575,7 @@ static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, cons
 
 cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cudaStream_t st) {
     CUtensorMap ma, mb;
-    if (!make_map(&ma, p.a, p.M, p.K, BM) || !make_map(&mb, p.b, p.N, p.K, BN)) return cudaErrorInvalidValue;
+    if (!make_map(&ma, p.a, p.M, p.K, PH) || !make_map(&mb, p.b, p.N, p.K, PH)) return cudaErrorInvalidValue;
     GemmParams gp;
     gp.M = static_cast<int>(p.M);
     gp.N = static_cast<int>(p.N);
