@@ -1,15 +1,22 @@
-// Persistent bf16 GEMM on the 5th-generation tensor cores (tcgen05 + TMEM), fed by TMA.
+// Persistent bf16 GEMM on the 5th-generation tensor cores (tcgen05 + TMEM), fed by TMA, run by pairs
+// of CTAs (clusters of two) over 256 x 256 output tiles.
 //
 //   C[M][N] = sum_k A(m, k) * B(n, k)        fp32 accumulation in tensor memory
 //
-// One CTA per SM, 192 threads:
-//   warp 0      TMA producer: 4-stage ring of (128 x 64) A and (256 x 64) B bf16 tiles, 128B swizzle
-//   warp 1      TMEM owner (512 columns = two 128 x 256 fp32 accumulators) and single-thread MMA issuer
-//   warps 2..5  epilogue: tcgen05.ld the accumulator (one TMEM lane quarter per warp) and
+// Per CTA, one per SM, 192 threads:
+//   warp 0      TMA producer: a 6-stage ring of this CTA's halves of the tile, rows r*128.. of A and
+//               rows r*128.. of B (128 x 64 bf16 each, 128B swizzle; r = rank in the pair)
+//   warp 1      TMEM owner (512 columns = two 128 x 256 fp32 accumulators, allocated by the pair
+//               together) and, in the leader CTA, the single-thread issuer of
+//               tcgen05.mma.cta_group::2 (M = 256, N = 256), which reads both CTAs' halves and writes
+//               each CTA's 128 accumulator rows into its own tensor memory
+//   warps 2..5  epilogue: tcgen05.ld this CTA's accumulator rows (one TMEM lane quarter per warp) and
 //               either store bf16 C, or run the LC-VQ weight-gradient epilogue (EPI_DW):
 //                 dP_g = (1/s) * dW_hat_g A        (straight-through estimator, Sec. 3.3)
 //                 dA  += dW_hat_g z_g^T,  db += dW_hat_g   (per-thread, reduced per CTA at the end)
-// The two accumulators let the epilogue of tile i overlap the main loop of tile i+1.
+// The two accumulators let the epilogue of tile i overlap the main loop of tile i+1. Holding half of
+// B per SM leaves room for six stages of operand data in flight (four with a whole 128 x 256 tile per
+// CTA), which is what the main loop waits on.
 // Operands may be K-major ([rows][K]) or MN-major ([K][rows]); both layouts are read by TMA
 // with 128-byte swizzle and described to the tensor core with the matching smem descriptor.
 #include <cuda.h>
@@ -20,24 +27,9 @@
 
 namespace lcq {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int A_STAGE = BM * BK * 2;   // 16 KB
-constexpr int B_STAGE = BN * BK * 2;   // 32 KB
+constexpr int BK = 64;
 constexpr int kGemmThreads = 192;
 constexpr uint32_t kTmemCols = 512;
-constexpr int kGroupM = 16;            // tile raster: groups of 16 M-tiles sweep all N-tiles
-
-struct GemmSmem {
-    uint8_t a[STAGES][A_STAGE];
-    uint8_t b[STAGES][B_STAGE];
-    uint64_t full[STAGES];
-    uint64_t empty[STAGES];
-    uint64_t tfull[2];
-    uint64_t tempty[2];
-    uint32_t tmem_base;
-    float Am[64];
-    float red[4][72];
-};
 
 struct GemmParams {
     int M, N, K;
@@ -56,9 +48,6 @@ __device__ __forceinline__ void tile_coords_group(int tile, int num_m, int num_n
     tm = first_m + r % gsize;
     tn = r / gsize;
 }
-__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int &tm, int &tn) {
-    tile_coords_group(tile, num_m, num_n, kGroupM, tm, tn);
-}
 
 template <bool MN>
 __device__ __forceinline__ uint64_t operand_desc(uint32_t stage_base, int kstep) {
@@ -72,18 +61,6 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t stage_base, int kstep)
     }
 }
 
-template <bool MN, int ROWS>
-__device__ __forceinline__ void load_operand(uint8_t *dst, const CUtensorMap *map, int row0, int k0, uint64_t *bar) {
-    if (MN) {
-#pragma unroll
-        for (int c = 0; c < ROWS / 64; ++c) tma_load_2d(dst + c * 8192, map, row0 + c * 64, k0, bar);
-    } else {
-        tma_load_2d(dst, map, k0, row0, bar);
-    }
-}
-
-// Epilogue of one 32-column chunk of an accumulator row: bf16 store, or the weight-gradient epilogue
-// (EPI_DW) with its per-thread dA, db sums.
 template <int EPI, int D>
 __device__ __forceinline__ void epilogue_chunk(const GemmParams &p, const float (&v)[32], int row, int col0,
                                                const float (&Am)[EPI == EPI_DW ? D * D : 1],
@@ -190,125 +167,6 @@ __device__ __forceinline__ void epilogue_dw_reduce(const float (&dA)[D * D], con
             const float x = ((red[0][i] + red[1][i]) + red[2][i]) + red[3][i];
             partials[static_cast<int64_t>(blockIdx.x) * NV + i] = x;
         }
-    }
-}
-
-template <int EPI, int D, bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kGemmThreads, 1)
-gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
-    // 1024-byte alignment of the stage buffers is required by the 128B swizzle atoms.
-    GemmSmem &s = *reinterpret_cast<GemmSmem *>(align_smem_1024(smem_raw));
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_m = (p.M + BM - 1) / BM, num_n = (p.N + BN - 1) / BN;
-    const int num_tiles = num_m * num_n;
-    const int num_kb = (p.K + BK - 1) / BK;
-
-    if (threadIdx.x == 0) {
-        prefetch_tensormap(&tmA);
-        prefetch_tensormap(&tmB);
-        for (int i = 0; i < STAGES; ++i) {
-            mbar_init(&s.full[i], 1);
-            mbar_init(&s.empty[i], 1);
-        }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&s.tfull[i], 1);
-            mbar_init(&s.tempty[i], 4);
-        }
-        fence_barrier_init();
-    }
-    if (EPI == EPI_DW && threadIdx.x < D * D) s.Am[threadIdx.x] = p.dw.A[threadIdx.x];
-    if (warp == 1) {
-        tmem_alloc(&s.tmem_base, kTmemCols);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = s.tmem_base;
-
-    if (warp == 0) {
-        if (lane == 0) {
-            // ------------------------------------------------------------ TMA producer
-            int it = 0;
-            bool ok = true;
-            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-                int tm, tn;
-                tile_coords(tile, num_m, num_n, tm, tn);
-                for (int kb = 0; kb < num_kb; ++kb, ++it) {
-                    const int st = it % STAGES;
-                    if (!mbar_wait(&s.empty[st], ((it / STAGES) & 1) ^ 1, p.status)) { ok = false; break; }
-                    mbar_arrive_expect_tx(&s.full[st], A_STAGE + B_STAGE);
-                    load_operand<A_MN, BM>(s.a[st], &tmA, tm * BM, kb * BK, &s.full[st]);
-                    load_operand<B_MN, BN>(s.b[st], &tmB, tn * BN, kb * BK, &s.full[st]);
-                }
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // ------------------------------------------------------------ MMA issuer
-            constexpr uint32_t idesc = idesc_bf16(BM, BN, A_MN, B_MN);
-            int it = 0, tcount = 0;
-            bool ok = true;
-            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tcount) {
-                const int acc = tcount & 1;
-                if (!mbar_wait(&s.tempty[acc], ((tcount >> 1) & 1) ^ 1, p.status)) break;
-                tc_fence_after();
-                const uint32_t dtm = tmem + acc * BN;
-                for (int kb = 0; kb < num_kb; ++kb, ++it) {
-                    const int st = it % STAGES;
-                    if (!mbar_wait(&s.full[st], (it / STAGES) & 1, p.status)) { ok = false; break; }
-                    tc_fence_after();
-                    const uint32_t abase = smem_u32(s.a[st]), bbase = smem_u32(s.b[st]);
-#pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {
-                        umma_bf16(dtm, operand_desc<A_MN>(abase, k), operand_desc<B_MN>(bbase, k), idesc,
-                                  (kb | k) != 0);
-                    }
-                    umma_commit(&s.empty[st]);
-                }
-                umma_commit(&s.tfull[acc]);
-            }
-        }
-    } else {
-        // ---------------------------------------------------------------- epilogue (warps 2..5)
-        const int q = warp & 3;   // TMEM lane quarter this warp may access
-        float dA[EPI == EPI_DW ? D * D : 1], db[EPI == EPI_DW ? D : 1];
-        float Am[EPI == EPI_DW ? D * D : 1];
-        if (EPI == EPI_DW) {
-#pragma unroll
-            for (int i = 0; i < D * D; ++i) { dA[i] = 0.0f; Am[i] = s.Am[i]; }
-#pragma unroll
-            for (int i = 0; i < D; ++i) db[i] = 0.0f;
-        }
-        int tcount = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tcount) {
-            int tm, tn;
-            tile_coords(tile, num_m, num_n, tm, tn);
-            const int acc = tcount & 1;
-            if (!mbar_wait(&s.tfull[acc], (tcount >> 1) & 1, p.status)) break;
-            tc_fence_after();
-            const int row = tm * BM + q * 32 + lane;
-            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                float v[32];
-                __syncwarp();   // tcgen05.ld is warp-collective: reconverge after the bounds checks
-                tmem_ld32(taddr + c * 32, v);
-                epilogue_chunk<EPI, D>(p, v, row, tn * BN + c * 32, Am, dA, db);
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.tempty[acc]);
-        }
-        if (EPI == EPI_DW) epilogue_dw_reduce<D>(dA, db, s.red, q, warp, lane, p.dw.partials);
-    }
-
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 1) {
-        tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
     }
 }
 
