@@ -252,21 +252,45 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
+// Work item w of pair cid (of G pairs): the whole tiles cid, cid + G, ...; then, when the tiles of the
+// last, partial wave split into two 128-column halves still fit one wave (2R <= G), half tile cid of
+// that wave (half = 0 or 1; -1 for a whole tile), so the last wave takes half the time.
+struct PairWork {
+    int tm, tn, half;
+};
+__device__ __forceinline__ bool pair_work(int w, int cid, int G, int num_m, int num_n, PairWork &o) {
+    const int tiles = num_m * num_n;
+    const int R = tiles % G;
+    const bool split = R > 0 && 2 * R <= G;
+    const int whole = split ? tiles - R : tiles;
+    const int nwhole = whole > cid ? (whole - cid + G - 1) / G : 0;
+    if (w < nwhole) {
+        tile_coords_group(cid + w * G, num_m, num_n, kPairGroupM, o.tm, o.tn);
+        o.half = -1;
+        return true;
+    }
+    if (!split || w != nwhole || cid >= 2 * R) return false;
+    tile_coords_group(whole + (cid >> 1), num_m, num_n, kPairGroupM, o.tm, o.tn);
+    o.half = cid & 1;
+    return true;
+}
+
 template <int EPI, int D, bool A_MN, bool B_MN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
-gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                 const __grid_constant__ CUtensorMap tmB64, const GemmParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     PairSmem &s = *reinterpret_cast<PairSmem *>(align_smem_1024(smem_raw));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = pair_rank();
     const int cid = static_cast<int>(blockIdx.x) >> 1, nclusters = static_cast<int>(gridDim.x) >> 1;
     const int num_m = (p.M + PM - 1) / PM, num_n = (p.N + PN - 1) / PN;
-    const int num_tiles = num_m * num_n;
     const int num_kb = (p.K + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
         prefetch_tensormap(&tmA);
         prefetch_tensormap(&tmB);
+        if (!B_MN) prefetch_tensormap(&tmB64);
         for (int i = 0; i < PSTAGES; ++i) {
             mbar_init(&s.full[i], 1);
             mbar_init(&s.empty[i], 1);
@@ -296,26 +320,34 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             // ------------------------------------------------------------ TMA producer (both CTAs)
             int it = 0;
             bool ok = true;
-            for (int tile = cid; tile < num_tiles && ok; tile += nclusters) {
-                int tm, tn;
-                tile_coords_group(tile, num_m, num_n, kPairGroupM, tm, tn);
+            PairWork wk;
+            for (int w = 0; ok && pair_work(w, cid, nclusters, num_m, num_n, wk); ++w) {
+                // a half tile's B: 64 rows per CTA of its 128 columns
+                const int brows = wk.half < 0 ? PH : PH / 2;
+                const int b0 = wk.tn * PN + (wk.half > 0 ? PN / 2 : 0) + static_cast<int>(rank) * brows;
+                const uint32_t bytes = 2u * static_cast<uint32_t>(P_HALF + brows * BK * 2);   // the pair's A and B
                 for (int kb = 0; kb < num_kb; ++kb, ++it) {
                     const int st = it % PSTAGES;
                     if (!mbar_wait(&s.empty[st], ((it / PSTAGES) & 1) ^ 1, p.status)) { ok = false; break; }
-                    if (rank == 0) mbar_arrive_expect_tx(&s.full[st], 4 * P_HALF);   // both CTAs' A and B halves
+                    if (rank == 0) mbar_arrive_expect_tx(&s.full[st], bytes);
                     const uint32_t fb = leader_smem(&s.full[st]);
-                    load_half<A_MN>(s.a[st], &tmA, tm * PM + static_cast<int>(rank) * PH, kb * BK, fb);
-                    load_half<B_MN>(s.b[st], &tmB, tn * PN + static_cast<int>(rank) * PH, kb * BK, fb);
+                    load_half<A_MN>(s.a[st], &tmA, wk.tm * PM + static_cast<int>(rank) * PH, kb * BK, fb);
+                    if (wk.half < 0) load_half<B_MN>(s.b[st], &tmB, b0, kb * BK, fb);
+                    else if (B_MN) tma_load_2d_to_leader(s.b[st], &tmB, b0, kb * BK, fb);   // one 64-row chunk
+                    else tma_load_2d_to_leader(s.b[st], &tmB64, kb * BK, b0, fb);
                 }
             }
         }
     } else if (warp == 1) {
         if (lane == 0 && rank == 0) {
             // ------------------------------------------------------------ MMA issuer (leader)
-            constexpr uint32_t idesc = idesc_bf16(PM, PN, A_MN, B_MN);
+            constexpr uint32_t idesc_whole = idesc_bf16(PM, PN, A_MN, B_MN);
+            constexpr uint32_t idesc_half = idesc_bf16(PM, PN / 2, A_MN, B_MN);
             int it = 0, tcount = 0;
             bool ok = true;
-            for (int tile = cid; tile < num_tiles && ok; tile += nclusters, ++tcount) {
+            PairWork wk;
+            for (int w = 0; ok && pair_work(w, cid, nclusters, num_m, num_n, wk); ++w, ++tcount) {
+                const uint32_t idesc = wk.half < 0 ? idesc_whole : idesc_half;
                 const int acc = tcount & 1;
                 if (!mbar_wait(&s.tempty[acc], ((tcount >> 1) & 1) ^ 1, p.status)) break;
                 tc_fence_after();
@@ -348,20 +380,21 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
         }
         const uint32_t tempty_leader0 = leader_smem(&s.tempty[0]), tempty_leader1 = leader_smem(&s.tempty[1]);
         int tcount = 0;
-        for (int tile = cid; tile < num_tiles; tile += nclusters, ++tcount) {
-            int tm, tn;
-            tile_coords_group(tile, num_m, num_n, kPairGroupM, tm, tn);
+        PairWork wk;
+        for (int w = 0; pair_work(w, cid, nclusters, num_m, num_n, wk); ++w, ++tcount) {
             const int acc = tcount & 1;
             if (!mbar_wait(&s.tfull[acc], (tcount >> 1) & 1, p.status)) break;
             tc_fence_after();
-            const int row = tm * PM + static_cast<int>(rank) * PH + q * 32 + lane;
+            const int row = wk.tm * PM + static_cast<int>(rank) * PH + q * 32 + lane;
             const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * PN;
+            const int col_base = wk.tn * PN + (wk.half > 0 ? PN / 2 : 0);
+            const int nchunks = wk.half < 0 ? PN / 32 : PN / 64;
 #pragma unroll 1
-            for (int c = 0; c < PN / 32; ++c) {
+            for (int c = 0; c < nchunks; ++c) {
                 float v[32];
                 __syncwarp();   // tcgen05.ld is warp-collective: reconverge after the bounds checks
                 tmem_ld32(taddr + c * 32, v);
-                epilogue_chunk<EPI, D>(p, v, row, tn * PN + c * 32, Am, dA, db);
+                epilogue_chunk<EPI, D>(p, v, row, col_base + c * 32, Am, dA, db);
             }
             tc_fence_before();
             __syncwarp();
@@ -418,22 +451,24 @@ int gemm_grid(int64_t M, int64_t N, int num_sms) {
 }
 
 template <int EPI, int D, bool A_MN, bool B_MN>
-static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, const GemmParams &gp, int grid,
-                              int trace_kind, cudaStream_t st) {
+static cudaError_t launch_one(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mb64,
+                              const GemmParams &gp, int grid, int trace_kind, cudaStream_t st) {
     auto k = gemm_pair_kernel<EPI, D, A_MN, B_MN>;
     const int smem = static_cast<int>(sizeof(PairSmem) + 1024);
     cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void *>(k), smem);
     if (e != cudaSuccess) return e;
     trace_begin(trace_kind, st);
-    k<<<grid, kGemmThreads, smem, st>>>(ma, mb, gp);   // cluster dimensions (2, 1, 1) from the kernel
+    k<<<grid, kGemmThreads, smem, st>>>(ma, mb, mb64, gp);   // cluster dimensions (2, 1, 1) from the kernel
     trace_end(trace_kind, st);
     count_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cudaStream_t st) {
-    CUtensorMap ma, mb;
-    if (!make_map(&ma, p.a, p.M, p.K, PH) || !make_map(&mb, p.b, p.N, p.K, PH)) return cudaErrorInvalidValue;
+    // mb64: K-major B in 64-row boxes, for the halves of a split last wave
+    CUtensorMap ma, mb, mb64;
+    if (!make_map(&ma, p.a, p.M, p.K, PH) || !make_map(&mb, p.b, p.N, p.K, PH) || !make_map(&mb64, p.b, p.N, p.K, PH / 2))
+        return cudaErrorInvalidValue;
     GemmParams gp;
     gp.M = static_cast<int>(p.M);
     gp.N = static_cast<int>(p.N);
@@ -444,14 +479,14 @@ cudaError_t launch_gemm(const GemmProblem &p, GemmEpilogue epi, int num_sms, cud
     gp.status = p.status;
     const int grid = gemm_grid(p.M, p.N, num_sms);
     if (epi == EPI_STORE_BF16) {
-        if (!p.a.mn_major && !p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, false>(ma, mb, gp, grid, p.trace_kind, st);
-        if (!p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, true>(ma, mb, gp, grid, p.trace_kind, st);
-        if (p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, true, true>(ma, mb, gp, grid, p.trace_kind, st);
-        return launch_one<EPI_STORE_BF16, 1, true, false>(ma, mb, gp, grid, p.trace_kind, st);
+        if (!p.a.mn_major && !p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, false>(ma, mb, mb64, gp, grid, p.trace_kind, st);
+        if (!p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, false, true>(ma, mb, mb64, gp, grid, p.trace_kind, st);
+        if (p.a.mn_major && p.b.mn_major) return launch_one<EPI_STORE_BF16, 1, true, true>(ma, mb, mb64, gp, grid, p.trace_kind, st);
+        return launch_one<EPI_STORE_BF16, 1, true, false>(ma, mb, mb64, gp, grid, p.trace_kind, st);
     }
     if (!(p.a.mn_major && p.b.mn_major)) return cudaErrorInvalidValue;
-    if (p.dw.d == 4) return launch_one<EPI_DW, 4, true, true>(ma, mb, gp, grid, p.trace_kind, st);
-    return launch_one<EPI_DW, 8, true, true>(ma, mb, gp, grid, p.trace_kind, st);
+    if (p.dw.d == 4) return launch_one<EPI_DW, 4, true, true>(ma, mb, mb64, gp, grid, p.trace_kind, st);
+    return launch_one<EPI_DW, 8, true, true>(ma, mb, mb64, gp, grid, p.trace_kind, st);
 }
 
 }  // namespace lcq

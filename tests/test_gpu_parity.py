@@ -225,12 +225,15 @@ def test_pack2b_matches_oracle(m, n):
 # ----------------------------------------------------------------------------- training layer
 
 LINEAR_CASES = [
-    # N tokens, m out, n in, d
+    # N tokens, m out, n in, d; the GEMMs run 256 x 256 tiles on pairs of CTAs
     (64, 512, 512, 4),     # the oracle-sized layer of the workload list
-    (200, 384, 320, 8),    # 2 x 2 tiles, ragged in M and N, 5 K-blocks
+    (200, 384, 320, 8),    # 1 x 2 pair tiles, ragged in M and N, 5 K-blocks
     (130, 136, 72, 4),     # ragged everywhere, K tail of 8
     (1, 8, 8, 8),          # one token, one group
-    (520, 1024, 256, 8),   # 5 x 4 tiles with two TMEM accumulators in flight
+    (520, 1024, 256, 8),   # 3 x 4 pair tiles with two TMEM accumulators in flight
+    # on 76 pairs (152 SMs) every GEMM of this case ends in a partial wave whose tiles run as 256 x 128
+    # halves: forward 16 x 5 pair tiles, dX 16 x 16, dW 5 x 16
+    (4096, 1280, 4096, 8),
 ]
 
 
