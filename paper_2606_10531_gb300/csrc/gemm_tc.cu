@@ -4,7 +4,7 @@
 //   C[M][N] = sum_k A(m, k) * B(n, k)        fp32 accumulation in tensor memory
 //
 // Per CTA, one per SM, 192 threads:
-//   warp 0      TMA producer: a 6-stage ring of this CTA's halves of the tile, rows r*128.. of A and
+//   warp 0      TMA producer: a 7-stage ring of this CTA's halves of the tile, rows r*128.. of A and
 //               rows r*128.. of B (128 x 64 bf16 each, 128B swizzle; r = rank in the pair)
 //   warp 1      TMEM owner (512 columns = two 128 x 256 fp32 accumulators, allocated by the pair
 //               together) and, in the leader CTA, the single-thread issuer of
@@ -15,7 +15,7 @@
 //                 dP_g = (1/s) * dW_hat_g A        (straight-through estimator, Sec. 3.3)
 //                 dA  += dW_hat_g z_g^T,  db += dW_hat_g   (per-thread, reduced per CTA at the end)
 // The two accumulators let the epilogue of tile i overlap the main loop of tile i+1. Holding half of
-// B per SM leaves room for six stages of operand data in flight (four with a whole 128 x 256 tile per
+// B per SM leaves room for seven stages of operand data in flight (four with a whole 128 x 256 tile per
 // CTA), which is what the main loop waits on.
 // Operands may be K-major ([rows][K]) or MN-major ([K][rows]); both layouts are read by TMA
 // with 128-byte swizzle and described to the tensor core with the matching smem descriptor.
@@ -172,17 +172,17 @@ __device__ __forceinline__ void epilogue_dw_reduce(const float (&dA)[D * D], con
 
 // ------------------------------------------------------------------ paired kernel (cta_group::2)
 //
-// The same GEMM on 256 x 256 tiles per pair of CTAs (a cluster of two). CTA r of the pair holds rows
-// r*128.. of the tile's A and rows r*128.. of its B in its own shared memory (32 KB per stage, so six
-// stages fit where the single-CTA kernel holds four 48 KB ones); the leader's tcgen05.mma.cta_group::2
-// (M = 256, N = 256) reads both CTAs' halves and writes each CTA's 128 accumulator rows into that
-// CTA's tensor memory. Both CTAs' TMA copies complete on the leader's full barrier (the copies'
-// .cta_group::2 form, the barrier addressed through mapa), the leader's MMA commits arrive on both
-// CTAs' empty and accumulator-full barriers (multicast), and both CTAs' epilogue warps arrive on the
-// leader's accumulator-empty barrier. Each CTA's epilogue handles its own 128 rows x 256 columns.
+// 256 x 256 tiles per pair of CTAs (a cluster of two). CTA r of the pair holds rows r*128.. of the
+// tile's A and rows r*128.. of its B in its own shared memory (32 KB per stage, so seven stages fit;
+// a whole 128 x 256 tile per CTA would take 48 KB per stage, four stages); the leader's
+// tcgen05.mma.cta_group::2 (M = 256, N = 256) reads both CTAs' halves and writes each CTA's 128
+// accumulator rows into that CTA's tensor memory. Both CTAs' TMA copies complete on the leader's full
+// barrier (the copies' .cta_group::2 form, the barrier addressed through mapa), the leader's MMA
+// commits arrive on both CTAs' empty and accumulator-full barriers (multicast), and both CTAs' epilogue
+// warps arrive on the leader's accumulator-empty barrier. Each CTA's epilogue handles its own 128 rows.
 
 constexpr int PM = 256, PN = 256, PH = 128;   // pair tile; rows of A and of B per CTA
-constexpr int PSTAGES = 6;
+constexpr int PSTAGES = 7;
 constexpr int P_HALF = PH * BK * 2;            // 16 KB: one CTA's A (or B) rows of a stage
 constexpr int kPairGroupM = 8;                 // pair-tile raster: groups of 8 M pair-tiles (2048 rows)
 
@@ -195,7 +195,6 @@ struct PairSmem {
     uint64_t tempty[2];        // leader's: both CTAs' epilogues have read the accumulator
     uint32_t tmem_base;
     float Am[64];
-    float red[4][72];
 };
 
 __device__ __forceinline__ uint32_t pair_rank() {
@@ -400,7 +399,9 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
         }
-        if (EPI == EPI_DW) epilogue_dw_reduce<D>(dA, db, s.red, q, warp, lane, p.dw.partials);
+        // the ring is idle once this CTA's last accumulator is complete (every MMA reading either CTA's
+        // stages has completed and no copy is pending): its first stage holds the reduction
+        if (EPI == EPI_DW) epilogue_dw_reduce<D>(dA, db, reinterpret_cast<float (*)[72]>(s.a[0]), q, warp, lane, p.dw.partials);
     }
 
     tc_fence_before();
