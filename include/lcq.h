@@ -259,6 +259,8 @@ lcq_status lcq_linear_fwd(const uint16_t *X, int64_t N, const float *P, int64_t 
  * P [m][n] fp32 (read only in CLIPPED and DGE modes; may be NULL otherwise).
  * dX may be NULL (skips the dX GEMM). dA and db are overwritten, not
  * accumulated; the sums are taken in a fixed order (bitwise reproducible).
+ * m must be a multiple of 8 as well as n (LCQ_ERR_SHAPE otherwise, before
+ * anything is enqueued): dY's rows are read by TMA in 16-byte units.
  * Needs lcq_workspace_size(LCQ_OP_LINEAR_BWD, N, m, n, d).
  */
 lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *packed_saved, const float *P,

@@ -69,7 +69,9 @@ __device__ __forceinline__ void epilogue_chunk(const GemmParams &p, const float 
     if (row >= p.M || col0 >= p.N) return;
     if (EPI == EPI_STORE_BF16) {
         uint16_t *dst = p.C + static_cast<int64_t>(row) * p.ldc + col0;
-        if (col0 + 32 <= p.N) {
+        // 16-byte stores need a 16-byte aligned row start: the row stride of C (the output width) need
+        // not be a multiple of 8
+        if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 reinterpret_cast<uint4 *>(dst)[u] =

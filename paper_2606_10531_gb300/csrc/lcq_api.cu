@@ -546,6 +546,8 @@ lcq_status lcq_linear_bwd(const uint16_t *X, const uint16_t *dY, const uint8_t *
                           uint16_t *dX, float *dP, float *dA, float *db, void *ws, size_t ws_bytes, void *stream) {
     LCQ_TRY(check_common(m, n, d));
     if (N < 0 || N > (int64_t(1) << 31)) return LCQ_ERR_SHAPE;
+    // dY is a TMA operand of both backward GEMMs: its rows (m bf16) must span a multiple of 16 bytes
+    if (m % 8 != 0) return LCQ_ERR_SHAPE;
     float inv_s, t, dge_k, dge_cap;
     int ste;
     LCQ_TRY(opts_of(opts, inv_s, t, ste, &dge_k, &dge_cap));

@@ -91,8 +91,10 @@ def test_linear_validation(L):
     assert fwd(o=ctypes.byref(bad)) == ARG
     bad_mode = lcq.lcq_opts(1.0, 0.0, 7, 0, 0.0, 0.0)
     assert fwd(o=ctypes.byref(bad_mode)) == UNSUP
-    bwd = lambda **k: L.lcq_linear_bwd(FAKE, FAKE, FAKE, k.get("P", None), 4, 8, 16, 8, FAKE, FAKE,  # noqa: E731
-                                       k.get("o", None), None, FAKE, k.get("dA", FAKE), FAKE, FAKE, big, None)
+    bwd = lambda **k: L.lcq_linear_bwd(FAKE, FAKE, FAKE, k.get("P", None), 4, k.get("m", 8), 16, 8, FAKE,  # noqa: E731
+                                       FAKE, k.get("o", None), None, FAKE, k.get("dA", FAKE), FAKE, FAKE, big, None)
+    assert fwd(m=12) != SHAPE                       # the forward takes any output width m
+    assert bwd(m=12) == SHAPE                       # the backward's dY rows are TMA operands: m % 8 == 0
     clipped = lcq.lcq_opts(1.0, 0.0, 1, 0, 0.0, 0.0)
     assert bwd(o=ctypes.byref(clipped)) == NULL     # CLIPPED needs P
     dge = lcq.lcq_opts(1.0, 0.0, 2, 0, 5.0, 3.0)

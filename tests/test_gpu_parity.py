@@ -234,6 +234,9 @@ LINEAR_CASES = [
     # on 76 pairs (152 SMs) every GEMM of this case ends in a partial wave whose tiles run as 256 x 128
     # halves: forward 16 x 5 pair tiles, dX 16 x 16, dW 5 x 16
     (4096, 1280, 4096, 8),
+    # ragged in M, N and K (K tails of 8, 40 and 32) with split last waves in the forward (16 x 5 pair
+    # tiles) and dW (5 x 17)
+    (4000, 1256, 4104, 4),
 ]
 
 
@@ -279,6 +282,31 @@ def test_linear_fwd_bwd_match_oracle(N, m, n, d, ste):
     errs = {"dX": max_rel(host_bf16(dX), g["dX"]), "dP": max_rel(dP.cpu().numpy(), g["dP"]),
             "dA": max_rel(dA.cpu().numpy(), g["dA"]), "db": max_rel(db.cpu().numpy(), g["db"])}
     assert all(e <= TOL_BF16 for e in errs.values()), errs
+
+
+def test_linear_forward_any_output_width():
+    """The forward takes any number of output rows m (here 1250: Y's rows are not 16-byte aligned, so
+    the GEMM epilogue stores them element by element); the backward, whose dY rows are TMA operands,
+    rejects m % 8 != 0 before it enqueues anything."""
+    torch = T()
+    N, m, n, d = 4000, 1250, 4104, 4
+    P, A, b, Xb, dYb = _linear_inputs(N, m, n, d, seed=4242)
+    Z = oracle.quantize(P)
+    Yref = oracle.linear_fwd(wl.bf16_to_f32(Xb), Z, A, b, d)
+    Y = empty_bf16(N, m)
+    packed = torch.empty((m, n // 4), dtype=torch.uint8, device="cuda")
+    wsf = lcq.workspace(lcq.LCQ_OP_LINEAR_FWD, N, m, n, d)
+    lcq.lcq_linear_fwd(dev_bf16(Xb), dev(P), d, dev(A), dev(b), Y, wsf, packed_saved=packed)
+    assert lcq.lcq_device_status(wsf) == 0
+    assert np.array_equal(packed.cpu().numpy(), oracle.pack2b(Z))
+    assert max_rel(host_bf16(Y), Yref) <= TOL_BF16
+    wsb = lcq.workspace(lcq.LCQ_OP_LINEAR_BWD, N, m, n, d)
+    dP = torch.empty((m, n), dtype=torch.float32, device="cuda")
+    dA = torch.empty((d, d), dtype=torch.float32, device="cuda")
+    db = torch.empty(d, dtype=torch.float32, device="cuda")
+    with pytest.raises(lcq.LCQError) as e:
+        lcq.lcq_linear_bwd(dev_bf16(Xb), dev_bf16(dYb), packed, m, n, d, dev(A), dev(b), dP, dA, db, wsb)
+    assert e.value.status == 2                     # LCQ_ERR_SHAPE
 
 
 def test_linear_backward_is_bitwise_reproducible():
