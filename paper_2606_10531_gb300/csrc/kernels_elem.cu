@@ -6,22 +6,27 @@
 //   reduce_partials  fixed-order sum of per-CTA dA/db partials
 //
 // encode and quant_decode stream their fp32 input through a shared-memory ring
-// filled by the bulk-copy (TMA) engine: one producer thread issues 22 KB
+// filled by the bulk-copy (TMA) engine: one producer thread issues 33 KB
 // cp.async.bulk copies, eleven compute warps consume them. In encode, thread t takes
 // the groups t, t + T, ... of a chunk (conflict-free shared-memory reads); in quant_decode
-// each compute thread owns 16 consecutive weights, i.e. whole groups for d = 4 and 8.
+// each compute thread owns 24 consecutive weights, i.e. whole groups for d = 4 and 8.
 #include "common.cuh"
 #include "internal.h"
 #include "invert.cuh"
 
 namespace lcq {
 
+// Encode is bound by its FMA-pipe issue at three warps per SM sub-partition (four would cap the
+// registers at 128): three groups of 8 weights per thread and stage measured faster than two
+// (encode with the MSE 0.722 against 0.750 ms on the Llama-3-70B layer) and than four, and so did
+// these warps against 15 compute warps at one or two groups each.
 constexpr int kComputeWarps = 11;                                // + 1 producer = 12 warps, 3 per SM sub-partition
-constexpr int kPerThread = 16;                                   // weights per compute thread per stage
-constexpr int kChunk = 32 * kComputeWarps * kPerThread;          // fp32 weights per stage (22 KB)
-constexpr int kStreamStages = 8;                                 // 176 KB ring (single-matrix kernels)
-constexpr int kBatchStages = 6;                                  // 132 KB ring (batched encode)
+constexpr int kPerThread = 24;                                   // weights per compute thread per stage
+constexpr int kChunk = 32 * kComputeWarps * kPerThread;          // fp32 weights per stage (33 KB)
+constexpr int kStreamStages = 6;                                 // 198 KB ring (single-matrix kernels)
+constexpr int kBatchStages = 5;                                  // 165 KB ring (batched encode)
 constexpr int kStreamThreads = 32 * (1 + kComputeWarps);
+static_assert(kPerThread % 8 == 0, "a compute thread's weights are whole 8-weight groups (16-byte stores)");
 constexpr float kRoundMagic = 12582912.0f;                       // 1.5 * 2^23
 
 struct StreamSmem {
@@ -338,9 +343,9 @@ __device__ __forceinline__ int batch_item_of(const EncodeBatchArgs &a, int64_t c
 }
 
 // One matrix of a batched encode, for one CTA: its constants and its chunks (the sequence the
-// producer streams). Kept out of line so that its loop is compiled on its own (measured faster).
+// producer streams).
 template <int D, bool kLatent>
-__device__ __noinline__ void encode_batch_matrix(EncBatchSmem &s, const EncodeBatchArgs &a, int j, int &it, bool &ok) {
+__device__ __forceinline__ void encode_batch_matrix(EncBatchSmem &s, const EncodeBatchArgs &a, int j, int &it, bool &ok) {
     const int lane = threadIdx.x & 31;
     const int t = threadIdx.x - 32;
     const int hswap = (D == 8) ? ((t >> 2) & 1) : 0;
@@ -489,17 +494,23 @@ quant_decode_kernel(QuantDecodeArgs a) {
             }
             const int64_t gidx = base + off;
             if (valid == kPerThread) {
+                // gidx is a multiple of 8 (kChunk and kPerThread are): 16-bit words of packed codes at
+                // an even byte offset, 16-byte runs of bf16
                 if (a.packed) {
-                    uint32_t p = 0;
+                    uint16_t *pk = reinterpret_cast<uint16_t *>(a.packed + gidx / 4);
 #pragma unroll
-                    for (int k = 0; k < kPerThread; ++k) p |= z[k] << (2 * k);
-                    *reinterpret_cast<uint32_t *>(a.packed + gidx / 4) = p;
+                    for (int h = 0; h < kPerThread / 8; ++h) {
+                        uint32_t p = 0;
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) p |= z[8 * h + k] << (2 * k);
+                        pk[h] = static_cast<uint16_t>(p);
+                    }
                 }
                 uint4 *dst = reinterpret_cast<uint4 *>(a.W_hat + gidx);
-                dst[0] = make_uint4(pack_bf16x2(wh[0], wh[1]), pack_bf16x2(wh[2], wh[3]), pack_bf16x2(wh[4], wh[5]),
-                                    pack_bf16x2(wh[6], wh[7]));
-                dst[1] = make_uint4(pack_bf16x2(wh[8], wh[9]), pack_bf16x2(wh[10], wh[11]),
-                                    pack_bf16x2(wh[12], wh[13]), pack_bf16x2(wh[14], wh[15]));
+#pragma unroll
+                for (int q = 0; q < kPerThread / 8; ++q)
+                    dst[q] = make_uint4(pack_bf16x2(wh[8 * q], wh[8 * q + 1]), pack_bf16x2(wh[8 * q + 2], wh[8 * q + 3]),
+                                        pack_bf16x2(wh[8 * q + 4], wh[8 * q + 5]), pack_bf16x2(wh[8 * q + 6], wh[8 * q + 7]));
             } else {
 #pragma unroll
                 for (int k = 0; k < kPerThread; k += 4) {
@@ -722,7 +733,7 @@ cudaError_t launch_wait_timeout_selftest(int32_t *status, cudaStream_t st) {
 
 static int stream_grid(int64_t total, int num_sms) {
     const int64_t nchunks = (total + kChunk - 1) / kChunk;
-    int64_t g = num_sms;   // persistent: one CTA (a 176 KB ring) per SM
+    int64_t g = num_sms;   // persistent: one CTA (a 198 KB ring) per SM
     if (nchunks < g) g = nchunks;
     return static_cast<int>(g < 1 ? 1 : g);
 }
