@@ -46,11 +46,13 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true", help="skip the separate encode / packed-product timings")
-    ap.add_argument("--case", choices=["linear", "encode", "gemv", "ldlq", "ldlq70", "ldl_factor", "xform"],
+    ap.add_argument("--case", choices=["linear", "encode", "gemv", "gemv_hadamard", "ldlq", "ldlq70", "ldl_factor",
+                                       "xform"],
                     default=None,
                     help="profiling: run one call in a loop (warmup + steps iterations) and exit; "
                          "linear = fwd+bwd of the 16384 x 4096 x 4096 q projection, encode = 70B gate "
-                         "28672 x 8192, gemv = 70B gate at --tokens tokens, ldlq = LDLQ sweep of a "
+                         "28672 x 8192, gemv = 70B gate at --tokens tokens, gemv_hadamard = the same with "
+                         "the online rotation, ldlq = LDLQ sweep of a "
                          "9728 x 4096 slice of the 8B gate (one wave, small case), ldlq70 = LDLQ sweep of "
                          "the 70B gate 28672 x 8192, ldl_factor = factorisation of its 8192 x 8192 proxy "
                          "Hessian, xform = activation transform of the q projection's 16384 x 4096 "
@@ -298,33 +300,35 @@ def time_gemv_70b(torch, lcq, wl, seed, device, pk):
         nbytes = mx0.m * mx0.n / 4 + 2 * B * mx0.n + 2 * B * mx0.m
         out[f"B{B}"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
                         "bytes": nbytes, "eager_us_l2_flushed": statistics.median(eager) * 1e6}
-    # the paper's deployment path: online Hadamard rotation of the activations, then the product (1 token)
-    X = wl.torch_X(torch, wl.llama3_70b_gate_decode(1)[0], seed + 2000, 1, device)
-    Y = torch.empty((1, mx0.m), dtype=torch.bfloat16, device=device)
-    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, 1, mx0.m, mx0.n, mx0.d, device)
-    for c in range(ncopies):
-        lcq.lcq_gemm_packed2b_hadamard(X, packs[c], mx0.n, mx0.d, A, b, Y, ws)
-    torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        for i in range(calls):
-            lcq.lcq_gemm_packed2b_hadamard(X, packs[i % ncopies], mx0.n, mx0.d, A, b, Y, ws)
-    graph.replay()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(replays):
+    # the paper's deployment path: online Hadamard rotation of the activations, then the product (the
+    # rotation runs inside the product: the one-token kernel's prologue, the tcgen05 kernel's prep)
+    for B in (1, 16):
+        X = wl.torch_X(torch, wl.llama3_70b_gate_decode(B)[0], seed + 2000, B, device)
+        Y = torch.empty((B, mx0.m), dtype=torch.bfloat16, device=device)
+        ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, B, mx0.m, mx0.n, mx0.d, device)
+        for c in range(ncopies):
+            lcq.lcq_gemm_packed2b_hadamard(X, packs[c], mx0.n, mx0.d, A, b, Y, ws)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for i in range(calls):
+                lcq.lcq_gemm_packed2b_hadamard(X, packs[i % ncopies], mx0.n, mx0.d, A, b, Y, ws)
         graph.replay()
-    e1.record()
-    torch.cuda.synchronize()
-    t = e0.elapsed_time(e1) * 1e-3 / (replays * calls)
-    nbytes = mx0.m * mx0.n / 4 + 2 * mx0.n + 2 * mx0.m
-    out["B1_hadamard"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
-                          "bytes": nbytes}
-    assert lcq.lcq_device_status(ws) == 0
-    del graph
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(replays):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        t = e0.elapsed_time(e1) * 1e-3 / (replays * calls)
+        nbytes = mx0.m * mx0.n / 4 + 2 * B * mx0.n + 2 * B * mx0.m
+        out[f"B{B}_hadamard"] = {"us": t * 1e6, "GB/s": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / pk["hbm"],
+                                 "bytes": nbytes}
+        assert lcq.lcq_device_status(ws) == 0
+        del graph
     out["workload"] = ("llama3-70b gate 28672x8192 packed 2-bit, d=8, bf16 activations; CUDA-graph replay of 24 "
-                       "calls over 6 code copies (352 MB > L2); B1_hadamard adds the online rotation")
+                       "calls over 6 code copies (352 MB > L2); B1_hadamard and B16_hadamard add the online rotation")
     return out
 
 
@@ -635,7 +639,7 @@ def summary(line):
         out["encode70b_codes_only_frac_hbm"] = r3(enc["codes_only"]["frac_hbm"])
     pd = line.get("packed_decode")
     if pd:
-        for k in ("B1", "B2", "B4", "B16", "B1_hadamard"):
+        for k in ("B1", "B2", "B4", "B16", "B1_hadamard", "B16_hadamard"):
             if k in pd:
                 out[f"packed_{k}_us"] = r3(pd[k]["us"])
                 out[f"packed_{k}_frac_hbm"] = r3(pd[k]["frac_hbm"])
@@ -810,8 +814,14 @@ def profile_case(args):
         Y = torch.empty((mx.N, mx.m), dtype=torch.bfloat16, device=device)
         ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B, mx.N, mx.m, mx.n, mx.d, device)
 
-        def run():
-            lcq.lcq_gemm_packed2b(X, packed, mx.n, mx.d, A, b, Y, ws)
+        if args.case == "gemv_hadamard":
+            ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, mx.N, mx.m, mx.n, mx.d, device)
+
+            def run():
+                lcq.lcq_gemm_packed2b_hadamard(X, packed, mx.n, mx.d, A, b, Y, ws)
+        else:
+            def run():
+                lcq.lcq_gemm_packed2b(X, packed, mx.n, mx.d, A, b, Y, ws)
         wss = [ws]
     for _ in range(args.warmup + args.steps):
         run()

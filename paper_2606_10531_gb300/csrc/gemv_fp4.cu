@@ -228,11 +228,125 @@ __device__ __forceinline__ void f4_load16(const void *__restrict__ Xv, int64_t n
     }
 }
 
-template <int D, bool F32IN>
+// Element e of the row sits in shared memory at word e ^ (((e >> 5) & 3) << 2): the 16-byte chunks of
+// each 64-byte group are permuted by bits 5-6 of the index, so that the 16-byte stores and loads of a
+// quarter warp, whose threads hold 16 consecutive elements each, fall on eight distinct 4-bank groups.
+__device__ __forceinline__ int64_t f4_swz(int64_t e) { return e ^ (((e >> 5) & 3) << 2); }
+
+// Radix-K butterflies of the Walsh-Hadamard transform over index bits [bit0, bit0 + log2 K) of the
+// row in shared memory: each thread takes the K elements of a group that differ only in those bits.
+// Consecutive threads take consecutive low indices (bit0 >= 9), so a warp's accesses hit 32 banks (the
+// permutation above moves words within aligned runs of 32; bits >= bit0 leave it unchanged).
+template <int K>
+__device__ __forceinline__ void f4_wht_pass(float *buf, int64_t n, int bit0) {
+    const int64_t groups = n / K;
+    const int64_t low = (int64_t(1) << bit0) - 1;
+    for (int64_t g = threadIdx.x; g < groups; g += kF4PrepThreads) {
+        const int64_t base = f4_swz((g & low) | ((g >> bit0) << bit0) * K);
+        float y[K];
+#pragma unroll
+        for (int k = 0; k < K; ++k) y[k] = buf[base + (static_cast<int64_t>(k) << bit0)];
+#pragma unroll
+        for (int h = 1; h < K; h <<= 1)
+#pragma unroll
+            for (int k = 0; k < K; ++k)
+                if ((k & h) == 0) {
+                    const float u = y[k], v = y[k + h];
+                    y[k] = u + v;
+                    y[k + h] = u - v;
+                }
+#pragma unroll
+        for (int k = 0; k < K; ++k) buf[base + (static_cast<int64_t>(k) << bit0)] = y[k];
+    }
+}
+
+// Normalized block Walsh-Hadamard rotation of one token's row (the online rotation of the rotated
+// deployment product, Sec. 2.2 / App. Inference Speed) on the prep layout: column (threadIdx.x + 512 gg)
+// * 16 + i sits in x[gg][i]. The block is 2^lb columns (6 <= lb <= 15, the largest power of two dividing
+// n), so the transform factors over index bits 0 .. lb-1, one butterfly stage (u, v) -> (u + v, u - v)
+// per bit, in any order: bits 0-3 in registers, bits 4-8 (the lane) by warp shuffles, bits 9 .. lb-1
+// (warp and gg) through the row in shared memory (n floats, permuted as f4_swz states), up to four bits
+// per pass. A column's partner in a bit below lb lies in its own block, so columns past the row's end
+// never feed real ones. The result is scaled by 2^(-lb/2).
+__device__ __forceinline__ void f4_rotate(float (&x)[kF4PrepGroups][16], int64_t n, int lb, float *buf) {
+    const int ngg = static_cast<int>((n / 16 + kF4PrepThreads - 1) / kF4PrepThreads);
+#pragma unroll
+    for (int gg = 0; gg < kF4PrepGroups; ++gg) {
+        if (gg >= ngg) continue;
+#pragma unroll
+        for (int h = 1; h < 16; h <<= 1)
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if ((i & h) == 0) {
+                    const float u = x[gg][i], v = x[gg][i + h];
+                    x[gg][i] = u + v;
+                    x[gg][i + h] = u - v;
+                }
+    }
+    const int lane = threadIdx.x & 31;
+    const int hmax = lb >= 9 ? 32 : 1 << (lb - 4);   // lane bit h is column bit 4 + log2 h
+#pragma unroll
+    for (int h = 1; h < 32; h <<= 1) {
+        if (h >= hmax) break;
+        const bool hi = (lane & h) != 0;
+#pragma unroll
+        for (int gg = 0; gg < kF4PrepGroups; ++gg) {
+            if (gg >= ngg) continue;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const float o = __shfl_xor_sync(0xffffffffu, x[gg][i], h);
+                x[gg][i] = hi ? o - x[gg][i] : x[gg][i] + o;
+            }
+        }
+    }
+    if (lb > 9) {
+#pragma unroll
+        for (int gg = 0; gg < kF4PrepGroups; ++gg) {
+            const int64_t c0 = (threadIdx.x + static_cast<int64_t>(gg) * kF4PrepThreads) * 16;
+            if (c0 >= n) continue;
+            float4 *dst = reinterpret_cast<float4 *>(buf + c0);
+            const int sw = static_cast<int>(c0 >> 5) & 3;   // bits 5-6 of the group's indices
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                dst[q ^ sw] = make_float4(x[gg][4 * q], x[gg][4 * q + 1], x[gg][4 * q + 2], x[gg][4 * q + 3]);
+        }
+        for (int bit0 = 9; bit0 < lb; bit0 += 4) {
+            __syncthreads();
+            switch (lb - bit0) {
+                case 1: f4_wht_pass<2>(buf, n, bit0); break;
+                case 2: f4_wht_pass<4>(buf, n, bit0); break;
+                case 3: f4_wht_pass<8>(buf, n, bit0); break;
+                default: f4_wht_pass<16>(buf, n, bit0); break;
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int gg = 0; gg < kF4PrepGroups; ++gg) {
+            const int64_t c0 = (threadIdx.x + static_cast<int64_t>(gg) * kF4PrepThreads) * 16;
+            if (c0 >= n) continue;
+            const float4 *src = reinterpret_cast<const float4 *>(buf + c0);
+            const int sw = static_cast<int>(c0 >> 5) & 3;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float4 f = src[q ^ sw];
+                x[gg][4 * q] = f.x; x[gg][4 * q + 1] = f.y; x[gg][4 * q + 2] = f.z; x[gg][4 * q + 3] = f.w;
+            }
+        }
+    }
+    const float s = rsqrtf(static_cast<float>(1 << lb));
+#pragma unroll
+    for (int gg = 0; gg < kF4PrepGroups; ++gg)
+#pragma unroll
+        for (int i = 0; i < 16; ++i) x[gg][i] *= s;
+}
+
+// ROT: rotate the token's bf16 row by the block Walsh-Hadamard transform of block 2^lb first (dynamic
+// shared memory: n floats when lb > 9).
+template <int D, bool F32IN, bool ROT>
 __global__ void __launch_bounds__(kF4PrepThreads)
 fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int NB, const float *__restrict__ A,
                 const float *__restrict__ b, uint8_t *__restrict__ dig, float *__restrict__ scale,
-                float *__restrict__ corr) {
+                float *__restrict__ corr, int lb) {
     // the main kernel may start streaming codes right away; it waits for these results itself
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float sA[D * D], sb[D];
@@ -252,6 +366,14 @@ fp4_prep_kernel(const void *__restrict__ Xv, int64_t n, int tiles, int ntok, int
     for (int gg = 0; gg < kF4PrepGroups; ++gg) {
         const int64_t gi = threadIdx.x + static_cast<int64_t>(gg) * kF4PrepThreads;
         if (gi < ngroups) f4_load16<D, F32IN>(Xv, n, t, gi * 16, xv[gg]);
+        else if (ROT) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) xv[gg][i] = 0.0f;
+        }
+    }
+    if (ROT) {
+        extern __shared__ __align__(16) float rot_buf[];
+        f4_rotate(xv, n, lb, rot_buf);
     }
     __syncthreads();
 
@@ -725,16 +847,28 @@ bool launch_packed_gemv_fp4(const PackedGemvArgs &a, int d, int num_sms, cudaStr
         return true;
     }
     using PrepFn = void (*)(const void *, int64_t, int, int, int, const float *, const float *, uint8_t *, float *,
-                            float *);
-    PrepFn prep = a.Xf ? (d == 4 ? fp4_prep_kernel<4, true> : fp4_prep_kernel<8, true>)
-                       : (d == 4 ? fp4_prep_kernel<4, false> : fp4_prep_kernel<8, false>);
+                            float *, int);
+    PrepFn prep = a.rotate ? (d == 4 ? fp4_prep_kernel<4, false, true> : fp4_prep_kernel<8, false, true>)
+                  : a.Xf   ? (d == 4 ? fp4_prep_kernel<4, true, false> : fp4_prep_kernel<8, true, false>)
+                           : (d == 4 ? fp4_prep_kernel<4, false, false> : fp4_prep_kernel<8, false, false>);
+    int lb = 0;
+    size_t prep_smem = 0;
+    if (a.rotate) {
+        // n % 64 == 0 and n <= 32768 (the plan), so the block is 2^6 .. 2^15 columns
+        while ((a.n >> (lb + 1)) << (lb + 1) == a.n && lb < 15) ++lb;
+        prep_smem = lb > 9 ? static_cast<size_t>(a.n) * sizeof(float) : 0;
+        if (prep_smem) {
+            err = ensure_dynamic_smem(reinterpret_cast<const void *>(prep), static_cast<int>(prep_smem));
+            if (err != cudaSuccess) return true;
+        }
+    }
     {
         // a programmatic dependent of the previous kernel in the stream: it may become resident on the
         // SMs this kernel's grid leaves free while that kernel still runs, and waits for it on the device
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(static_cast<unsigned>(a.N));
         cfg.blockDim = dim3(kF4PrepThreads);
-        cfg.dynamicSmemBytes = 0;
+        cfg.dynamicSmemBytes = prep_smem;
         cfg.stream = st;
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -742,7 +876,7 @@ bool launch_packed_gemv_fp4(const PackedGemvArgs &a, int d, int num_sms, cudaStr
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         err = cudaLaunchKernelEx(&cfg, prep, a.Xf ? static_cast<const void *>(a.Xf) : static_cast<const void *>(a.X),
-                                 a.n, pl.tiles, static_cast<int>(a.N), pl.NB, a.A, a.b, dig, scale, corr);
+                                 a.n, pl.tiles, static_cast<int>(a.N), pl.NB, a.A, a.b, dig, scale, corr, lb);
         count_launch();
         if (err == cudaSuccess) err = cudaGetLastError();
         if (err != cudaSuccess) return true;

@@ -1293,15 +1293,25 @@ static cudaError_t launch_packed_gemv_dp(const PackedGemvArgs &a, int d, int num
 
 bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err) {
     err = cudaSuccess;
-    if (!(a.n % 64 == 0 && a.n <= kDpMaxN && a.m >= 16 && a.N == kDpMaxTokens)) return false;
     PackedGemvArgs r = a;
     r.rotate = true;
     r.Xf = nullptr;
     int R, stages, nkc, hb;
-    if (!dp_plan(r, num_sms, R, stages, nkc, hb)) return false;
-    bool done = false;
+    if (a.n % 64 == 0 && a.n <= kDpMaxN && a.m >= 16 && a.N == kDpMaxTokens && dp_plan(r, num_sms, R, stages, nkc, hb)) {
+        // one token: the rotation runs in the dp kernel's prologue
+        bool done = false;
+        trace_begin(LCQ_K_GEMV, st);
+        err = launch_packed_gemv_dp(r, d, num_sms, st, done);
+        if (err == cudaSuccess) {
+            trace_end(LCQ_K_GEMV, st);
+            err = cudaGetLastError();
+        }
+        return true;
+    }
+    // 1-16 tokens, n % 64 == 0, n <= 32768: the rotation runs in the tcgen05 kernel's prep kernel (a
+    // begin mark left when that kernel does not apply is overwritten by the next one)
     trace_begin(LCQ_K_GEMV, st);
-    err = launch_packed_gemv_dp(r, d, num_sms, st, done);
+    if (!launch_packed_gemv_fp4(r, d, num_sms, st, err)) return false;
     if (err == cudaSuccess) {
         trace_end(LCQ_K_GEMV, st);
         err = cudaGetLastError();

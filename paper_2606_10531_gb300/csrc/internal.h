@@ -185,8 +185,9 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
 // error otherwise.
 size_t packed_gemv_fp4_workspace(int64_t N, int64_t n);
 bool launch_packed_gemv_fp4(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err);
-// The rotated product with the rotation in the one-token kernel's prologue. Returns false (nothing
-// launched) when that kernel does not apply; err holds a launch error otherwise.
+// The rotated product with the rotation inside the product: in the one-token kernel's prologue, else
+// in the tcgen05 kernel's prep kernel (1-16 tokens). Returns false (nothing launched) when neither
+// applies; err holds a launch error otherwise.
 bool launch_packed_gemv_rotated(const PackedGemvArgs &a, int d, int num_sms, cudaStream_t st, cudaError_t &err);
 // Row-wise normalized block Walsh-Hadamard rotation (block = largest power of two dividing n, <= 32768).
 int hadamard_block_size(int64_t n);

@@ -303,7 +303,8 @@ lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_
     float *Xr = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kHeader);
     uint8_t *base = static_cast<uint8_t *>(ws) + kHeader + align256(static_cast<size_t>(N) * static_cast<size_t>(n) * 4);
     {
-        // one token: the rotation runs in the product kernel's prologue
+        // the rotation runs inside the product (the one-token kernel's prologue or the tcgen05
+        // kernel's prep) where one of those kernels takes the shape
         PackedGemvArgs a;
         a.X = X; a.Xf = nullptr; a.N = N; a.m = m; a.n = n; a.packed = packed; a.A = A; a.b = b; a.Y = Y;
         a.Xp = reinterpret_cast<uint16_t *>(base);

@@ -568,6 +568,36 @@ def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
     assert max_rel(host_bf16(Y), ref) <= TOL_BF16
 
 
+# 1-16 tokens with n % 64 == 0 and n <= 32768 (but one token at n = 8192): the rotation runs in the
+# tcgen05 kernel's prep kernel, so the call is two launches (prep and product) and no rotation kernel.
+# The rotated activations then take the digit path, so each output is held to digit_product_bound of
+# the rotated X. Rotation blocks: 2^6 (n = 576, lanes only), 2^9 (n = 512, every bit in registers or
+# shuffles), 2^11 (n = 14336, one shared-memory pass), 2^13 in three blocks (n = 24576), 2^15 (n =
+# 32768, two passes).
+@pytest.mark.parametrize("N", [1, 2, 7, 16])
+@pytest.mark.parametrize("m,n,d", [(300, 576, 8), (129, 512, 4), (1000, 14336, 8), (77, 24576, 4), (260, 32768, 8),
+                                   (513, 8192, 8)])
+def test_gemm_packed2b_hadamard_tcgen05_prep(N, m, n, d):
+    if N == 1 and n == 8192:
+        pytest.skip("one token at n = 8192 rotates in the one-token kernel (test above)")
+    rng = np.random.default_rng(13 * N + m + n + d)
+    Z = rng.integers(0, 4, (m, n)).astype(np.uint8)
+    A, b = config_A(d, rng), config_b(d, rng)
+    X = rng.normal(0, 1, (N, n))
+    X[:, rng.random(n) < 0.01] *= 50.0
+    Xb = wl.bf16_bits(X.astype(np.float32))
+    Xf = wl.bf16_to_f32(Xb)
+    ref = oracle.gemm_packed2b_hadamard(Xf, oracle.pack2b(Z), A, b, d, n)
+    Y = empty_bf16(N, m)
+    ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)
+    before = lcq.lcq_launch_count()
+    lcq.lcq_gemm_packed2b_hadamard(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
+    assert lcq.lcq_launch_count() - before == 2
+    assert lcq.lcq_device_status(ws) == 0
+    bound = digit_product_bound(oracle.hadamard_rotate(Xf, n), Z, A, b, d, ref)
+    assert within(host_bf16(Y), ref, bound) <= 1.0
+
+
 # 2-16 tokens with n % 64 == 0 take the tcgen05 kernel (kind::mxf4): the codes are fp4 operands in
 # tensor memory and the activations exact integer digits, q = rint(X' 8191 / max|X'_t|) per token, so
 # its only errors are that rounding (at most 2^-14 of max|X'_t| per element) and the bf16 output
