@@ -327,7 +327,10 @@ lcq_status lcq_hadamard(const float *in, int64_t rows, int64_t n, float *out, vo
  * (App. Inference Speed: Hadamard transform, then the fused affine-dequant product):
  *   Y = (X H) W_hat^T, with the codes encoding the rotated weights W H (see lcq_hadamard).
  * Arguments as lcq_gemm_packed2b; needs lcq_workspace_size(LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d).
- * The rotated activations are kept in fp32.
+ * The rotated activations are kept in fp32. The rotation runs inside the product where a product
+ * kernel takes the shape: one token at n = 8192 in the one-token kernel's prologue, 1-16 tokens with
+ * n % 64 == 0 and n <= 32768 in the tcgen05 kernel's prep (two launches per call); other shapes rotate
+ * into the workspace in a kernel of their own first.
  */
 lcq_status lcq_gemm_packed2b_hadamard(const uint16_t *X, int64_t N, const uint8_t *packed, int64_t m, int64_t n,
                                       int d, const float *A, const float *b, uint16_t *Y,

@@ -288,14 +288,15 @@ __device__ __forceinline__ void f4_rotate(float (&x)[kF4PrepGroups][16], int64_t
 #pragma unroll
     for (int h = 1; h < 32; h <<= 1) {
         if (h >= hmax) break;
-        const bool hi = (lane & h) != 0;
+        // the upper lane of a pair forms o - x, the lower x + o: one fma by -1 or 1 (exact, one rounding)
+        const float sgn = (lane & h) ? -1.0f : 1.0f;
 #pragma unroll
         for (int gg = 0; gg < kF4PrepGroups; ++gg) {
             if (gg >= ngg) continue;
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
                 const float o = __shfl_xor_sync(0xffffffffu, x[gg][i], h);
-                x[gg][i] = hi ? o - x[gg][i] : x[gg][i] + o;
+                x[gg][i] = fmaf(sgn, x[gg][i], o);
             }
         }
     }
