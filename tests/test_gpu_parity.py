@@ -586,15 +586,15 @@ def test_gemm_packed2b_hadamard_tcgen05_prep(N, m, n, d):
     X = rng.normal(0, 1, (N, n))
     X[:, rng.random(n) < 0.01] *= 50.0
     Xb = wl.bf16_bits(X.astype(np.float32))
-    Xf = wl.bf16_to_f32(Xb)
-    ref = oracle.gemm_packed2b_hadamard(Xf, oracle.pack2b(Z), A, b, d, n)
+    Xr = oracle.hadamard_rotate(wl.bf16_to_f32(Xb), n)      # rotated once: reference and bound
+    ref = oracle.gemm_packed2b(Xr, oracle.pack2b(Z), A, b, d, n)   # = gemm_packed2b_hadamard(X)
     Y = empty_bf16(N, m)
     ws = lcq.workspace(lcq.LCQ_OP_GEMM_PACKED2B_HADAMARD, N, m, n, d)
     before = lcq.lcq_launch_count()
     lcq.lcq_gemm_packed2b_hadamard(dev_bf16(Xb), dev(oracle.pack2b(Z)), n, d, dev(A), dev(b), Y, ws)
     assert lcq.lcq_launch_count() - before == 2
     assert lcq.lcq_device_status(ws) == 0
-    bound = digit_product_bound(oracle.hadamard_rotate(Xf, n), Z, A, b, d, ref)
+    bound = digit_product_bound(Xr, Z, A, b, d, ref)
     assert within(host_bf16(Y), ref, bound) <= 1.0
 
 
