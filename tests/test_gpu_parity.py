@@ -572,11 +572,11 @@ def test_gemm_packed2b_hadamard_matches_oracle(N, m, n, d):
 # tcgen05 kernel's prep kernel, so the call is two launches (prep and product) and no rotation kernel.
 # The rotated activations then take the digit path, so each output is held to digit_product_bound of
 # the rotated X. Rotation blocks: 2^6 (n = 576, lanes only), 2^9 (n = 512, every bit in registers or
-# shuffles), 2^11 (n = 14336, one shared-memory pass), 2^13 in three blocks (n = 24576), 2^15 (n =
-# 32768, two passes).
+# shuffles), then one shared-memory pass of 2, 4, 8 or 16 points (n = 3072, 14336, 4096, and 2^13 in
+# three blocks at n = 24576) or two passes (16 + 2 points at n = 16384, 16 + 4 at n = 32768).
 @pytest.mark.parametrize("N", [1, 2, 7, 16])
 @pytest.mark.parametrize("m,n,d", [(300, 576, 8), (129, 512, 4), (1000, 14336, 8), (77, 24576, 4), (260, 32768, 8),
-                                   (513, 8192, 8)])
+                                   (513, 8192, 8), (90, 3072, 8), (140, 4096, 4), (64, 16384, 8)])
 def test_gemm_packed2b_hadamard_tcgen05_prep(N, m, n, d):
     if N == 1 and n == 8192:
         pytest.skip("one token at n = 8192 rotates in the one-token kernel (test above)")
