@@ -191,7 +191,8 @@ __host__ __device__ inline void f4_range(int r, int slices, int ranges, int &s0,
 // thread turns its values into q = rint(X' * 8191 / max) and the five digits, stored as e2m1 nibbles
 // in the MMA's K order: within 16 columns, K position 8 p + i carries column 2 i + p (the order the
 // code expansion produces). Digit row t * 5 + j of tile k is 256 bytes at dig[(k * NB + t * 5 + j) *
-// 256]; the last token's CTA also zeroes rows 5 ntok .. NB - 1.
+// 256]; the last token's CTA also zeroes rows 5 ntok .. NB - 1. With the online rotation (ROT), the
+// token's row is rotated by the block Walsh-Hadamard transform first, in this same layout (f4_rotate).
 
 constexpr int kF4PrepThreads = 512;
 constexpr int kF4PrepGroups = 4;           // groups of 16 columns per thread: n <= 32768

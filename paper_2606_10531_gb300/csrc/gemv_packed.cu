@@ -1325,7 +1325,7 @@ cudaError_t launch_packed_gemv(const PackedGemvArgs &a, int d, int num_sms, cuda
     if (a.N > kFp4MinTokens) {
         // 2-16 tokens, n % 64 == 0, n <= 32768: codes as fp4 tensor-core operands in tensor memory
         // (tcgen05); faster than the mma.sync kernel below at every token count from 2 (70B gate:
-        // 17.2-18.0 against 18.4-18.6 us at 2-8 tokens), which keeps the other shapes
+        // 14.5-14.9 against 18.4-18.6 us at 2-8 tokens), which keeps the other shapes
         cudaError_t e = cudaSuccess;
         if (launch_packed_gemv_fp4(a, d, num_sms, st, e)) {
             if (e != cudaSuccess) return e;
