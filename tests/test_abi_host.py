@@ -141,6 +141,65 @@ def test_encode_batch_validation(L):
     assert 0 < L.lcq_workspace_size(6, 1, 0, 0, 8) < L.lcq_workspace_size(6, 7, 0, 0, 8)
 
 
+def test_rotation_transform_ldlq_and_init_validation(L):
+    big = 1 << 30
+    assert L.lcq_hadamard(FAKE, 2, 12, FAKE, None) == SHAPE          # n % 8 != 0
+    assert L.lcq_hadamard(None, 0, 16, None, None) == OK             # empty: no device
+    assert L.lcq_hadamard(None, 2, 16, FAKE, None) == NULL
+    assert L.lcq_hadamard(FAKE + 4, 2, 16, FAKE, None) == ALIGN
+
+    def gh(X=FAKE, N=2, n=64, d=8, A=FAKE, ws=FAKE, ws_bytes=big):
+        return L.lcq_gemm_packed2b_hadamard(X, N, FAKE, 8, n, d, A, FAKE, FAKE, ws, ws_bytes, None)
+    assert gh(d=5) == UNSUP
+    assert gh(N=-1) == SHAPE
+    assert gh(n=60) == SHAPE
+    assert gh(X=None) == NULL
+    assert gh(A=None) == NULL
+    assert gh(ws_bytes=16) == WS
+    assert gh(ws=FAKE + 16) == ALIGN                                 # workspace must be 256-byte aligned
+
+    def xf(N=4, n=64, d=8, A=FAKE, Xp=FAKE, r=FAKE):
+        return L.lcq_activation_transform(FAKE, N, n, d, A, FAKE, Xp, r, None)
+    assert xf(d=6) == UNSUP
+    assert xf(N=-1) == SHAPE
+    assert xf(N=0) == OK
+    assert xf(Xp=None, r=None) == NULL                              # nothing to write
+    assert xf(r=FAKE + 4) == ALIGN
+    assert xf(A=None) == NULL
+
+    assert L.lcq_ldl_factor(FAKE, 64, 5, FAKE, FAKE, FAKE, big, None) == UNSUP
+    assert L.lcq_ldl_factor(FAKE, 0, 8, FAKE, FAKE, FAKE, big, None) == OK
+    assert L.lcq_ldl_factor(FAKE, 65544, 8, FAKE, FAKE, FAKE, big, None) == SHAPE   # n > 65536
+    assert L.lcq_ldl_factor(None, 64, 8, FAKE, FAKE, FAKE, big, None) == NULL
+    assert L.lcq_ldl_factor(FAKE, 64, 8, FAKE, FAKE, FAKE, 16, None) == WS
+
+    def lq(n=64, A=FAKE, U=FAKE, ws_bytes=big):
+        return L.lcq_ldlq(FAKE, 64, n, 8, A, FAKE, U, FAKE, None, None, None, FAKE, ws_bytes, None)
+    assert lq(n=60) == SHAPE
+    assert lq(U=None) == NULL
+    assert lq(A=None) == NULL
+    assert lq(ws_bytes=16) == WS
+
+    assert L.lcq_init_codebook(FAKE, 6, FAKE, FAKE, None) == UNSUP
+    assert L.lcq_init_codebook(None, 8, FAKE, FAKE, None) == NULL
+    assert L.lcq_init_latent(FAKE, 4, 6, FAKE, None, None, None) == SHAPE   # n % 4 != 0
+    assert L.lcq_init_latent(FAKE, 0, 0, FAKE, None, None, None) == SHAPE
+
+
+@pytest.mark.parametrize("m,n", [(0, 16), (4096, 0), (0, 14336)])
+def test_init_latent_constants_match_the_oracle(L, m, n):
+    """The preprocessing constants of Eq. xavier_preprocess (s = 2a/3, t = 3/2, a = sqrt(6/(m+n))) are
+    computed on the host; for an empty matrix the call returns them without touching a device. s is
+    the oracle's fp64 value rounded to fp32."""
+    import numpy as np
+    import oracle
+    s, t = ctypes.c_float(-1.0), ctypes.c_float(-1.0)
+    assert L.lcq_init_latent(None, m, n, None, ctypes.byref(s), ctypes.byref(t), None) == OK
+    _, s_ref, t_ref = oracle.init_latent(np.zeros((m, n), np.uint8), m, n)
+    assert s.value == float(np.float32(s_ref))
+    assert t.value == t_ref == 1.5
+
+
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(ImportError, match="liblcq.so not found"):
         lcq.load_library(str(tmp_path / "liblcq.so"))
